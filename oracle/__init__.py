@@ -1,0 +1,141 @@
+"""fp64 CPU oracle of the tree-verification pass (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's CPU baseline
+leg import this package.  The product library never does.
+
+``oracle.c`` holds the arithmetic (tree sets, attention, LM head, greedy
+acceptance); this module compiles it with gcc, loads it with ctypes and adds
+the KV compaction, which is a plain gather written out below.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile oracle.c into liboracle.so (gcc, OpenMP, -O2, no fast-math)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        cmd = ["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11", "-o", tmp, _SRC, "-lm"]
+        subprocess.run(cmd, check=True)
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            lib = ctypes.CDLL(_LIB)
+            P = ctypes.c_void_p
+            i32, i64 = ctypes.c_int, ctypes.c_int64
+            lib.oracle_tree.argtypes = [P, i32, P, P]
+            lib.oracle_tree_attention.argtypes = [P, P, P, i64, i32, i32, i32, i32, i32, P, P]
+            lib.oracle_lm_head.argtypes = [P, P, i32, i32, i32, P, P, P, P, P]
+            lib.oracle_accept.argtypes = [P, i32, P, P, P, P, P]
+            lib.oracle_num_threads.argtypes = []
+            for f in (lib.oracle_tree, lib.oracle_tree_attention, lib.oracle_lm_head,
+                      lib.oracle_accept, lib.oracle_num_threads):
+                f.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def num_threads() -> int:
+    return int(_load().oracle_num_threads())
+
+
+def tree(parent):
+    """(depth[n], in_anc[n][n] bool) for a parent array rooted at node 0."""
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    n = len(parent)
+    depth = np.zeros(n, dtype=np.int32)
+    in_anc = np.zeros((n, n), dtype=np.uint8)
+    if _load().oracle_tree(_ptr(parent), n, _ptr(depth), _ptr(in_anc)) != 0:
+        raise ValueError("not a tree rooted at node 0")
+    return depth, in_anc.astype(bool)
+
+
+def tree_attention(q, k, v, L: int, parent, n_kv_heads: int | None = None):
+    """One layer of tree-masked attention.
+
+    q: [N][Hq][d] bf16 bits.  k, v: [Hkv][S][d] bf16 bits with S >= L + N.
+    Returns float64 [N][Hq][d]."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    N, Hq, d = q.shape
+    Hkv = k.shape[0] if n_kv_heads is None else n_kv_heads
+    if k.shape[1] < L + N or k.shape != v.shape or k.shape[2] != d:
+        raise ValueError("bad kv shape")
+    out = np.zeros((N, Hq, d), dtype=np.float64)
+    rc = _load().oracle_tree_attention(_ptr(q), _ptr(k), _ptr(v), k.shape[1] * d, L, N, Hq, Hkv, d,
+                                        _ptr(parent), _ptr(out))
+    if rc != 0:
+        raise ValueError(f"oracle_tree_attention rc={rc}")
+    return out
+
+
+def lm_head(hidden, W, want_logits: bool = False):
+    """(argmax int32[R], top1 f64[R], entropy f64[R], gap f64[R][, logits f64[R][V]])."""
+    hidden = np.ascontiguousarray(hidden, dtype=np.uint16)
+    W = np.ascontiguousarray(W, dtype=np.uint16)
+    R, D = hidden.shape
+    V = W.shape[0]
+    if W.shape[1] != D:
+        raise ValueError("d_model mismatch")
+    argmax = np.zeros(R, dtype=np.int32)
+    top1 = np.zeros(R)
+    ent = np.zeros(R)
+    gap = np.zeros(R)
+    logits = np.zeros((R, V)) if want_logits else None
+    rc = _load().oracle_lm_head(_ptr(hidden), _ptr(W), R, D, V, _ptr(argmax), _ptr(top1), _ptr(ent),
+                                _ptr(gap), _ptr(logits) if want_logits else None)
+    if rc != 0:
+        raise ValueError(f"oracle_lm_head rc={rc}")
+    return (argmax, top1, ent, gap, logits) if want_logits else (argmax, top1, ent, gap)
+
+
+def accept(parent, draft, argmax):
+    """(accept_len, path list, bonus token)."""
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    draft = np.ascontiguousarray(draft, dtype=np.int32)
+    argmax = np.ascontiguousarray(argmax, dtype=np.int32)
+    n = len(parent)
+    path = np.zeros(max(n, 1), dtype=np.int32)
+    alen = np.zeros(1, dtype=np.int32)
+    bonus = np.zeros(1, dtype=np.int32)
+    if _load().oracle_accept(_ptr(parent), n, _ptr(draft), _ptr(argmax), _ptr(alen), _ptr(path),
+                             _ptr(bonus)) != 0:
+        raise ValueError("not a tree rooted at node 0")
+    k = int(alen[0])
+    return k, [int(x) for x in path[:k]], int(bonus[0])
+
+
+def kv_compact(cache, L: int, path):
+    """KV-cache update after acceptance: slot L + j takes the contents of slot
+    L + path[j] for j < len(path); every other slot is unchanged.
+
+    cache: [..., S, d] (any dtype).  Returns a new array; reads only the old one."""
+    old = np.asarray(cache)
+    new = old.copy()
+    for j, src in enumerate(path):
+        new[..., L + j, :] = old[..., L + src, :]
+    return new

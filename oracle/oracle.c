@@ -1,0 +1,253 @@
+/*
+ * oracle.c -- plain fp64 CPU reference of the per-step tree-verification pass
+ * of Medusa/Hydra multi-token-prediction decoding (EntMTP, Sec. 2.3, 3.2, 4).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product library links, loads or
+ * calls this file; only the tests, the smoke check and the benchmark's CPU
+ * baseline leg do.  It shares no code, header or table with the CUDA path.
+ *
+ * Every routine is the plain definition of what the verification pass
+ * computes, evaluated in double precision from the same bf16 inputs that the
+ * GPU sees.  No blocking, fusion or reordering beyond the definition; the only
+ * parallelism is an OpenMP loop over independent outputs.
+ *
+ *   tree           anc(i) = {i} U anc(parent(i)), depth(root) = 0
+ *                  (the precompiled tree masks / position offsets, Sec. 1, 2.3)
+ *   attention      node i attends to the whole prefix [0, L) and to the tree
+ *                  slots L + j of its ancestors-or-self j (tree decoding, Sec. 3.2)
+ *   LM head        z = W h; greedy token argmax z (lowest index on ties);
+ *                  p = softmax(z); top-1 probability max p (the p0 of Sec. 4);
+ *                  entropy -sum p ln p in nats
+ *   acceptance     node i is accepted when every non-root node j on its root
+ *                  path carries the draft token that the target model would
+ *                  emit greedily after j's parent: draft[j] == argmax[parent(j)].
+ *                  The accepted path ends at the deepest accepted node (smallest
+ *                  index among equally deep ones); accept_len = depth + 1 counts
+ *                  the accepted drafts plus the bonus token argmax[j*]
+ *                  (greedy form of the verification step, Sec. 3.2 / 5.1 tau).
+ *
+ * Pinned by tests/test_oracle_pins.py against independent references
+ * (torch float64 attention, brute-force path enumeration, closed forms).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORACLE_MAX_NODES 64
+
+static double bf16_value(uint16_t bits)
+{
+    uint32_t u = (uint32_t)bits << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+int oracle_num_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/*
+ * Tree bookkeeping.  in_anc[i * n + j] = 1 when j is i or an ancestor of i.
+ * depth[i] = number of edges from the root.  Returns 0, or -1 when parent[]
+ * is not a tree rooted at node 0 (parent[0] must be -1, every other parent in
+ * [0, n), no cycles).  Nodes need not be in any particular order.
+ */
+int oracle_tree(const int32_t *parent, int n, int32_t *depth, uint8_t *in_anc)
+{
+    if (n < 1 || n > ORACLE_MAX_NODES || parent[0] != -1)
+        return -1;
+    for (int i = 1; i < n; ++i)
+        if (parent[i] < 0 || parent[i] >= n)
+            return -1;
+    memset(in_anc, 0, (size_t)n * n);
+    for (int i = 0; i < n; ++i) {
+        int j = i, steps = 0;
+        while (j != -1) {
+            if (steps > n)
+                return -1; /* cycle */
+            in_anc[(size_t)i * n + j] = 1;
+            j = (j == 0) ? -1 : parent[j];
+            ++steps;
+        }
+        depth[i] = steps - 1;
+    }
+    return 0;
+}
+
+/*
+ * Tree-masked attention of one layer.
+ *   q    [N][Hq][d]              bf16 bits, post-rotary
+ *   k, v [Hkv][head_stride] rows  bf16 bits; key slot s of kv head g starts at
+ *        g * head_stride + s * d.  Slots [0, L) are the prefix, [L, L + N) the
+ *        tree nodes in node order.
+ *   out  [N][Hq][d]              double
+ * q head h reads kv head h / (Hq / Hkv).  Softmax scale 1/sqrt(d).
+ */
+int oracle_tree_attention(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                          int64_t head_stride, int L, int N, int Hq, int Hkv, int d,
+                          const int32_t *parent, double *out)
+{
+    if (Hkv < 1 || Hq % Hkv != 0 || d < 1 || L < 0)
+        return -1;
+    uint8_t in_anc[ORACLE_MAX_NODES * ORACLE_MAX_NODES];
+    int32_t depth[ORACLE_MAX_NODES];
+    if (oracle_tree(parent, N, depth, in_anc) != 0)
+        return -1;
+    const int group = Hq / Hkv;
+    const double scale = 1.0 / sqrt((double)d);
+    const int n_keys = L + N;
+
+#pragma omp parallel
+    {
+        double *score = (double *)malloc(sizeof(double) * (size_t)n_keys);
+        int *allowed = (int *)malloc(sizeof(int) * (size_t)n_keys);
+#pragma omp for schedule(dynamic)
+        for (int ih = 0; ih < N * Hq; ++ih) {
+            const int i = ih / Hq, h = ih % Hq, g = h / group;
+            const uint16_t *qi = q + ((size_t)i * Hq + h) * d;
+            const uint16_t *kg = k + (size_t)g * head_stride;
+            const uint16_t *vg = v + (size_t)g * head_stride;
+            int n_allowed = 0;
+            for (int s = 0; s < L; ++s)
+                allowed[n_allowed++] = s;
+            for (int j = 0; j < N; ++j)
+                if (in_anc[(size_t)i * N + j])
+                    allowed[n_allowed++] = L + j;
+            double mx = -INFINITY;
+            for (int a = 0; a < n_allowed; ++a) {
+                const uint16_t *ks = kg + (size_t)allowed[a] * d;
+                double dot = 0.0;
+                for (int c = 0; c < d; ++c)
+                    dot += bf16_value(qi[c]) * bf16_value(ks[c]);
+                score[a] = dot * scale;
+                if (score[a] > mx)
+                    mx = score[a];
+            }
+            double denom = 0.0;
+            for (int a = 0; a < n_allowed; ++a) {
+                score[a] = exp(score[a] - mx);
+                denom += score[a];
+            }
+            double *o = out + ((size_t)i * Hq + h) * d;
+            for (int c = 0; c < d; ++c)
+                o[c] = 0.0;
+            for (int a = 0; a < n_allowed; ++a) {
+                const uint16_t *vs = vg + (size_t)allowed[a] * d;
+                const double w = score[a] / denom;
+                for (int c = 0; c < d; ++c)
+                    o[c] += w * bf16_value(vs[c]);
+            }
+        }
+        free(score);
+        free(allowed);
+    }
+    (void)n_keys;
+    return 0;
+}
+
+/*
+ * LM head and the per-row statistics of the greedy verifier.
+ *   hidden [R][D], W [V][D] (nn.Linear layout), both bf16 bits.
+ *   argmax[r]  first index of the largest logit
+ *   top1[r]    largest softmax probability
+ *   entropy[r] -sum_v p_v ln p_v (nats, temperature 1)
+ *   gap[r]     largest minus second-largest logit (may be NULL)
+ *   logits     [R][V] (may be NULL)
+ */
+int oracle_lm_head(const uint16_t *hidden, const uint16_t *W, int R, int D, int V,
+                   int32_t *argmax, double *top1, double *entropy, double *gap,
+                   double *logits)
+{
+    if (R < 0 || D < 1 || V < 1)
+        return -1;
+    double *z = (double *)malloc(sizeof(double) * (size_t)R * V);
+    if (!z)
+        return -2;
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int r = 0; r < R; ++r)
+        for (int vv = 0; vv < V; ++vv) {
+            const uint16_t *h = hidden + (size_t)r * D;
+            const uint16_t *w = W + (size_t)vv * D;
+            double acc = 0.0;
+            for (int c = 0; c < D; ++c)
+                acc += bf16_value(w[c]) * bf16_value(h[c]);
+            z[(size_t)r * V + vv] = acc;
+        }
+    for (int r = 0; r < R; ++r) {
+        const double *zr = z + (size_t)r * V;
+        int best = 0;
+        for (int vv = 1; vv < V; ++vv)
+            if (zr[vv] > zr[best])
+                best = vv;
+        double second = -INFINITY;
+        for (int vv = 0; vv < V; ++vv)
+            if (vv != best && zr[vv] > second)
+                second = zr[vv];
+        double denom = 0.0;
+        for (int vv = 0; vv < V; ++vv)
+            denom += exp(zr[vv] - zr[best]);
+        double ent = 0.0, pmax = 0.0;
+        for (int vv = 0; vv < V; ++vv) {
+            const double p = exp(zr[vv] - zr[best]) / denom;
+            if (p > 0.0)
+                ent -= p * log(p);
+            if (p > pmax)
+                pmax = p;
+        }
+        argmax[r] = best;
+        top1[r] = pmax;
+        entropy[r] = ent;
+        if (gap)
+            gap[r] = zr[best] - second;
+        if (logits)
+            memcpy(logits + (size_t)r * V, zr, sizeof(double) * (size_t)V);
+    }
+    free(z);
+    return 0;
+}
+
+/*
+ * Greedy tree acceptance.
+ *   parent[N], draft[N] (draft[0] ignored), argmax[N] (target greedy token
+ *   after each node).
+ * Outputs accept_len (>= 1), path[0 .. accept_len) = root .. j*, and the bonus
+ * token argmax[j*].  Returns 0 or -1 for an invalid tree.
+ */
+int oracle_accept(const int32_t *parent, int N, const int32_t *draft,
+                  const int32_t *argmax, int32_t *accept_len, int32_t *path,
+                  int32_t *bonus)
+{
+    uint8_t in_anc[ORACLE_MAX_NODES * ORACLE_MAX_NODES];
+    int32_t depth[ORACLE_MAX_NODES];
+    if (oracle_tree(parent, N, depth, in_anc) != 0)
+        return -1;
+    int best = 0;
+    for (int i = 0; i < N; ++i) {
+        int ok = 1;
+        for (int j = i; j != 0; j = parent[j])
+            if (draft[j] != argmax[parent[j]]) {
+                ok = 0;
+                break;
+            }
+        if (ok && (depth[i] > depth[best] || (depth[i] == depth[best] && i < best)))
+            best = i;
+    }
+    const int len = depth[best] + 1;
+    for (int j = best, pos = len - 1; pos >= 0; --pos) {
+        path[pos] = j;
+        j = (j == 0) ? -1 : parent[j];
+    }
+    *accept_len = len;
+    *bonus = argmax[best];
+    return 0;
+}
