@@ -1,0 +1,413 @@
+"""Benchmark of the per-step tree-verification pass on GB300.
+
+Default workload: the long-context full decode step of a 7B Llama-shaped
+model, batch 1: 32 layers of tree attention at 32 heads x 128 over a bf16 KV
+cache of L=16384 per layer, a 64-node depth-5 draft tree, then the 4096 x
+32000 bf16 LM head with argmax / top-1 / entropy, greedy acceptance and the
+KV-cache update.  One step = one verify_step call through the C ABI.
+
+Prints one JSON line (rank 0).  Metric: verify-steps/s (with tree-tokens/s
+and the fraction of the HBM roofline: KV + LM-head bytes over the measured
+copy bandwidth).  Inputs are seeded synthetic tensors of the model's shapes,
+resident in HBM and larger than L2 (8.9 GB touched per step), so no L2 flush
+is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config c4|c2|c1] [--impl ours|reference]
+
+--impl reference times the fp64 CPU oracle (the reference arm of this
+build) on the host cores on a bounded sample of the same workload,
+extrapolated to a full step.
+Under torchrun each rank runs an independent replica on its own GPU (weak
+scaling); the step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2606_27550_gb300 import synth  # noqa: E402
+
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload(cfg: str):
+    sh = synth.SHAPES[cfg]()
+    N = sh.N
+    kv_bytes = sh.n_layers * 2 * (sh.L + N) * sh.n_kv_heads * sh.head_dim * 2
+    w_bytes = sh.vocab * sh.d_model * 2
+    flops = 2 * N * sh.d_model * sh.vocab + 4 * N * (sh.L + N) * sh.head_dim * sh.n_q_heads * sh.n_layers
+    return sh, kv_bytes, w_bytes, flops
+
+
+def dist_info():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ----------------------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 100 ms while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for ln in out.strip().splitlines():
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[4:8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, x in enumerate(r) if x.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+
+def traffic_from_profiles(kernel: str):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if its
+    source hash still matches the current kernel source (else None)."""
+    import hashlib
+
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    for ln in open(path):
+        f = ln.split()
+        if len(f) >= 4 and f[0] == kernel and not ln.startswith("#"):
+            src = os.path.join(ROOT, "paper_2606_27550_gb300", "csrc", f[1])
+            if not os.path.exists(src):
+                return None
+            h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+            return float(f[3]) if h == f[2] else None
+    return None
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_27550_gb300 as tv
+    from paper_2606_27550_gb300 import build as tvbuild
+
+    world, rank, local = dist_info()
+    tvbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    sh, kv_bytes, w_bytes, flops = workload(args.config)
+    N, L, H, Hkv, d, D, V, nl = (sh.N, sh.L, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_model, sh.vocab,
+                                 sh.n_layers)
+    seed = 1234 + rank
+    bf = torch.bfloat16
+    k = synth.device_normal_bf16_(torch.empty((nl, Hkv, sh.L_cap, d), dtype=bf, device=dev), seed + 1)
+    v = synth.device_normal_bf16_(torch.empty((nl, Hkv, sh.L_cap, d), dtype=bf, device=dev), seed + 2)
+    q = synth.device_normal_bf16_(torch.empty((nl, N, H, d), dtype=bf, device=dev), seed + 3)
+    W = synth.device_normal_bf16_(torch.empty((V, D), dtype=bf, device=dev), seed + 4, std=sh.w_std)
+    hidden = synth.device_normal_bf16_(torch.empty((N, D), dtype=bf, device=dev), seed + 5)
+
+    bank = tv.Bank(16, local)
+    bid, order = bank.add(sh.parent)
+    kv = tv.KvCache(k, v, L)
+    out = torch.empty((nl, N, H, d), dtype=bf, device=dev)
+    am = torch.empty(N, dtype=torch.int32, device=dev)
+    t1 = torch.empty(N, dtype=torch.float32, device=dev)
+    en = torch.empty(N, dtype=torch.float32, device=dev)
+    res = tv.make_result(dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(N, nl, Hkv, H, d, V, local), dev)
+    stream = torch.cuda.current_stream()
+
+    # drafts: the greedy token of each node's parent with probability p, from an untimed LM-head pass
+    tv.lm_head_stats(hidden, W, am, t1, en, ws)
+    torch.cuda.synchronize()
+    drafts = torch.from_numpy(synth.gen_drafts(seed, sh.parent, am.cpu().numpy(), V, sh.p_match)).to(dev)
+
+    def step():
+        tv.verify_step(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, 0, stream)
+
+    visible = os.environ.get("CUDA_VISIBLE_DEVICES")
+    sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
+    sampler.start()
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    elapsed_ms = e0.elapsed_time(e1)
+    if world > 1:
+        dist.barrier()
+        t = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    r = tv.parse_result(res)
+
+    # per-kernel durations: the same work through the stage entry points, events between stages
+    n_k = max(3, min(args.steps, 50))
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_k)]
+    for i in range(n_k):
+        ev[i][0].record(stream)
+        tv.lm_head_stats(hidden, W, am, t1, en, ws, stream)
+        ev[i][1].record(stream)
+        tv.tree_attention(bank, bid, kv, q, out, ws, 0, nl, stream)
+        ev[i][2].record(stream)
+        tv.greedy_accept(bank, bid, drafts, am, V, L, res, stream)
+        tv.kv_compact(kv, res, stream)
+        ev[i][3].record(stream)
+    torch.cuda.synchronize()
+    t_lm = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    t_at = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    t_ac = statistics.mean(e[2].elapsed_time(e[3]) for e in ev)
+
+    # end to end: per step, pinned host -> device inputs, verify_step, device -> host result, host sync
+    q_h = torch.empty(q.shape, dtype=bf, pin_memory=True).copy_(q)
+    h_h = torch.empty(hidden.shape, dtype=bf, pin_memory=True).copy_(hidden)
+    d_h = torch.empty(drafts.shape, dtype=torch.int32, pin_memory=True).copy_(drafts)
+    res_h = torch.empty(res.shape, dtype=torch.int32, pin_memory=True)
+    stats_h = torch.empty((3, N), dtype=torch.float32, pin_memory=True)
+    h2d = q_h.numel() * 2 + h_h.numel() * 2 + d_h.numel() * 4
+    d2h = res_h.numel() * 4 + stats_h.numel() * 4
+    n_e2e = max(3, min(args.steps, 50))
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(n_e2e):
+        q.copy_(q_h, non_blocking=True)
+        hidden.copy_(h_h, non_blocking=True)
+        drafts.copy_(d_h, non_blocking=True)
+        step()
+        res_h.copy_(res, non_blocking=True)
+        stats_h[0].copy_(am.view(torch.float32), non_blocking=True)
+        stats_h[1].copy_(t1, non_blocking=True)
+        stats_h[2].copy_(en, non_blocking=True)
+        stream.synchronize()
+        _ = int(res_h[0])  # the per-step host read of the accepted length
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    clocks = sampler.stop()
+
+    if world > 1:
+        dist.destroy_process_group()
+    bank.close()
+    if rank != 0:
+        return
+
+    peaks, peak_src = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    ms = elapsed_ms / args.steps
+    value = world * args.steps / (elapsed_ms / 1e3)
+    at_gbs = kv_bytes / (t_at * 1e-3) / 1e9
+    line = {
+        "metric": "verify-steps/s",
+        "value": round(value, 3),
+        "unit": "verify-steps/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded normal bf16 K/V, queries, hidden rows; LM head N(0, 0.02^2)); "
+                "drafts = parent greedy token with p, else uniform",
+        "config": {"workload": sh.name, "layers": nl, "q_heads": H, "kv_heads": Hkv, "head_dim": d, "L": L,
+                   "tree_nodes": N, "tree_depth": int(synth.depth_of(sh.parent).max()), "d_model": D, "vocab": V,
+                   "batch": 1, "l2": f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)"},
+        "tree_tokens_per_s": round(value * N, 1),
+        "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
+                         "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
+                         "peak_gbs": hbm, "peak_src": peak_src},
+        "roofline": {"kernel": "k1_tree_attention", "bound": "hbm", "achieved": round(at_gbs, 1), "peak": hbm,
+                     "unit": "GB/s", "frac": round(at_gbs / hbm, 4), "traffic": traffic_from_profiles("k1_tree_attention"),
+                     "algorithmic_bytes": kv_bytes, "avg_launch_ms": round(t_at, 4)},
+        "kernels_ms": {"k2_lm_head": round(t_lm, 4), "k1_tree_attention": round(t_at, 4),
+                       "k3_accept_compact": round(t_ac, 4)},
+        "lm_head_gbs": round(w_bytes / (t_lm * 1e-3) / 1e9, 1),
+        "accept_len_last": r["accept_len"],
+        "e2e": {"value": round(world * n_e2e / e2e_s, 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.config, budget_s=args.cpu_budget)
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- CPU oracle (reference arm)
+
+
+def cpu_sample_step(cfg: str, attn_units: int, vocab_slices: int, seed: int = 0):
+    """Runs the fp64 oracle on `attn_units` (layer, kv head) attention units and
+    `vocab_slices` 1/32 vocab slices of the LM head plus acceptance; returns
+    (extrapolated seconds of one full step, sample description)."""
+    import oracle
+
+    sh, _, _, _ = workload(cfg)
+    N, L, d, D, V = sh.N, sh.L, sh.head_dim, sh.d_model, sh.vocab
+    g = synth.rng(seed, 99)
+    units_total = sh.n_layers * sh.n_kv_heads
+    group = sh.n_q_heads // sh.n_kv_heads
+    k = synth.normal_bf16(g, (1, L + N, d))
+    v = synth.normal_bf16(g, (1, L + N, d))
+    q = synth.normal_bf16(g, (N, group, d))
+    slice_rows = (V + 31) // 32
+    Wslice = synth.normal_bf16(g, (slice_rows, D), sh.w_std)
+    hidden = synth.normal_bf16(g, (N, D))
+    t0 = time.perf_counter()
+    for _ in range(attn_units):
+        oracle.tree_attention(q, k, v, L, sh.parent)
+    t_attn = (time.perf_counter() - t0) / attn_units
+    t0 = time.perf_counter()
+    for _ in range(vocab_slices):
+        am, _, _, _ = oracle.lm_head(hidden, Wslice)
+    t_lm = (time.perf_counter() - t0) / vocab_slices
+    t0 = time.perf_counter()
+    drafts = synth.gen_drafts(seed, sh.parent, am, slice_rows, sh.p_match)
+    oracle.accept(sh.parent, drafts, am)
+    t_acc = time.perf_counter() - t0
+    full = t_attn * units_total + t_lm * 32 + t_acc
+    sample = (f"{attn_units} of {units_total} (layer, kv head) attention units ({N} nodes x {group} q heads x "
+              f"{L + N} keys x d {d}) and {vocab_slices} of 32 vocab slices ({slice_rows} x {D}) of the LM head "
+              f"for {N} rows, plus acceptance; time extrapolated to one full step")
+    return full, sample, t_attn + t_lm
+
+
+def cpu_baseline(cfg: str, budget_s: float = 20.0):
+    """The oracle timed on this host's cores on a bounded sample of the workload."""
+    import oracle
+
+    oracle.build()
+    _, _, probe = cpu_sample_step(cfg, 1, 1)
+    n = int(max(1, min(64, budget_s / max(probe, 1e-6))))
+    full, sample, _ = cpu_sample_step(cfg, n, n, seed=1)
+    return {"value": round(1.0 / full, 6), "unit": "verify-steps/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": sample, "s_per_full_step": round(full, 3)}
+
+
+def run_reference(args):
+    import oracle
+
+    world, rank, _ = dist_info()
+    if rank != 0:
+        return
+    oracle.build()
+    sh, _, _, _ = workload(args.config)
+    for i in range(args.warmup):
+        cpu_sample_step(args.config, 1, 1, seed=i)
+    times = []
+    sample = ""
+    for i in range(args.steps):
+        full, sample, _ = cpu_sample_step(args.config, 1, 1, seed=100 + i)
+        times.append(full)
+    mean = statistics.mean(times)
+    value = 1.0 / mean
+    line = {
+        "impl": "reference",
+        "metric": "verify-steps/s",
+        "value": round(value, 6),
+        "unit": "verify-steps/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(mean * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded)",
+        "config": {"workload": sh.name},
+        "cpu_baseline": {"value": round(value, 6), "unit": "verify-steps/s", "cores": oracle.num_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 6), "unit": "verify-steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c4"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

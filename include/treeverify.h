@@ -1,0 +1,220 @@
+/*
+ * treeverify.h -- C ABI of the GB300 tree-verification library.
+ *
+ * One decode step of Medusa/Hydra multi-token-prediction decoding verifies a
+ * draft tree of N <= 64 candidate tokens in one target-model pass: tree-masked
+ * attention over the KV cache, the LM head with the greedy token, top-1
+ * probability and entropy per node, greedy acceptance of the longest root path
+ * whose drafts the target agrees with, and the KV-cache update that keeps the
+ * accepted path (EntMTP, Sec. 3.2: proposal -> tree decoding -> verification ->
+ * KV-cache update).  Trees live in a TopologyBank of precompiled topologies so
+ * that switching trees between steps is an O(1) pointer swap (Sec. 1 and
+ * Sec. 4, "Cost").
+ *
+ * Conventions that hold for every entry point:
+ *  - Device pointers are owned by the caller.  The library allocates device
+ *    memory only in tb_create (the bank); no other call allocates.
+ *  - Calls that take a stream only enqueue work on it and return without
+ *    synchronising.  Host-side argument errors are returned before anything is
+ *    enqueued.  Errors that only the GPU can detect are reported in the
+ *    workspace status word (tb_workspace_status) and, for verify_step and
+ *    greedy_accept, in tb_result.status.
+ *  - bf16 tensors are IEEE bfloat16 bit patterns.  All device buffers must be
+ *    16-byte aligned.
+ *  - Errors are negative tb_status codes; tb_last_error() returns a message
+ *    for the last failing call on the calling thread.  No C++ exception
+ *    crosses this interface.
+ */
+#ifndef TREEVERIFY_H
+#define TREEVERIFY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define TB_API __attribute__((visibility("default")))
+#else
+#define TB_API
+#endif
+
+#define TB_MAX_NODES 64 /* nodes per draft tree, root included */
+
+typedef enum {
+    TB_OK = 0,
+    TB_EINVAL = -1,      /* bad argument (pointer, size, stride, alignment, tree) */
+    TB_ENOMEM = -2,      /* device allocation failed (tb_create only) */
+    TB_ECUDA = -3,       /* a CUDA runtime or driver call failed */
+    TB_ENOTFOUND = -4,   /* bank_id does not name a topology */
+    TB_ECAPACITY = -5,   /* bank full, workspace too small, or L + N > L_cap */
+    TB_ETIMEOUT = -6,    /* a bounded device-side wait expired (kernel gave up) */
+    TB_EUNSUPPORTED = -7 /* shape outside what the kernels implement */
+} tb_status;
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st *tb_stream;
+
+/* Opaque TopologyBank: the precompiled draft trees of one device. */
+typedef struct tb_bank tb_bank;
+
+/* ------------------------------------------------------------------------
+ * Topologies (Sec. 2.3: draft trees with precomputed attention masks,
+ * position offsets and gather indices; Sec. 4 "Cost": per-tree buffers, so a
+ * switch is a pointer swap with no GPU work).
+ * ---------------------------------------------------------------------- */
+
+/* Pure host.  Validates parent[0..n) as a tree rooted at node 0 (parent[0] ==
+ * -1, every other parent in [0, n), no cycle) and returns it in canonical
+ * breadth-first order: children of a node in increasing original index.
+ *   order[c]      original index of canonical node c          (may be NULL)
+ *   bfs_parent[c] canonical parent (-1 for the root)          (may be NULL)
+ *   depth[c]      edges from the root = position offset        (may be NULL)
+ *   anc[c]        bit j set iff canonical node j is c or an ancestor of c
+ *                 (the tree attention mask row of c)          (may be NULL)
+ * In canonical order parent < child and depth is non-decreasing.
+ * Returns TB_EINVAL for 1 > n > 64 or a parent array that is not such a tree. */
+TB_API tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
+                          int32_t *depth, uint64_t *anc);
+
+/* Creates an empty bank of max_topologies (1..4096) trees on CUDA device
+ * `device` and allocates its device table.  Synchronous. */
+TB_API tb_status tb_create(tb_bank **out, int max_topologies, int device);
+
+/* Canonicalises parent[0..n) (host array, see tb_canonicalize), uploads the
+ * ancestor bitsets, depths and parents once (synchronous copy), and returns
+ * its id (0, 1, ... in insertion order).  `order` (n entries, may be NULL)
+ * receives the canonical -> caller index map: draft tokens, queries and tree
+ * K/V slots are passed in canonical order.  TB_ECAPACITY when the bank is full. */
+TB_API tb_status tb_add_topology(tb_bank *bank, const int32_t *parent, int n, int *out_id, int32_t *order);
+
+/* Host copy of a stored topology (canonical order).  Any output may be NULL;
+ * parent/depth/anc need room for *n entries (at most 64). */
+TB_API tb_status tb_get_topology(const tb_bank *bank, int id, int *n, int32_t *parent, int32_t *depth,
+                          uint64_t *anc);
+
+/* Frees the bank's device table.  Work already enqueued that uses the bank
+ * must have completed.  NULL is accepted. */
+TB_API tb_status tb_destroy(tb_bank *bank);
+
+/* ------------------------------------------------------------------------
+ * KV cache and results
+ * ---------------------------------------------------------------------- */
+
+/* The caller's bf16 KV cache.  Element (layer, kv head g, slot s, c) of K is at
+ * k + layer * layer_stride + g * head_stride + s * head_dim + c, likewise V.
+ * Slots [0, L) hold the prefix; the N tree nodes of the step occupy slots
+ * [L, L + N) in canonical node order (the keys/values of the draft tokens,
+ * produced by the model's K/V projection before the call).  Strides are in
+ * elements and must be multiples of 8; head_dim is 64 or 128. */
+typedef struct tb_kv {
+    void *k;
+    void *v;
+    int64_t layer_stride;
+    int64_t head_stride;
+    int32_t n_layers;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    int32_t L;     /* prefix length of this step */
+    int32_t L_cap; /* slots per head: L + N <= L_cap */
+} tb_kv;
+
+/* Device-resident result of one verification, written by the GPU. */
+typedef struct tb_result {
+    int32_t accept_len;  /* accepted tokens incl. the bonus token: depth(j*) + 1 */
+    int32_t bonus_token; /* target greedy token after the last accepted node */
+    int32_t new_L;       /* L + accept_len: the prefix length for the next step */
+    int32_t status;      /* TB_OK or a device-detected tb_status */
+    int32_t path[TB_MAX_NODES]; /* path[0 .. accept_len) = root .. j*, canonical ids */
+} tb_result;
+
+/* ------------------------------------------------------------------------
+ * Workspace: scratch for split-L attention partials, LM-head partials and
+ * arrival counters.  Caller-allocated device memory; must be zero-filled
+ * before its first use (tb_workspace_init) and again after any call that
+ * reported TB_ETIMEOUT.  Kernels leave their counters at zero on success.
+ * One workspace must not be used by two calls that can run concurrently.
+ * ---------------------------------------------------------------------- */
+
+/* Bytes of workspace for calls with up to max_rows LM-head rows and up to
+ * n_layers x n_kv_heads attention heads of head_dim, vocab entries, on device
+ * `device` (the grid size depends on its SM count). */
+TB_API size_t tb_workspace_size(int max_rows, int n_layers, int n_kv_heads, int n_q_heads, int head_dim,
+                         int vocab, int device);
+
+/* Zero-fills the workspace on `stream` (asynchronous). */
+TB_API tb_status tb_workspace_init(void *workspace, size_t workspace_bytes, tb_stream stream);
+
+/* Synchronously reads the workspace status word: TB_OK or the first
+ * device-detected error (TB_ETIMEOUT, TB_EINVAL). */
+TB_API tb_status tb_workspace_status(const void *workspace, int32_t *status);
+
+/* ------------------------------------------------------------------------
+ * The verification pass and its stages
+ * ---------------------------------------------------------------------- */
+
+/* Tree-masked attention (tree decoding, Sec. 3.2; mask = ancestor bitsets,
+ * Sec. 2.3) for layers [layer_begin, layer_begin + n_layers) of kv:
+ *   O[i, h] = sum_s softmax_s(q[i, h] . k[s, g] / sqrt(head_dim)) v[s, g]
+ * over s in [0, L) and the tree slots L + j of the ancestors-or-self j of node
+ * i; g = h / (n_q_heads / n_kv_heads).
+ *   q   bf16 [n_layers][N][n_q_heads][head_dim] (post-rotary), read only
+ *   out bf16 [n_layers][N][n_q_heads][head_dim]
+ * N is the topology's node count.  n_q_heads must be a multiple of
+ * n_kv_heads, N * (n_q_heads / n_kv_heads) <= 256. */
+TB_API tb_status tree_attention(const tb_bank *bank, int bank_id, const tb_kv *kv, int layer_begin,
+                         int n_layers, const void *q, int n_q_heads, void *out, void *workspace,
+                         size_t workspace_bytes, tb_stream stream);
+
+/* Fused LM head: z_r = W h_r for every row, never written to memory; per row
+ * the greedy token argmax_v z (lowest index on ties), the top-1 probability
+ * max softmax(z) (the base-LM p0 of Sec. 4) and the entropy -sum p ln p in
+ * nats (the entropy feature of the scheduler, Sec. 4 / App. A).
+ *   hidden bf16 [n_rows][d_model]; lm_head bf16 [vocab][d_model] (nn.Linear)
+ *   argmax int32 [n_rows]; top1, entropy float [n_rows]
+ * 1 <= n_rows <= 256, d_model a multiple of 8, vocab >= 1. */
+TB_API tb_status lm_head_stats(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
+                        int32_t *argmax, float *top1, float *entropy, void *workspace,
+                        size_t workspace_bytes, tb_stream stream);
+
+/* Greedy acceptance (verification, Sec. 3.2, greedy form): node i is accepted
+ * when every non-root node j on its root path has draft_tokens[j] ==
+ * argmax[parent(j)]; j* is the deepest accepted node (smallest canonical id
+ * among equally deep ones).  Writes accept_len, path, bonus_token =
+ * argmax[j*], new_L = L + accept_len and status into *result.  A draft token
+ * outside [0, vocab) never matches and sets status TB_EINVAL.
+ * draft_tokens, argmax: device int32 [N]; draft_tokens[0] is ignored. */
+TB_API tb_status greedy_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens,
+                        const int32_t *argmax, int vocab, int L, tb_result *result,
+                        tb_stream stream);
+
+/* KV-cache update after acceptance (Sec. 3.2): for every layer and kv head of
+ * kv, slot L + j receives the K and V of slot L + path[j], j < accept_len,
+ * read from the device tb_result written by greedy_accept.  In place; all
+ * other slots are untouched. */
+TB_API tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream);
+
+#define TB_NO_COMPACT 1 /* verify_step flag: skip the KV-cache update */
+
+/* One full verification step of topology bank_id: tree_attention over all
+ * kv->n_layers layers, lm_head_stats over the N node rows, greedy_accept, and
+ * (unless TB_NO_COMPACT) kv_compact, enqueued on `stream` in that order.
+ *   hidden bf16 [N][d_model] (final hidden state of each node)
+ *   attn_out bf16 [n_layers][N][n_q_heads][head_dim]
+ *   argmax int32 / top1, entropy float [N]; result: device tb_result. */
+TB_API tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q,
+                      int n_q_heads, const void *hidden, const void *lm_head, int d_model,
+                      int vocab, const int32_t *draft_tokens, void *attn_out, int32_t *argmax,
+                      float *top1, float *entropy, tb_result *result, void *workspace,
+                      size_t workspace_bytes, int flags, tb_stream stream);
+
+/* Message for the last failing call on this thread ("" if none). */
+TB_API const char *tb_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TREEVERIFY_H */

@@ -1,0 +1,254 @@
+"""GB300 tree-verification library: Python binding of libtreeverify.so.
+
+Thin ctypes marshalling over the C ABI declared in include/treeverify.h; the
+functions keep the C names.  Every step of the verification pass runs in the
+library's CUDA kernels; this module only turns torch tensors into pointers
+and sizes.  PyTorch provides device memory and streams.
+
+Importing this module does not require a GPU; calling the compute entry
+points does, and a missing library raises immediately (there is no CPU
+fallback).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libtreeverify.so")
+
+TB_OK, TB_EINVAL, TB_ENOMEM, TB_ECUDA, TB_ENOTFOUND, TB_ECAPACITY, TB_ETIMEOUT, TB_EUNSUPPORTED = (
+    0, -1, -2, -3, -4, -5, -6, -7)
+TB_MAX_NODES = 64
+TB_NO_COMPACT = 1
+RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
+
+API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
+       "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
+       "kv_compact", "verify_step", "tb_last_error")
+
+
+class TreeVerifyError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str):
+        super().__init__(f"{where} failed ({status}): {message}")
+        self.status = status
+
+
+class TbKv(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("layer_stride", ctypes.c_int64),
+                ("head_stride", ctypes.c_int64), ("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("L", ctypes.c_int32), ("L_cap", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Loads libtreeverify.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with paper_2606_27550_gb300.build.build()")
+    lib = ctypes.CDLL(path)
+    P, i32, i64, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t
+    sig = {
+        "tb_canonicalize": [P, i32, P, P, P, P],
+        "tb_create": [P, i32, i32],
+        "tb_add_topology": [P, P, i32, P, P],
+        "tb_get_topology": [P, i32, P, P, P, P],
+        "tb_destroy": [P],
+        "tb_workspace_size": [i32, i32, i32, i32, i32, i32, i32],
+        "tb_workspace_init": [P, sz, P],
+        "tb_workspace_status": [P, P],
+        "tree_attention": [P, i32, P, i32, i32, P, i32, P, P, sz, P],
+        "lm_head_stats": [P, i32, P, i32, i32, P, P, P, P, sz, P],
+        "greedy_accept": [P, i32, P, P, i32, i32, P, P],
+        "kv_compact": [P, P, P],
+        "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
+        "tb_last_error": [],
+    }
+    for name, args in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ctypes.c_int
+    lib.tb_workspace_size.restype = ctypes.c_size_t
+    lib.tb_last_error.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _check(rc: int, where: str):
+    if rc != TB_OK:
+        raise TreeVerifyError(rc, where, load().tb_last_error().decode())
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+# --------------------------------------------------------------------- topologies
+
+
+def tb_canonicalize(parent):
+    """(order, bfs_parent, depth, anc) of a parent array (pure host)."""
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    n = len(parent)
+    order = np.zeros(n, np.int32)
+    bp = np.zeros(n, np.int32)
+    depth = np.zeros(n, np.int32)
+    anc = np.zeros(n, np.uint64)
+    _check(load().tb_canonicalize(_ptr(parent), n, _ptr(order), _ptr(bp), _ptr(depth), _ptr(anc)), "tb_canonicalize")
+    return order, bp, depth, anc
+
+
+class Bank:
+    """A TopologyBank on one device (tb_create / tb_add_topology / tb_destroy)."""
+
+    def __init__(self, max_topologies: int = 64, device: int = 0):
+        h = ctypes.c_void_p()
+        _check(load().tb_create(ctypes.byref(h), max_topologies, device), "tb_create")
+        self.handle = h
+        self.device = device
+        self.sizes: list[int] = []
+
+    def add(self, parent):
+        """Adds a topology; returns (bank_id, order) with order[canonical] = caller index."""
+        parent = np.ascontiguousarray(parent, dtype=np.int32)
+        out = ctypes.c_int()
+        order = np.zeros(len(parent), np.int32)
+        _check(load().tb_add_topology(self.handle, _ptr(parent), len(parent), ctypes.byref(out), _ptr(order)),
+               "tb_add_topology")
+        self.sizes.append(len(parent))
+        return out.value, order
+
+    def get(self, bank_id: int):
+        n = ctypes.c_int()
+        parent = np.zeros(TB_MAX_NODES, np.int32)
+        depth = np.zeros(TB_MAX_NODES, np.int32)
+        anc = np.zeros(TB_MAX_NODES, np.uint64)
+        _check(load().tb_get_topology(self.handle, bank_id, ctypes.byref(n), _ptr(parent), _ptr(depth), _ptr(anc)),
+               "tb_get_topology")
+        k = n.value
+        return parent[:k].copy(), depth[:k].copy(), anc[:k].copy()
+
+    def n_nodes(self, bank_id: int) -> int:
+        return self.sizes[bank_id]
+
+    def close(self):
+        if self.handle:
+            _check(load().tb_destroy(self.handle), "tb_destroy")
+            self.handle = None
+
+    def __del__(self):  # pragma: no cover
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# --------------------------------------------------------------------- KV cache, workspace, result
+
+
+@dataclass
+class KvCache:
+    """bf16 K and V caches shaped [n_layers][n_kv_heads][L_cap][head_dim]."""
+
+    k: object
+    v: object
+    L: int
+
+    def as_c(self) -> TbKv:
+        n_layers, n_kv_heads, L_cap, head_dim = self.k.shape
+        s = self.k.stride()
+        return TbKv(self.k.data_ptr(), self.v.data_ptr(), s[0], s[1], n_layers, n_kv_heads, head_dim, self.L, L_cap)
+
+
+def tb_workspace_size(max_rows: int, n_layers: int, n_kv_heads: int, n_q_heads: int, head_dim: int, vocab: int,
+                      device: int = -1) -> int:
+    return int(load().tb_workspace_size(max_rows, n_layers, n_kv_heads, n_q_heads, head_dim, vocab, device))
+
+
+def make_workspace(nbytes: int, device="cuda"):
+    """Zero-filled device workspace (torch uint8)."""
+    import torch
+
+    return torch.zeros(nbytes, dtype=torch.uint8, device=device)
+
+
+def tb_workspace_init(ws, stream=None):
+    _check(load().tb_workspace_init(_ptr(ws), ws.numel(), _stream(stream)), "tb_workspace_init")
+
+
+def tb_workspace_status(ws) -> int:
+    st = ctypes.c_int32()
+    _check(load().tb_workspace_status(_ptr(ws), ctypes.byref(st)), "tb_workspace_status")
+    return st.value
+
+
+def make_result(device="cuda"):
+    """Device buffer for one tb_result (int32[68])."""
+    import torch
+
+    return torch.zeros(RESULT_INTS, dtype=torch.int32, device=device)
+
+
+def parse_result(res) -> dict:
+    r = [int(x) for x in (res.cpu() if hasattr(res, "cpu") else res)]
+    k = r[0]
+    return {"accept_len": k, "bonus_token": r[1], "new_L": r[2], "status": r[3], "path": r[4:4 + k]}
+
+
+# --------------------------------------------------------------------- the pass
+
+
+def tree_attention(bank: Bank, bank_id: int, kv: KvCache, q, out, ws, layer_begin: int = 0, n_layers: int | None = None,
+                   stream=None):
+    """q, out: bf16 [n_layers][N][n_q_heads][head_dim]."""
+    c = kv.as_c()
+    nl = c.n_layers - layer_begin if n_layers is None else n_layers
+    _check(load().tree_attention(bank.handle, bank_id, ctypes.byref(c), layer_begin, nl, _ptr(q), q.shape[2],
+                                 _ptr(out), _ptr(ws), ws.numel(), _stream(stream)), "tree_attention")
+
+
+def lm_head_stats(hidden, lm_head, argmax, top1, entropy, ws, stream=None):
+    """hidden bf16 [R][d_model]; lm_head bf16 [V][d_model]; outputs [R]."""
+    R, D = hidden.shape
+    _check(load().lm_head_stats(_ptr(hidden), R, _ptr(lm_head), D, lm_head.shape[0], _ptr(argmax), _ptr(top1),
+                                _ptr(entropy), _ptr(ws), ws.numel(), _stream(stream)), "lm_head_stats")
+
+
+def greedy_accept(bank: Bank, bank_id: int, draft, argmax, vocab: int, L: int, result, stream=None):
+    _check(load().greedy_accept(bank.handle, bank_id, _ptr(draft), _ptr(argmax), vocab, L, _ptr(result),
+                                _stream(stream)), "greedy_accept")
+
+
+def kv_compact(kv: KvCache, result, stream=None):
+    c = kv.as_c()
+    _check(load().kv_compact(ctypes.byref(c), _ptr(result), _stream(stream)), "kv_compact")
+
+
+def verify_step(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft, attn_out, argmax, top1, entropy,
+                result, ws, flags: int = 0, stream=None):
+    c = kv.as_c()
+    _check(load().verify_step(bank.handle, bank_id, ctypes.byref(c), _ptr(q), q.shape[2], _ptr(hidden),
+                              _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(draft), _ptr(attn_out),
+                              _ptr(argmax), _ptr(top1), _ptr(entropy), _ptr(result), _ptr(ws), ws.numel(), flags,
+                              _stream(stream)), "verify_step")

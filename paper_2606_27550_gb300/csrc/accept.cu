@@ -1,0 +1,152 @@
+// accept.cu -- greedy tree acceptance and KV-cache compaction (K3).
+//
+// Verification (Sec. 3.2, greedy form): a non-root node j "matches" when its
+// draft token equals the target's greedy token after its parent,
+// draft[j] == argmax[parent(j)].  Node i is accepted when every non-root node
+// of its ancestor-or-self set matches; with the ancestor bitset anc[i] this is
+// (anc[i] & ~match & ~root) == 0, one AND per node.  The accepted path ends at
+// the deepest accepted node j* (smallest canonical id among equally deep
+// ones); it is exactly the set bits of anc[j*] in increasing id order because
+// canonical order puts every parent before its children.  accept_len =
+// depth(j*) + 1 tokens are emitted: the accepted drafts plus the bonus token
+// argmax[j*] (Sec. 5.1: tau counts tokens per draft-verify cycle).
+//
+// KV-cache update (Sec. 3.2): slot L + j takes slot L + path[j] for
+// j < accept_len, in every layer and kv head.  path[j] >= j and path is
+// increasing, so copying rows in increasing j never reads a row that an
+// earlier copy overwrote; one warp copies one (layer, head, K|V) row set in
+// that order, with a warp barrier between rows.
+//
+// Every CTA recomputes the (tiny) acceptance itself, so acceptance and
+// compaction run as one launch without a grid-wide barrier.
+#include "kernels.cuh"
+
+namespace tv {
+
+__device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k, int row_bytes, int room, int lane)
+{
+    for (int j = 1; j < k; ++j) {
+        const int src = path[j];
+        if (src != j && src > j && src < room) {
+            const uint8_t *s = base + (size_t)src * row_bytes;
+            uint8_t *d = base + (size_t)j * row_bytes;
+            for (int off = lane * 16; off < row_bytes; off += 32 * 16)
+                *reinterpret_cast<uint4 *>(d + off) = *reinterpret_cast<const uint4 *>(s + off);
+        }
+        __syncwarp();
+    }
+}
+
+__global__ void __launch_bounds__(256) k3_accept_compact(const AcceptParams p)
+{
+    __shared__ int s_path[kMaxNodes];
+    __shared__ int s_len;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (p.from_result) {
+        if (threadIdx.x < kMaxNodes)
+            s_path[threadIdx.x] = p.result->path[threadIdx.x];
+        if (threadIdx.x == 0)
+            s_len = min(max(p.result->accept_len, 1), kMaxNodes);
+        __syncthreads();
+    } else {
+        if (warp == 0) {
+            const TreeDesc *t = p.tree;
+            const int n = t->n;
+            uint64_t match = 0;
+            bool bad = false;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int i = lane + 32 * h;
+                bool m = false;
+                if (i >= 1 && i < n) {
+                    const int tok = p.draft[i];
+                    bad |= (tok < 0 || tok >= p.vocab);
+                    m = (tok == p.argmax[t->parent[i]]);
+                }
+                const uint32_t bits = __ballot_sync(0xffffffffu, m);
+                match |= (uint64_t)bits << (32 * h);
+            }
+            const bool any_bad = __any_sync(0xffffffffu, bad);
+            // key = depth * 128 + (127 - id): the max is the deepest, smallest-id accepted node
+            int best = 127;  // the root (depth 0, id 0) is always accepted
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int i = lane + 32 * h;
+                if (i < n) {
+                    const uint64_t a = t->anc[i];
+                    if ((a & ~match & ~1ull) == 0ull) {
+                        const int key = t->depth[i] * 128 + (127 - i);
+                        best = max(best, key);
+                    }
+                }
+            }
+#pragma unroll
+            for (int m = 16; m >= 1; m >>= 1)
+                best = max(best, __shfl_xor_sync(0xffffffffu, best, m));
+            const int jstar = 127 - (best & 127);
+            const uint64_t pa = t->anc[jstar];
+            const int len = __popcll(pa);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int i = lane + 32 * h;
+                if ((pa >> i) & 1ull)
+                    s_path[__popcll(pa & ((1ull << i) - 1ull))] = i;
+            }
+            if (lane == 0) {
+                s_len = len;
+                if (blockIdx.x == 0) {
+                    tb_result *r = p.result;
+                    r->accept_len = len;
+                    r->bonus_token = p.argmax[jstar];
+                    r->new_L = p.L + len;
+                    int st = TB_OK;
+                    const int ws = p.ws_status ? *p.ws_status : 0;
+                    if (ws & kStatusTimeout)
+                        st = TB_ETIMEOUT;
+                    else if (any_bad || (ws & kStatusBadToken))
+                        st = TB_EINVAL;
+                    r->status = st;
+                }
+            }
+            __syncwarp();
+            if (blockIdx.x == 0)
+                for (int i = lane; i < kMaxNodes; i += 32)
+                    p.result->path[i] = (i < len) ? s_path[i] : -1;
+        }
+        __syncthreads();
+    }
+
+    if (p.n_layers == 0)
+        return;
+    const int k = s_len;
+    if (k <= 1)
+        return;
+    const int units = p.n_layers * p.n_kv_heads * 2;
+    const int warps_per_cta = blockDim.x >> 5;
+    for (int unit = blockIdx.x * warps_per_cta + warp; unit < units; unit += gridDim.x * warps_per_cta) {
+        const int which = unit & 1;
+        const int lh = unit >> 1;
+        const int head = lh % p.n_kv_heads, layer = lh / p.n_kv_heads;
+        uint8_t *base = (which ? p.v : p.k) + layer * p.layer_stride_b + head * p.head_stride_b +
+                        (size_t)p.L * p.row_bytes;
+        copy_rows(base, s_path, k, p.row_bytes, p.L_cap - p.L, lane);
+    }
+}
+
+cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream)
+{
+    int grid = 1;
+    if (p.n_layers > 0) {
+        const int units = p.n_layers * p.n_kv_heads * 2;
+        grid = (units + 7) / 8;
+        if (grid > 2 * n_sm)
+            grid = 2 * n_sm;
+        if (grid < 1)
+            grid = 1;
+    }
+    k3_accept_compact<<<grid, 256, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace tv

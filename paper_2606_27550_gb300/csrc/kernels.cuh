@@ -1,0 +1,54 @@
+// kernels.cuh -- host-side interface between the C-ABI layer and the kernels.
+#pragma once
+
+#include "common.cuh"
+
+namespace tv {
+
+// LM head (lm_head.cu)
+struct LmPlan {
+    int R_pad, n_tiles, n_kblocks, stages, tmem_cols, group_size, n_groups;
+    size_t smem_bytes;
+    size_t ws_bytes;  // partials (tile + group), 256-byte aligned
+};
+LmPlan lm_plan(int R, int D, int V);
+cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
+                           float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
+                           const char **err);
+
+// tree attention (attention.cu)
+struct AttnPlan {
+    int group, rows, row_blocks, T, n_units, P;
+    long long total;
+};
+AttnPlan attn_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
+size_t attn_slot_floats(int d);
+cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
+                        const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                        cudaStream_t stream, const char **err);
+
+// acceptance + compaction (accept.cu)
+struct AcceptParams {
+    const TreeDesc *tree;
+    const int32_t *draft;
+    const int32_t *argmax;
+    int vocab, L;
+    tb_result *result;
+    const int *ws_status;  // may be null
+    // compaction (n_layers == 0: acceptance only)
+    uint8_t *k;
+    uint8_t *v;
+    long long layer_stride_b, head_stride_b;
+    int n_layers, n_kv_heads, row_bytes;
+    int L_cap;        // slots per head: copies touching slots >= L_cap are skipped
+    int from_result;  // compaction driven by an existing result (kv_compact): no acceptance
+};
+cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
+
+// tensor maps (treeverify.cu)
+bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                  uint32_t box_inner, uint32_t box_outer, const char **err);
+bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_heads, int n_layers,
+                  int64_t head_stride, int64_t layer_stride, const char **err);
+
+}  // namespace tv

@@ -1,0 +1,371 @@
+// lm_head.cu -- fused LM head with per-row greedy statistics (K2 + merge).
+//
+// For every tree row r: z = W h_r over the whole vocabulary, reduced on the
+// fly to (max, argmax, s = sum e^(z-max), t = sum e^(z-max)(z-max)); logits
+// never reach memory.  top1 = 1/s, entropy = ln s - t/s (nats).
+// These are the verifier's greedy token, the base-LM top-1 probability p0 and
+// the entropy feature that the EntMTP scheduler consumes (Sec. 4, "Path-value
+// score" and "Cost": computed from the verifier logits already on chip).
+//
+// Design (swap-AB): one CTA per 128-entry vocab tile.  The tile of W
+// ([128][64] bf16 per k-block, 128-byte swizzled by TMA) is the MMA's M=128 A
+// operand; the tree rows ([R_pad][64] per k-block, same swizzle) are the
+// N = R_pad B operand.  tcgen05.mma (kind::f16, f32 accumulate) builds the
+// 128 x R_pad logit tile in TMEM over d_model/64 k-blocks fed by a multi-stage
+// TMA ring.  Warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, then all
+// four warps read TMEM (lane = vocab entry), transpose through shared memory
+// and reduce each row.  Per-tile statistics are merged in two levels by
+// atomic arrival tickets (the last CTA of a group merges the group; the last
+// group merges everything); no CTA ever waits for another.
+#include <math.h>
+
+#include "kernels.cuh"
+
+namespace tv {
+
+struct LmParams {
+    CUtensorMap tmap_w;  // (d_model, vocab), box (64, 128), 128B swizzle
+    CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad), 128B swizzle
+    int R, R_pad, D, V;
+    int n_tiles, n_kblocks, stages, tmem_cols;
+    int group_size, n_groups;
+    float4 *part_tile;   // [n_tiles][R_pad]  (max, argmax bits, s, t)
+    float4 *part_group;  // [n_groups][R_pad]
+    int *counters;       // [n_groups + 1], zero between launches
+    int *status;
+    int32_t *argmax;
+    float *top1;
+    float *entropy;
+};
+
+struct RowStat {
+    float m;  // running max logit
+    int idx;  // its vocab index (lowest on ties)
+    float s;  // sum e^(z - m)
+    float t;  // sum e^(z - m) (z - m)
+};
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ RowStat stat_empty()
+{
+    return RowStat{-INFINITY, 0x7fffffff, 0.f, 0.f};
+}
+
+// Combines the statistics of two disjoint vocab subsets.
+__device__ __forceinline__ RowStat stat_merge(RowStat a, RowStat b)
+{
+    if (b.m > a.m || (b.m == a.m && b.idx < a.idx)) {
+        RowStat x = a;
+        a = b;
+        b = x;
+    }
+    if (b.s == 0.f)
+        return a;
+    const float delta = b.m - a.m;  // <= 0
+    const float e = ex2_approx(delta * kLog2e);
+    a.s += b.s * e;
+    a.t += (b.t + delta * b.s) * e;
+    return a;
+}
+
+__device__ __forceinline__ RowStat stat_shfl_xor(RowStat a, int mask)
+{
+    RowStat b;
+    b.m = __shfl_xor_sync(0xffffffffu, a.m, mask);
+    b.idx = __shfl_xor_sync(0xffffffffu, a.idx, mask);
+    b.s = __shfl_xor_sync(0xffffffffu, a.s, mask);
+    b.t = __shfl_xor_sync(0xffffffffu, a.t, mask);
+    return b;
+}
+
+__device__ __forceinline__ RowStat warp_merge(RowStat a)
+{
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1)
+        a = stat_merge(a, stat_shfl_xor(a, m));
+    return a;
+}
+
+__device__ __forceinline__ float4 stat_pack(RowStat a)
+{
+    return make_float4(a.m, __int_as_float(a.idx), a.s, a.t);
+}
+
+__device__ __forceinline__ RowStat stat_unpack(float4 v)
+{
+    return RowStat{v.x, __float_as_int(v.y), v.z, v.w};
+}
+
+// Copies count x R_pad partials (global, written by other CTAs) into shared
+// memory, then each warp merges rows warp, warp+4, ...  Writes either the
+// merged partial (dst != nullptr) or the final per-row outputs.
+__device__ void merge_partials(const LmParams &p, const float4 *src, int count, float4 *sbuf, float4 *dst)
+{
+    const int n = count * p.R_pad;
+    for (int i = threadIdx.x; i < n; i += blockDim.x)
+        sbuf[i] = __ldcg(src + i);
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int r = warp; r < p.R; r += 4) {
+        RowStat acc = stat_empty();
+        for (int k = lane; k < count; k += 32)
+            acc = stat_merge(acc, stat_unpack(sbuf[k * p.R_pad + r]));
+        acc = warp_merge(acc);
+        if (lane == 0) {
+            if (dst) {
+                dst[r] = stat_pack(acc);
+            } else {
+                p.argmax[r] = acc.idx;
+                p.top1[r] = 1.0f / acc.s;
+                p.entropy[r] = logf(acc.s) - acc.t / acc.s;
+            }
+        }
+    }
+    __syncthreads();
+}
+
+__global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[8];
+    __shared__ __align__(8) uint64_t empty_bar[8];
+    __shared__ __align__(8) uint64_t acc_bar;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+    __shared__ int ticket;
+
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = p.stages;
+    const uint32_t h_bytes = (uint32_t)p.R_pad * 128u;
+    uint8_t *sW = smem;
+    uint8_t *sH = smem + (size_t)S * 16384;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tile = blockIdx.x;
+    const int v0 = tile * 128;
+    const int nk = p.n_kblocks;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        mbar_init(&acc_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&p.tmap_w);
+        prefetch_tmap(&p.tmap_h);
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, (uint32_t)p.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer
+        int issued = 0;
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % S;
+            const uint32_t ph = (uint32_t)(kb / S) & 1u;
+            if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
+                break;
+            mbar_arrive_expect_tx(&full_bar[s], 16384u + h_bytes);
+            tma_load_2d(sW + (size_t)s * 16384, &p.tmap_w, &full_bar[s], kb * 64, v0);
+            tma_load_2d(sH + (size_t)s * h_bytes, &p.tmap_h, &full_bar[s], kb * 64, 0);
+            issued = kb + 1;
+        }
+        if (issued < nk) {
+            // gave up: let the copies already in flight land before the CTA exits
+            for (int kb = (issued > S ? issued - S : 0); kb < issued; ++kb)
+                mbar_wait_drain(&full_bar[kb % S], (uint32_t)(kb / S) & 1u);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer
+        constexpr uint32_t kIdescM = 128;
+        const uint32_t idesc = idesc_bf16_f32(kIdescM, p.R_pad);
+        for (int kb = 0; kb < nk; ++kb) {
+            const int s = kb % S;
+            const uint32_t ph = (uint32_t)(kb / S) & 1u;
+            if (!mbar_wait_bounded(&full_bar[s], ph, &abort_flag, p.status))
+                break;
+            tc_fence_after();
+            const uint32_t a_base = smem_u32(sW + (size_t)s * 16384);
+            const uint32_t b_base = smem_u32(sH + (size_t)s * h_bytes);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const uint64_t a = smem_desc_sw128(a_base + k * 32, 0, 1024);
+                const uint64_t b = smem_desc_sw128(b_base + k * 32, 0, 1024);
+                tc_mma_f16_ss(tmem, a, b, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
+            tc_commit(&empty_bar[s]);
+        }
+        tc_commit(&acc_bar);
+    }
+    __syncwarp();
+
+    // ---------------- epilogue: TMEM -> shared (transposed) -> per-row stats
+    mbar_wait_bounded(&acc_bar, 0, &abort_flag, p.status);
+    tc_fence_after();
+    __syncthreads();
+    const bool ok = (abort_flag == 0);
+    float *logits = reinterpret_cast<float *>(smem);  // [R_pad][128], aliases the drained ring
+    if (ok) {
+        const uint32_t row_addr = tmem + ((uint32_t)(32 * warp) << 16);
+        for (int c0 = 0; c0 < p.R_pad; c0 += 16) {
+            uint32_t r[16];
+            tmem_ld_32x32b_x16(row_addr + (uint32_t)c0, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                logits[(c0 + j) * 128 + 32 * warp + lane] = __uint_as_float(r[j]);
+        }
+    } else if (warp == 1 && lane == 0) {
+        mbar_wait_drain(&acc_bar, 0);  // MMAs issued before giving up must finish before dealloc
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1)
+        tmem_dealloc(tmem, (uint32_t)p.tmem_cols);
+    if (!ok)
+        return;
+
+    for (int r = warp; r < p.R; r += 4) {
+        RowStat st = stat_empty();
+        float z[4];
+        bool valid[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int j = lane + 32 * k;
+            z[k] = logits[r * 128 + j];
+            valid[k] = (v0 + j) < p.V;
+            if (valid[k] && z[k] > st.m) {
+                st.m = z[k];
+                st.idx = v0 + j;
+            }
+        }
+        if (st.idx != 0x7fffffff) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (valid[k]) {
+                    const float dz = z[k] - st.m;
+                    const float e = ex2_approx(dz * kLog2e);
+                    st.s += e;
+                    st.t += e * dz;
+                }
+        }
+        st = warp_merge(st);
+        if (lane == 0)
+            p.part_tile[(size_t)tile * p.R_pad + r] = stat_pack(st);
+    }
+
+    // ---------------- two-level merge by arrival tickets
+    __threadfence();
+    __syncthreads();
+    const int g = tile / p.group_size;
+    const int g_first = g * p.group_size;
+    const int g_count = min(p.group_size, p.n_tiles - g_first);
+    if (threadIdx.x == 0)
+        ticket = atomicAdd(&p.counters[g], 1);
+    __syncthreads();
+    if (ticket != g_count - 1)
+        return;
+    __threadfence();
+    float4 *sbuf = reinterpret_cast<float4 *>(smem);
+    merge_partials(p, p.part_tile + (size_t)g_first * p.R_pad, g_count, sbuf, p.part_group + (size_t)g * p.R_pad);
+    if (threadIdx.x == 0)
+        p.counters[g] = 0;
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0)
+        ticket = atomicAdd(&p.counters[p.n_groups], 1);
+    __syncthreads();
+    if (ticket != p.n_groups - 1)
+        return;
+    __threadfence();
+    merge_partials(p, p.part_group, p.n_groups, sbuf, nullptr);
+    if (threadIdx.x == 0)
+        p.counters[p.n_groups] = 0;
+}
+
+// ----------------------------------------------------------------------------
+// host side
+
+static int ceil_div(int a, int b)
+{
+    return (a + b - 1) / b;
+}
+
+LmPlan lm_plan(int R, int D, int V)
+{
+    LmPlan pl{};
+    pl.R_pad = ceil_div(R, 16) * 16;
+    pl.n_tiles = ceil_div(V, 128);
+    pl.n_kblocks = ceil_div(D, 64);
+    const int stage_bytes = 16384 + pl.R_pad * 128;
+    pl.stages = (110 * 1024) / stage_bytes;
+    if (pl.stages > 8)
+        pl.stages = 8;
+    if (pl.stages < 2)
+        pl.stages = 2;
+    int cols = 32;
+    while (cols < pl.R_pad)
+        cols *= 2;
+    pl.tmem_cols = cols;
+    int gs = 1;
+    while (gs * gs < pl.n_tiles)
+        ++gs;
+    pl.group_size = gs;
+    pl.n_groups = ceil_div(pl.n_tiles, gs);
+    size_t pipe = (size_t)pl.stages * stage_bytes;
+    size_t tr = (size_t)pl.R_pad * 128 * 4;
+    size_t mg = (size_t)(gs > pl.n_groups ? gs : pl.n_groups) * pl.R_pad * 16;
+    size_t sm = pipe;
+    if (tr > sm)
+        sm = tr;
+    if (mg > sm)
+        sm = mg;
+    pl.smem_bytes = sm + 1024;
+    pl.ws_bytes = ((size_t)pl.n_tiles * pl.R_pad * 16 + (size_t)pl.n_groups * pl.R_pad * 16 + 255) / 256 * 256;
+    return pl;
+}
+
+cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
+                           float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
+                           const char **err)
+{
+    const LmPlan pl = lm_plan(R, D, V);
+    LmParams p{};
+    if (!make_tmap_2d(&p.tmap_w, W, (uint64_t)D, (uint64_t)V, (uint64_t)D * 2, 64, 128, err))
+        return cudaErrorInvalidValue;
+    if (!make_tmap_2d(&p.tmap_h, hidden, (uint64_t)D, (uint64_t)R, (uint64_t)D * 2, 64, (uint32_t)pl.R_pad, err))
+        return cudaErrorInvalidValue;
+    p.R = R;
+    p.R_pad = pl.R_pad;
+    p.D = D;
+    p.V = V;
+    p.n_tiles = pl.n_tiles;
+    p.n_kblocks = pl.n_kblocks;
+    p.stages = pl.stages;
+    p.tmem_cols = pl.tmem_cols;
+    p.group_size = pl.group_size;
+    p.n_groups = pl.n_groups;
+    p.part_tile = static_cast<float4 *>(parts);
+    p.part_group = p.part_tile + (size_t)pl.n_tiles * pl.R_pad;
+    p.counters = counters;
+    p.status = status;
+    p.argmax = argmax;
+    p.top1 = top1;
+    p.entropy = entropy;
+    cudaError_t e = cudaFuncSetAttribute(k2_lm_head, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
+    if (e != cudaSuccess)
+        return e;
+    k2_lm_head<<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace tv

@@ -1,0 +1,661 @@
+// treeverify.cu -- host side of the C ABI (include/treeverify.h): the
+// TopologyBank, argument validation, workspace layout, TMA tensor maps and
+// the launches of the three kernels of the verification pass.
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "kernels.cuh"
+
+namespace tv {
+
+// ------------------------------------------------------------------ errors
+
+static thread_local char g_err[512];
+
+static tb_status fail(tb_status st, const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+static tb_status ok()
+{
+    g_err[0] = 0;
+    return TB_OK;
+}
+
+static tb_status cuda_fail(cudaError_t e, const char *what)
+{
+    return fail(TB_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// ------------------------------------------------------------------ tensor maps
+
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static std::once_flag g_encode_once;
+
+static bool get_encode(const char **err)
+{
+    std::call_once(g_encode_once, [] {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    });
+    if (!g_encode) {
+        *err = "cuTensorMapEncodeTiled unavailable from the driver";
+        return false;
+    }
+    return true;
+}
+
+bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                  uint32_t box_inner, uint32_t box_outer, const char **err)
+{
+    if (!get_encode(err))
+        return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled (2-D) rejected the tensor";
+        return false;
+    }
+    return true;
+}
+
+bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_heads, int n_layers,
+                  int64_t head_stride, int64_t layer_stride, const char **err)
+{
+    if (!get_encode(err))
+        return false;
+    cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)n_keys, (cuuint64_t)n_heads, (cuuint64_t)n_layers};
+    cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)head_stride * 2, (cuuint64_t)layer_stride * 2};
+    cuuint32_t box[4] = {64, 64, 1, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled (KV cache) rejected the tensor";
+        return false;
+    }
+    return true;
+}
+
+// ------------------------------------------------------------------ workspace layout
+//
+//   [0, 256)                    status word
+//   [256, 256 + 64 KiB)         attention unit counters (16384 int32)
+//   [.., + 4 KiB)               LM-head group counters (1024 int32)
+//   [kPartBase, ..)             attention partials, then LM-head partials
+// Counters sit at fixed offsets so that calls of different shapes sharing one
+// workspace always find them zero; partials are written before they are read.
+
+constexpr size_t kAttnCounterOff = 256;
+constexpr int kMaxAttnUnits = 16384;
+constexpr size_t kLmCounterOff = kAttnCounterOff + (size_t)kMaxAttnUnits * 4;
+constexpr int kMaxLmCounters = 1024;
+constexpr size_t kPartBase = kLmCounterOff + (size_t)kMaxLmCounters * 4;
+
+static size_t align256(size_t x)
+{
+    return (x + 255) / 256 * 256;
+}
+
+static size_t attn_part_bytes(int P, int d)
+{
+    return align256((size_t)P * 2 * attn_slot_floats(d) * 4);
+}
+
+static int sm_count(int device)
+{
+    static std::mutex mu;
+    static std::vector<int> cache;
+    std::lock_guard<std::mutex> lk(mu);
+    if (device < 0)
+        return 0;
+    if ((int)cache.size() <= device)
+        cache.resize(device + 1, 0);
+    if (cache[device] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
+            return 0;
+        cache[device] = n;
+    }
+    return cache[device];
+}
+
+static int current_device()
+{
+    int d = -1;
+    if (cudaGetDevice(&d) != cudaSuccess)
+        return -1;
+    return d;
+}
+
+static bool aligned16(const void *p)
+{
+    return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
+}
+
+}  // namespace tv
+
+using namespace tv;
+
+// ------------------------------------------------------------------ bank
+
+struct tb_bank {
+    int device;
+    int capacity;
+    int count;
+    TreeDesc *d_desc;
+    std::vector<TreeDesc> h_desc;
+    std::vector<int32_t> h_parent;  // canonical parents, capacity x 64
+};
+
+extern "C" tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
+                                     int32_t *depth, uint64_t *anc)
+{
+    if (!parent)
+        return fail(TB_EINVAL, "tb_canonicalize: parent is NULL");
+    if (n < 1 || n > TB_MAX_NODES)
+        return fail(TB_EINVAL, "tb_canonicalize: n=%d outside 1..%d", n, TB_MAX_NODES);
+    if (parent[0] != -1)
+        return fail(TB_EINVAL, "tb_canonicalize: parent[0] must be -1 (node 0 is the root)");
+    int children_count[TB_MAX_NODES] = {0};
+    for (int i = 1; i < n; ++i) {
+        if (parent[i] < 0 || parent[i] >= n || parent[i] == i)
+            return fail(TB_EINVAL, "tb_canonicalize: parent[%d]=%d out of range", i, parent[i]);
+        ++children_count[parent[i]];
+    }
+    // breadth-first from the root, children in increasing original index
+    int queue[TB_MAX_NODES];
+    int newid[TB_MAX_NODES];
+    for (int i = 0; i < n; ++i)
+        newid[i] = -1;
+    int head = 0, tail = 0;
+    queue[tail++] = 0;
+    newid[0] = 0;
+    while (head < tail) {
+        const int x = queue[head++];
+        for (int c = 1; c < n; ++c)
+            if (parent[c] == x && newid[c] < 0) {
+                newid[c] = tail;
+                queue[tail++] = c;
+            }
+    }
+    if (tail != n)
+        return fail(TB_EINVAL, "tb_canonicalize: %d of %d nodes are not reachable from the root (cycle)", n - tail,
+                    n);
+    int32_t cpar[TB_MAX_NODES], cdep[TB_MAX_NODES];
+    uint64_t canc[TB_MAX_NODES];
+    for (int c = 0; c < n; ++c) {
+        const int orig = queue[c];
+        cpar[c] = (c == 0) ? -1 : newid[parent[orig]];
+        cdep[c] = (c == 0) ? 0 : cdep[cpar[c]] + 1;
+        canc[c] = (1ull << c) | (c == 0 ? 0ull : canc[cpar[c]]);
+    }
+    for (int c = 0; c < n; ++c) {
+        if (order)
+            order[c] = queue[c];
+        if (bfs_parent)
+            bfs_parent[c] = cpar[c];
+        if (depth)
+            depth[c] = cdep[c];
+        if (anc)
+            anc[c] = canc[c];
+    }
+    return ok();
+}
+
+extern "C" tb_status tb_create(tb_bank **out, int max_topologies, int device)
+{
+    if (!out)
+        return fail(TB_EINVAL, "tb_create: out is NULL");
+    *out = nullptr;
+    if (max_topologies < 1 || max_topologies > 4096)
+        return fail(TB_EINVAL, "tb_create: max_topologies=%d outside 1..4096", max_topologies);
+    int ndev = 0;
+    cudaError_t e = cudaGetDeviceCount(&ndev);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_create: cudaGetDeviceCount");
+    if (device < 0 || device >= ndev)
+        return fail(TB_EINVAL, "tb_create: device %d outside 0..%d", device, ndev - 1);
+    int prev = current_device();
+    if ((e = cudaSetDevice(device)) != cudaSuccess)
+        return cuda_fail(e, "tb_create: cudaSetDevice");
+    tb_bank *b = new (std::nothrow) tb_bank();
+    if (!b)
+        return fail(TB_ENOMEM, "tb_create: host allocation failed");
+    b->device = device;
+    b->capacity = max_topologies;
+    b->count = 0;
+    b->d_desc = nullptr;
+    e = cudaMalloc(&b->d_desc, sizeof(TreeDesc) * (size_t)max_topologies);
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        delete b;
+        return fail(TB_ENOMEM, "tb_create: cudaMalloc of %zu bytes: %s", sizeof(TreeDesc) * (size_t)max_topologies,
+                    cudaGetErrorString(e));
+    }
+    b->h_desc.resize(max_topologies);
+    b->h_parent.assign((size_t)max_topologies * TB_MAX_NODES, -1);
+    *out = b;
+    return ok();
+}
+
+extern "C" tb_status tb_add_topology(tb_bank *bank, const int32_t *parent, int n, int *out_id, int32_t *order)
+{
+    if (!bank || !out_id)
+        return fail(TB_EINVAL, "tb_add_topology: NULL bank or out_id");
+    if (bank->count >= bank->capacity)
+        return fail(TB_ECAPACITY, "tb_add_topology: bank full (%d topologies)", bank->capacity);
+    int32_t ord[TB_MAX_NODES], bp[TB_MAX_NODES], dep[TB_MAX_NODES];
+    uint64_t anc[TB_MAX_NODES];
+    tb_status st = tb_canonicalize(parent, n, ord, bp, dep, anc);
+    if (st != TB_OK)
+        return st;
+    TreeDesc t;
+    memset(&t, 0, sizeof t);
+    t.n = n;
+    int md = 0;
+    for (int c = 0; c < n; ++c) {
+        t.anc[c] = anc[c];
+        t.parent[c] = (int8_t)bp[c];
+        t.depth[c] = (int8_t)dep[c];
+        if (dep[c] > md)
+            md = dep[c];
+    }
+    t.max_depth = md;
+    const int id = bank->count;
+    int prev = current_device();
+    cudaError_t e = cudaSetDevice(bank->device);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(bank->d_desc + id, &t, sizeof t, cudaMemcpyHostToDevice);
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_add_topology: upload");
+    bank->h_desc[id] = t;
+    for (int c = 0; c < n; ++c)
+        bank->h_parent[(size_t)id * TB_MAX_NODES + c] = bp[c];
+    bank->count = id + 1;
+    if (order)
+        memcpy(order, ord, sizeof(int32_t) * n);
+    *out_id = id;
+    return ok();
+}
+
+extern "C" tb_status tb_get_topology(const tb_bank *bank, int id, int *n, int32_t *parent, int32_t *depth,
+                                     uint64_t *anc)
+{
+    if (!bank)
+        return fail(TB_EINVAL, "tb_get_topology: bank is NULL");
+    if (id < 0 || id >= bank->count)
+        return fail(TB_ENOTFOUND, "tb_get_topology: no topology %d (bank holds %d)", id, bank->count);
+    const TreeDesc &t = bank->h_desc[id];
+    if (n)
+        *n = t.n;
+    for (int c = 0; c < t.n; ++c) {
+        if (parent)
+            parent[c] = bank->h_parent[(size_t)id * TB_MAX_NODES + c];
+        if (depth)
+            depth[c] = t.depth[c];
+        if (anc)
+            anc[c] = t.anc[c];
+    }
+    return ok();
+}
+
+extern "C" tb_status tb_destroy(tb_bank *bank)
+{
+    if (!bank)
+        return ok();
+    int prev = current_device();
+    cudaError_t e = cudaSetDevice(bank->device);
+    if (e == cudaSuccess && bank->d_desc)
+        e = cudaFree(bank->d_desc);
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    delete bank;
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_destroy");
+    return ok();
+}
+
+extern "C" const char *tb_last_error(void)
+{
+    return g_err;
+}
+
+// ------------------------------------------------------------------ workspace
+
+extern "C" size_t tb_workspace_size(int max_rows, int n_layers, int n_kv_heads, int n_q_heads, int head_dim,
+                                    int vocab, int device)
+{
+    (void)n_layers;
+    (void)n_kv_heads;
+    (void)n_q_heads;
+    if (device < 0)
+        device = current_device();
+    const int nsm = sm_count(device);
+    if (nsm <= 0)
+        return 0;
+    size_t bytes = kPartBase;
+    if (head_dim > 0)
+        bytes += attn_part_bytes(2 * nsm, head_dim);
+    if (max_rows > 0 && vocab > 0)
+        bytes += align256(lm_plan(max_rows, 64, vocab).ws_bytes);
+    return bytes;
+}
+
+extern "C" tb_status tb_workspace_init(void *workspace, size_t workspace_bytes, tb_stream stream)
+{
+    if (!workspace)
+        return fail(TB_EINVAL, "tb_workspace_init: workspace is NULL");
+    cudaError_t e = cudaMemsetAsync(workspace, 0, workspace_bytes, (cudaStream_t)stream);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_workspace_init");
+    return ok();
+}
+
+extern "C" tb_status tb_workspace_status(const void *workspace, int32_t *status)
+{
+    if (!workspace || !status)
+        return fail(TB_EINVAL, "tb_workspace_status: NULL argument");
+    int32_t w = 0;
+    cudaError_t e = cudaMemcpy(&w, workspace, sizeof w, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_workspace_status");
+    *status = (w & kStatusTimeout) ? TB_ETIMEOUT : (w & kStatusBadToken) ? TB_EINVAL : TB_OK;
+    return ok();
+}
+
+// ------------------------------------------------------------------ validation helpers
+
+static tb_status check_bank(const tb_bank *bank, int id, const char *fn)
+{
+    if (!bank)
+        return fail(TB_EINVAL, "%s: bank is NULL", fn);
+    if (id < 0 || id >= bank->count)
+        return fail(TB_ENOTFOUND, "%s: bank_id %d not in bank (holds %d)", fn, id, bank->count);
+    if (current_device() != bank->device)
+        return fail(TB_EINVAL, "%s: current device %d is not the bank's device %d", fn, current_device(),
+                    bank->device);
+    return TB_OK;
+}
+
+static tb_status check_kv(const tb_kv *kv, int N, const char *fn)
+{
+    if (!kv || !kv->k || !kv->v)
+        return fail(TB_EINVAL, "%s: kv, kv->k or kv->v is NULL", fn);
+    if (!aligned16(kv->k) || !aligned16(kv->v))
+        return fail(TB_EINVAL, "%s: kv->k / kv->v must be 16-byte aligned", fn);
+    if (kv->head_dim != 64 && kv->head_dim != 128)
+        return fail(TB_EUNSUPPORTED, "%s: head_dim %d (64 or 128 supported)", fn, kv->head_dim);
+    if (kv->n_layers < 1 || kv->n_kv_heads < 1)
+        return fail(TB_EINVAL, "%s: n_layers=%d n_kv_heads=%d", fn, kv->n_layers, kv->n_kv_heads);
+    if (kv->L < 0 || kv->L_cap < 1)
+        return fail(TB_EINVAL, "%s: L=%d L_cap=%d", fn, kv->L, kv->L_cap);
+    if ((long long)kv->L + N > kv->L_cap)
+        return fail(TB_ECAPACITY, "%s: L + N = %lld exceeds L_cap %d", fn, (long long)kv->L + N, kv->L_cap);
+    if (kv->head_stride % 8 || kv->layer_stride % 8)
+        return fail(TB_EINVAL, "%s: strides must be multiples of 8 elements", fn);
+    if (kv->head_stride < (int64_t)kv->L_cap * kv->head_dim)
+        return fail(TB_EINVAL, "%s: head_stride %lld < L_cap * head_dim", fn, (long long)kv->head_stride);
+    if (kv->n_layers > 1 && kv->layer_stride < (int64_t)kv->n_kv_heads * kv->head_stride)
+        return fail(TB_EINVAL, "%s: layer_stride %lld overlaps heads", fn, (long long)kv->layer_stride);
+    return TB_OK;
+}
+
+static tb_status check_ws(void *ws, size_t bytes, size_t need, const char *fn)
+{
+    if (!ws)
+        return fail(TB_EINVAL, "%s: workspace is NULL", fn);
+    if (!aligned16(ws))
+        return fail(TB_EINVAL, "%s: workspace must be 16-byte aligned", fn);
+    if (bytes < need)
+        return fail(TB_ECAPACITY, "%s: workspace of %zu bytes, %zu needed", fn, bytes, need);
+    return TB_OK;
+}
+
+// ------------------------------------------------------------------ stages
+
+struct AttnArgs {
+    const tb_bank *bank;
+    int bank_id;
+    const tb_kv *kv;
+    int layer_begin, n_layers;
+    const void *q;
+    int Hq;
+    void *out;
+};
+
+static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan)
+{
+    tb_status st = check_bank(a.bank, a.bank_id, fn);
+    if (st != TB_OK)
+        return st;
+    const int N = a.bank->h_desc[a.bank_id].n;
+    if ((st = check_kv(a.kv, N, fn)) != TB_OK)
+        return st;
+    if (!a.q || !a.out || !aligned16(a.q) || !aligned16(a.out))
+        return fail(TB_EINVAL, "%s: q / out NULL or not 16-byte aligned", fn);
+    if (a.layer_begin < 0 || a.n_layers < 1 || a.layer_begin + a.n_layers > a.kv->n_layers)
+        return fail(TB_EINVAL, "%s: layers [%d, %d) outside the cache's %d", fn, a.layer_begin,
+                    a.layer_begin + a.n_layers, a.kv->n_layers);
+    if (a.Hq < a.kv->n_kv_heads || a.Hq % a.kv->n_kv_heads)
+        return fail(TB_EINVAL, "%s: n_q_heads %d not a multiple of n_kv_heads %d", fn, a.Hq, a.kv->n_kv_heads);
+    if (N * (a.Hq / a.kv->n_kv_heads) > 256)
+        return fail(TB_EUNSUPPORTED, "%s: N * group = %d > 256 query rows per kv head", fn,
+                    N * (a.Hq / a.kv->n_kv_heads));
+    const int nsm = sm_count(a.bank->device);
+    *plan = attn_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
+    if (plan->n_units > kMaxAttnUnits)
+        return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, plan->n_units, kMaxAttnUnits);
+    return TB_OK;
+}
+
+static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn)
+{
+    const char *err = "";
+    const int N = a.bank->h_desc[a.bank_id].n;
+    cudaError_t e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
+                                reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
+                                reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
+    if (e == cudaErrorInvalidValue && err[0])
+        return fail(TB_EINVAL, "%s: %s", fn, err);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return TB_OK;
+}
+
+static tb_status lm_validate(const void *hidden, int R, const void *W, int D, int V, const void *am, const void *t1,
+                             const void *en, const char *fn, LmPlan *plan)
+{
+    if (!hidden || !W || !am || !t1 || !en)
+        return fail(TB_EINVAL, "%s: NULL LM-head argument", fn);
+    if (!aligned16(hidden) || !aligned16(W))
+        return fail(TB_EINVAL, "%s: hidden / lm_head must be 16-byte aligned", fn);
+    if (R < 1 || R > 256)
+        return fail(TB_EUNSUPPORTED, "%s: %d rows (1..256 supported)", fn, R);
+    if (D < 8 || D % 8)
+        return fail(TB_EINVAL, "%s: d_model %d must be a positive multiple of 8", fn, D);
+    if (V < 1)
+        return fail(TB_EINVAL, "%s: vocab %d", fn, V);
+    *plan = lm_plan(R, D, V);
+    if (plan->n_groups + 1 > kMaxLmCounters)
+        return fail(TB_EUNSUPPORTED, "%s: vocab %d too large", fn, V);
+    return TB_OK;
+}
+
+static tb_status lm_enqueue(const void *hidden, int R, const void *W, int D, int V, int32_t *am, float *t1, float *en,
+                            uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn)
+{
+    const char *err = "";
+    cudaError_t e = lm_head_launch(hidden, R, W, D, V, am, t1, en, ws + part_off,
+                                   reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws), stream,
+                                   &err);
+    if (e == cudaErrorInvalidValue && err[0])
+        return fail(TB_EINVAL, "%s: %s", fn, err);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return TB_OK;
+}
+
+static AcceptParams accept_params(const tb_bank *bank, int id, const int32_t *draft, const int32_t *argmax, int vocab,
+                                  int L, tb_result *result, const int *ws_status)
+{
+    AcceptParams p{};
+    p.tree = bank->d_desc + id;
+    p.draft = draft;
+    p.argmax = argmax;
+    p.vocab = vocab;
+    p.L = L;
+    p.result = result;
+    p.ws_status = ws_status;
+    return p;
+}
+
+static void add_compaction(AcceptParams &p, const tb_kv *kv)
+{
+    p.k = static_cast<uint8_t *>(kv->k);
+    p.v = static_cast<uint8_t *>(kv->v);
+    p.layer_stride_b = (long long)kv->layer_stride * 2;
+    p.head_stride_b = (long long)kv->head_stride * 2;
+    p.n_layers = kv->n_layers;
+    p.n_kv_heads = kv->n_kv_heads;
+    p.row_bytes = kv->head_dim * 2;
+    p.L = kv->L;
+    p.L_cap = kv->L_cap;
+}
+
+// ------------------------------------------------------------------ entry points
+
+extern "C" tb_status tree_attention(const tb_bank *bank, int bank_id, const tb_kv *kv, int layer_begin, int n_layers,
+                                    const void *q, int n_q_heads, void *out, void *workspace, size_t workspace_bytes,
+                                    tb_stream stream)
+{
+    const char *fn = "tree_attention";
+    AttnArgs a{bank, bank_id, kv, layer_begin, n_layers, q, n_q_heads, out};
+    AttnPlan plan;
+    tb_status st = attn_validate(a, fn, &plan);
+    if (st != TB_OK)
+        return st;
+    const size_t need = kPartBase + attn_part_bytes(plan.P, kv->head_dim);
+    if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
+        return st;
+    if ((st = attn_enqueue(a, static_cast<uint8_t *>(workspace), kPartBase, (cudaStream_t)stream, fn)) != TB_OK)
+        return st;
+    return ok();
+}
+
+extern "C" tb_status lm_head_stats(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
+                                   int32_t *argmax, float *top1, float *entropy, void *workspace,
+                                   size_t workspace_bytes, tb_stream stream)
+{
+    const char *fn = "lm_head_stats";
+    LmPlan plan;
+    tb_status st = lm_validate(hidden, n_rows, lm_head, d_model, vocab, argmax, top1, entropy, fn, &plan);
+    if (st != TB_OK)
+        return st;
+    if ((st = check_ws(workspace, workspace_bytes, kPartBase + plan.ws_bytes, fn)) != TB_OK)
+        return st;
+    if ((st = lm_enqueue(hidden, n_rows, lm_head, d_model, vocab, argmax, top1, entropy,
+                         static_cast<uint8_t *>(workspace), kPartBase, (cudaStream_t)stream, fn)) != TB_OK)
+        return st;
+    return ok();
+}
+
+extern "C" tb_status greedy_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens,
+                                   const int32_t *argmax, int vocab, int L, tb_result *result, tb_stream stream)
+{
+    const char *fn = "greedy_accept";
+    tb_status st = check_bank(bank, bank_id, fn);
+    if (st != TB_OK)
+        return st;
+    if (!draft_tokens || !argmax || !result)
+        return fail(TB_EINVAL, "%s: NULL argument", fn);
+    if (vocab < 1 || L < 0)
+        return fail(TB_EINVAL, "%s: vocab=%d L=%d", fn, vocab, L);
+    AcceptParams p = accept_params(bank, bank_id, draft_tokens, argmax, vocab, L, result, nullptr);
+    cudaError_t e = accept_launch(p, sm_count(bank->device), (cudaStream_t)stream);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
+}
+
+extern "C" tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream)
+{
+    const char *fn = "kv_compact";
+    tb_status st = check_kv(kv, 0, fn);
+    if (st != TB_OK)
+        return st;
+    if (!result)
+        return fail(TB_EINVAL, "%s: result is NULL", fn);
+    AcceptParams p{};
+    p.result = const_cast<tb_result *>(result);
+    p.from_result = 1;
+    add_compaction(p, kv);
+    cudaError_t e = accept_launch(p, sm_count(current_device()), (cudaStream_t)stream);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
+}
+
+extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q, int n_q_heads,
+                                 const void *hidden, const void *lm_head, int d_model, int vocab,
+                                 const int32_t *draft_tokens, void *attn_out, int32_t *argmax, float *top1,
+                                 float *entropy, tb_result *result, void *workspace, size_t workspace_bytes, int flags,
+                                 tb_stream stream)
+{
+    const char *fn = "verify_step";
+    AttnArgs a{bank, bank_id, kv, 0, kv ? kv->n_layers : 0, q, n_q_heads, attn_out};
+    AttnPlan aplan;
+    tb_status st = attn_validate(a, fn, &aplan);
+    if (st != TB_OK)
+        return st;
+    const int N = bank->h_desc[bank_id].n;
+    LmPlan lplan;
+    if ((st = lm_validate(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
+        return st;
+    if (!draft_tokens || !result)
+        return fail(TB_EINVAL, "%s: draft_tokens / result is NULL", fn);
+    const size_t attn_bytes = attn_part_bytes(aplan.P, kv->head_dim);
+    const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
+    if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
+        return st;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = (cudaStream_t)stream;
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s,
+                         fn)) != TB_OK)
+        return st;
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+        return st;
+    AcceptParams p =
+        accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
+    if (!(flags & TB_NO_COMPACT))
+        add_compaction(p, kv);
+    cudaError_t e = accept_launch(p, sm_count(bank->device), s);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
+}
