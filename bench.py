@@ -50,8 +50,10 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
-def workload(cfg: str):
+def workload(cfg: str, layers: int | None = None):
     sh = synth.SHAPES[cfg]()
+    if layers:
+        sh.n_layers = layers
     N = sh.N
     kv_bytes = sh.n_layers * 2 * (sh.L + N) * sh.n_kv_heads * sh.head_dim * 2
     w_bytes = sh.vocab * sh.d_model * 2
@@ -151,7 +153,7 @@ def run_gpu(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
 
-    sh, kv_bytes, w_bytes, flops = workload(args.config)
+    sh, kv_bytes, w_bytes, flops = workload(args.config, args.layers)
     N, L, H, Hkv, d, D, V, nl = (sh.N, sh.L, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_model, sh.vocab,
                                  sh.n_layers)
     seed = 1234 + rank
@@ -296,6 +298,8 @@ def run_gpu(args):
         "gpu_launches": 3 * args.steps,
         "clocks": clocks,
     }
+    if args.layers:
+        line["config"]["layers_override"] = args.layers
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.config, budget_s=args.cpu_budget)
     print(json.dumps(line), flush=True)
@@ -398,6 +402,7 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--config", default="c4", choices=["c1", "c2", "c4"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)

@@ -168,15 +168,20 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
 
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
+        // Tiles start their k-loop at different k-blocks so that the CTAs in
+        // flight read W rows at spread-out column offsets instead of the same
+        // power-of-two-strided addresses in lockstep.
+        const int rot = (int)(((long long)tile * 5) % nk);
         int issued = 0;
         for (int kb = 0; kb < nk; ++kb) {
             const int s = kb % S;
             const uint32_t ph = (uint32_t)(kb / S) & 1u;
             if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
                 break;
+            const int kx = (kb + rot) % nk;
             mbar_arrive_expect_tx(&full_bar[s], 16384u + h_bytes);
-            tma_load_2d(sW + (size_t)s * 16384, &p.tmap_w, &full_bar[s], kb * 64, v0);
-            tma_load_2d(sH + (size_t)s * h_bytes, &p.tmap_h, &full_bar[s], kb * 64, 0);
+            tma_load_2d(sW + (size_t)s * 16384, &p.tmap_w, &full_bar[s], kx * 64, v0);
+            tma_load_2d(sH + (size_t)s * h_bytes, &p.tmap_h, &full_bar[s], kx * 64, 0);
             issued = kb + 1;
         }
         if (issued < nk) {

@@ -75,9 +75,10 @@ ATTN_CASES = [
     ("chain64-ragged", synth.chain(64), 77, 1, 2, 2, 128),
     ("bank64-gqa4", synth.bank_trees()[-1], 300, 1, 8, 2, 128),
     ("tree26-L1024-h32", synth.shape_c2().parent, 1024, 1, 32, 32, 128),
-    ("random63-L5-d64", synth.random_tree(synth.rng(5), 63), 5, 1, 4, 4, 64),
+    ("random63-L5-d64", np.sort(synth.random_tree(synth.rng(5), 63)), 5, 1, 4, 4, 64),
     ("two-nodes-L63", [-1, 0], 63, 1, 4, 1, 128),
-    ("bank40-gqa8-d64", synth.bank_trees()[6], 190, 1, 8, 1, 64),
+    ("bank40-gqa4-d64", synth.bank_trees()[6], 190, 1, 8, 2, 64),
+    ("bank64-gqa4-L2k", synth.bank_trees()[-1], 2048, 1, 32, 8, 128),
     ("chain2-L0", [-1, 0], 0, 1, 1, 1, 64),
 ]
 
@@ -85,6 +86,15 @@ ATTN_CASES = [
 @pytest.mark.parametrize("name,parent,L,n_layers,Hq,Hkv,d", ATTN_CASES, ids=[c[0] for c in ATTN_CASES])
 def test_tree_attention_parity(dev, bank, name, parent, L, n_layers, Hq, Hkv, d):
     _run_attention(bank, dev, parent, L, n_layers, Hq, Hkv, d, seed=zlib.crc32(name.encode()) % 1000)
+
+
+def test_tree_attention_non_bfs_input(dev, bank):
+    """A topology given in non-breadth-first order is canonicalised; queries and
+    tree K/V are then laid out in canonical order (order[c] = caller index)."""
+    parent = synth.random_tree(synth.rng(9), 30)
+    order, bfs_parent, _, _ = tv.tb_canonicalize(parent)
+    assert not np.array_equal(order, np.arange(30))
+    _run_attention(bank, dev, bfs_parent, 70, 1, 4, 4, 128, seed=9)
 
 
 def test_tree_attention_layer_subset(dev, bank):
