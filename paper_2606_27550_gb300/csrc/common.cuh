@@ -8,7 +8,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/treeverify.h"
+#include "treeverify.h"
 
 namespace tv {
 

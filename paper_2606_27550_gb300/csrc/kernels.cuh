@@ -7,7 +7,7 @@ namespace tv {
 
 // LM head (lm_head.cu)
 struct LmPlan {
-    int R_pad, n_tiles, n_kblocks, stages, tmem_cols, group_size, n_groups;
+    int R_pad, n_tiles, n_kblocks, stages, tmem_cols, group_size, n_groups, bps;
     size_t smem_bytes;
     size_t ws_bytes;  // partials (tile + group), 256-byte aligned
 };
@@ -44,6 +44,9 @@ struct AcceptParams {
     int from_result;  // compaction driven by an existing result (kv_compact): no acceptance
 };
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
+
+// sets the message returned by tb_last_error() on this thread (treeverify.cu)
+tb_status record_error(tb_status st, const char *fmt, ...);
 
 // tensor maps (treeverify.cu)
 bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,

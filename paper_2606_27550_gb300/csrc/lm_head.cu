@@ -18,6 +18,7 @@
 // atomic arrival tickets (the last CTA of a group merges the group; the last
 // group merges everything); no CTA ever waits for another.
 #include <math.h>
+#include <stdlib.h>
 
 #include "kernels.cuh"
 
@@ -28,6 +29,7 @@ struct LmParams {
     CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad), 128B swizzle
     int R, R_pad, D, V;
     int n_tiles, n_kblocks, stages, tmem_cols;
+    int bps;             // 64-column boxes per pipeline stage
     int group_size, n_groups;
     float4 *part_tile;   // [n_tiles][R_pad]  (max, argmax bits, s, t)
     float4 *part_group;  // [n_groups][R_pad]
@@ -137,14 +139,16 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = p.stages;
-    const uint32_t h_bytes = (uint32_t)p.R_pad * 128u;
+    const int B = p.bps;
+    const uint32_t hb = (uint32_t)p.R_pad * 128u;  // one hidden-row box
+    const uint32_t w_stage = 16384u * B, h_stage = hb * B;
     uint8_t *sW = smem;
-    uint8_t *sH = smem + (size_t)S * 16384;
+    uint8_t *sH = smem + (size_t)S * w_stage;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tile = blockIdx.x;
     const int v0 = tile * 128;
-    const int nk = p.n_kblocks;
+    const int nk = p.n_kblocks;  // stages of B boxes
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -167,10 +171,11 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     const uint32_t tmem = tmem_slot;
 
     if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer
-        // Tiles start their k-loop at different k-blocks so that the CTAs in
-        // flight read W rows at spread-out column offsets instead of the same
-        // power-of-two-strided addresses in lockstep.
+        // ---------------- TMA producer: one stage = B adjacent 64-column boxes of
+        // W (128 rows) and of the hidden rows, so each W row is fetched as a
+        // contiguous run of B x 128 bytes.
+        // Tiles start their k-loop at different stages so that the CTAs in
+        // flight read W rows at spread-out column offsets.
         const int rot = (int)(((long long)tile * 5) % nk);
         int issued = 0;
         for (int kb = 0; kb < nk; ++kb) {
@@ -179,9 +184,12 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
                 break;
             const int kx = (kb + rot) % nk;
-            mbar_arrive_expect_tx(&full_bar[s], 16384u + h_bytes);
-            tma_load_2d(sW + (size_t)s * 16384, &p.tmap_w, &full_bar[s], kx * 64, v0);
-            tma_load_2d(sH + (size_t)s * h_bytes, &p.tmap_h, &full_bar[s], kx * 64, 0);
+            mbar_arrive_expect_tx(&full_bar[s], w_stage + h_stage);
+            for (int b = 0; b < B; ++b) {
+                const int x = (kx * B + b) * 64;
+                tma_load_2d(sW + (size_t)s * w_stage + (size_t)b * 16384, &p.tmap_w, &full_bar[s], x, v0);
+                tma_load_2d(sH + (size_t)s * h_stage + (size_t)b * hb, &p.tmap_h, &full_bar[s], x, 0);
+            }
             issued = kb + 1;
         }
         if (issued < nk) {
@@ -199,13 +207,15 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             if (!mbar_wait_bounded(&full_bar[s], ph, &abort_flag, p.status))
                 break;
             tc_fence_after();
-            const uint32_t a_base = smem_u32(sW + (size_t)s * 16384);
-            const uint32_t b_base = smem_u32(sH + (size_t)s * h_bytes);
+            for (int b = 0; b < B; ++b) {
+                const uint32_t a_base = smem_u32(sW + (size_t)s * w_stage + (size_t)b * 16384);
+                const uint32_t b_base = smem_u32(sH + (size_t)s * h_stage + (size_t)b * hb);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const uint64_t a = smem_desc_sw128(a_base + k * 32, 0, 1024);
-                const uint64_t b = smem_desc_sw128(b_base + k * 32, 0, 1024);
-                tc_mma_f16_ss(tmem, a, b, idesc, (kb | k) != 0 ? 1u : 0u);
+                for (int k = 0; k < 4; ++k) {
+                    const uint64_t a = smem_desc_sw128(a_base + k * 32, 0, 1024);
+                    const uint64_t bd = smem_desc_sw128(b_base + k * 32, 0, 1024);
+                    tc_mma_f16_ss(tmem, a, bd, idesc, (kb | b | k) != 0 ? 1u : 0u);
+                }
             }
             tc_commit(&empty_bar[s]);
         }
@@ -305,13 +315,24 @@ static int ceil_div(int a, int b)
     return (a + b - 1) / b;
 }
 
+// Boxes per stage: the widest contiguous W run per row that still leaves two
+// stages per CTA and two CTAs per SM.
+static int lm_boxes_per_stage(int R_pad)
+{
+    const char *env = getenv("TV_LM_BPS");
+    if (env && atoi(env) >= 1 && atoi(env) <= 4)
+        return atoi(env);
+    return 1;
+}
+
 LmPlan lm_plan(int R, int D, int V)
 {
     LmPlan pl{};
     pl.R_pad = ceil_div(R, 16) * 16;
     pl.n_tiles = ceil_div(V, 128);
-    pl.n_kblocks = ceil_div(D, 64);
-    const int stage_bytes = 16384 + pl.R_pad * 128;
+    pl.bps = lm_boxes_per_stage(pl.R_pad);
+    pl.n_kblocks = ceil_div(D, 64 * pl.bps);
+    const int stage_bytes = (16384 + pl.R_pad * 128) * pl.bps;
     pl.stages = (110 * 1024) / stage_bytes;
     if (pl.stages > 8)
         pl.stages = 8;
@@ -355,6 +376,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.V = V;
     p.n_tiles = pl.n_tiles;
     p.n_kblocks = pl.n_kblocks;
+    p.bps = pl.bps;
     p.stages = pl.stages;
     p.tmem_cols = pl.tmem_cols;
     p.group_size = pl.group_size;

@@ -28,6 +28,15 @@ static tb_status fail(tb_status st, const char *fmt, ...)
     return st;
 }
 
+tb_status record_error(tb_status st, const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
 static tb_status ok()
 {
     g_err[0] = 0;
