@@ -210,6 +210,27 @@ TB_API tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, 
                       float *top1, float *entropy, tb_result *result, void *workspace,
                       size_t workspace_bytes, int flags, tb_stream stream);
 
+/* lm_head_stats for callers that cannot allocate device memory.  Code that
+ * runs inside a host framework which owns every device allocation, in a
+ * sandbox that forbids cudaMalloc, or next to a memory pool that is already
+ * fully carved up has no way to provide the workspace that lm_head_stats
+ * needs.  This variant computes the same argmax / top1 / entropy with the
+ * same kernel, but keeps its scratch in a 4 MiB array compiled into the
+ * library (every GPU that loads the library holds it until the process
+ * exits); it calls no cudaMalloc, cudaFree or allocating library routine.
+ *  - The first call on a device looks up that array's device address
+ *    (cudaGetSymbolAddress) with the device current; make that first call
+ *    before capturing the stream into a graph.
+ *  - Every call clears the array's arrival counters on `stream` and reuses the
+ *    array, which keeps the previous call's partial results: calls that can
+ *    overlap on the GPU (different streams without ordering) race.
+ *  - Shapes whose scratch exceeds the array (n_rows x vocab partials larger
+ *    than 4 MiB) are rejected with TB_ECAPACITY before anything is enqueued.
+ * Arguments, layouts and tolerances are those of lm_head_stats.  The paper has
+ * no counterpart: this is an integration convenience of this library. */
+TB_API tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
+                                       int32_t *argmax, float *top1, float *entropy, tb_stream stream);
+
 /* Message for the last failing call on this thread ("" if none). */
 TB_API const char *tb_last_error(void);
 

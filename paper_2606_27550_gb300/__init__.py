@@ -28,7 +28,7 @@ RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
-       "kv_compact", "verify_step", "tb_last_error")
+       "kv_compact", "verify_step", "lm_head_stats_noalloc", "tb_last_error")
 
 
 class TreeVerifyError(RuntimeError):
@@ -69,6 +69,7 @@ def load(path: str = LIB_PATH):
         "greedy_accept": [P, i32, P, P, i32, i32, P, P],
         "kv_compact": [P, P, P],
         "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
+        "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, P],
         "tb_last_error": [],
     }
     for name, args in sig.items():
@@ -252,3 +253,11 @@ def verify_step(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft
                               _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(draft), _ptr(attn_out),
                               _ptr(argmax), _ptr(top1), _ptr(entropy), _ptr(result), _ptr(ws), ws.numel(), flags,
                               _stream(stream)), "verify_step")
+
+
+def lm_head_stats_noalloc(hidden, lm_head, argmax, top1, entropy, stream=None):
+    """lm_head_stats with the library's built-in scratch array instead of a
+    caller workspace, for callers that cannot allocate device memory."""
+    R, D = hidden.shape
+    _check(load().lm_head_stats_noalloc(_ptr(hidden), R, _ptr(lm_head), D, lm_head.shape[0], _ptr(argmax),
+                                        _ptr(top1), _ptr(entropy), _stream(stream)), "lm_head_stats_noalloc")
