@@ -123,20 +123,27 @@ class ClockSampler:
 def traffic_from_profiles(kernel: str):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if its
     source hash still matches the current kernel source (else None)."""
-    import hashlib
-
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
     for ln in open(path):
         f = ln.split()
         if len(f) >= 4 and f[0] == kernel and not ln.startswith("#"):
-            src = os.path.join(ROOT, "paper_2606_27550_gb300", "csrc", f[1])
-            if not os.path.exists(src):
-                return None
-            h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-            return float(f[3]) if h == f[2] else None
+            return float(f[3]) if kernel_source_hash(f[1]) == f[2] else None
     return None
+
+
+def kernel_source_hash(files: str) -> str:
+    """sha256[:16] over the comma-separated csrc files a kernel is built from."""
+    import hashlib
+
+    h = hashlib.sha256()
+    for name in files.split(","):
+        src = os.path.join(ROOT, "paper_2606_27550_gb300", "csrc", name)
+        if not os.path.exists(src):
+            return ""
+        h.update(open(src, "rb").read())
+    return h.hexdigest()[:16]
 
 
 def run_gpu(args):
@@ -209,6 +216,9 @@ def run_gpu(args):
     # per-kernel durations: the same work through the stage entry points, events between stages
     n_k = max(3, min(args.steps, 50))
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_k)]
+    # keep the GPU busy while the host enqueues, so that the events bracket
+    # device time only (no host launch gaps between stages)
+    torch.cuda._sleep(200_000_000)
     for i in range(n_k):
         ev[i][0].record(stream)
         tv.lm_head_stats(hidden, W, am, t1, en, ws, stream)

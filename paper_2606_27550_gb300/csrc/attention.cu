@@ -438,10 +438,10 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
     const AttnPlan pl = attn_plan(kv->L, N, Hq, kv->n_kv_heads, n_layers, n_sm);
     AttnParams p{};
     if (!make_tmap_kv(&p.tmap_k, kv->k, d, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
-                      kv->layer_stride, err))
+                      kv->layer_stride, 64, err))
         return cudaErrorInvalidValue;
     if (!make_tmap_kv(&p.tmap_v, kv->v, d, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
-                      kv->layer_stride, err))
+                      kv->layer_stride, 64, err))
         return cudaErrorInvalidValue;
     p.q = static_cast<const __nv_bfloat16 *>(q);
     p.out = static_cast<__nv_bfloat16 *>(out);
@@ -466,13 +466,11 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
     const size_t smem = attn_smem_bytes(d);
     cudaError_t e;
     if (d == 128) {
-        e = cudaFuncSetAttribute(k1_tree_attention<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
+        if ((e = allow_max_smem((const void *)k1_tree_attention<128>)) != cudaSuccess)
             return e;
         k1_tree_attention<128><<<pl.P, 160, smem, stream>>>(p);
     } else {
-        e = cudaFuncSetAttribute(k1_tree_attention<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess)
+        if ((e = allow_max_smem((const void *)k1_tree_attention<64>)) != cudaSuccess)
             return e;
         k1_tree_attention<64><<<pl.P, 160, smem, stream>>>(p);
     }

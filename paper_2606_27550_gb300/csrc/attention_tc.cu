@@ -1,0 +1,616 @@
+// attention_tc.cu -- tree-masked attention on the 5th-generation tensor cores
+// (K1, head_dim 128).
+//
+// Same operation and work split as attention.cu (tree decoding, Sec. 3.2;
+// ancestor-bitset mask, Sec. 2.3; flattened (layer, kv head, row block) x
+// key-tile space split evenly over a persistent grid, ticketed log-sum-exp
+// merge of split units), with the contractions on tcgen05:
+//
+//   S   = Q K^T   tcgen05.mma kind::f16, M = 128 query rows, N = 128 keys,
+//                 K = 128 = head_dim; Q and the K tile are 128-byte-swizzled
+//                 K-major shared-memory operands; S accumulates in TMEM.
+//   O  += P V     M = 128 rows, N = 128 = head_dim, K = 128 keys; P (bf16)
+//                 is the TMEM A operand, the V tile an MN-major shared-memory
+//                 operand; O accumulates in TMEM.
+//
+// One CTA per SM, 6 warps:
+//   warp 0       TMA producer: 128-key K and V tiles (4 boxes of 64 x 128)
+//                through a 3-stage mbarrier ring.
+//   warp 1       TMEM allocation (512 columns) and the single MMA-issuing
+//                thread; S of tile i+1 is issued before O += P V of tile i so
+//                that the softmax of tile i overlaps the next QK^T.
+//   warps 2-5    one thread per query row (TMEM lane): row max, exp2 with a
+//                lazily rescaled reference maximum (O and l are rescaled only
+//                when the maximum grows by more than 2^8), P written back to
+//                TMEM, and the segment epilogue (normalise, or write a partial
+//                for the merge).
+// TMEM columns: S0 [0,128), S1 [128,256), P0 [256,320), P1 [320,384),
+// O [384,512).  Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that
+// the rows are spread over the four lane quadrants (all four SM sub-partitions
+// share the softmax).
+#include "kernels.cuh"
+
+namespace tv {
+
+namespace {
+
+constexpr int kD = 128;            // head_dim
+constexpr int kBN = 128;           // keys per tile
+constexpr int kStages = 3;
+constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
+constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
+constexpr int kStage = 2 * kTile;  // K + V
+constexpr int kQBytes = 2 * kAtom;
+constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
+constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 256, kColP1 = 320, kColO = 384;
+constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
+
+struct TcParams {
+    CUtensorMap tmap_k;  // (128, L + N, Hkv, layers), box (64, 128, 1, 1), 128B swizzle
+    CUtensorMap tmap_v;
+    const __nv_bfloat16 *q;
+    __nv_bfloat16 *out;
+    const TreeDesc *tree;
+    int L, N, Hq, Hkv, group, layer_begin, n_layers;
+    int rows, row_blocks, T, n_units;
+    long long total;
+    int P;
+    float scale_log2;
+    float *part;
+    int *counters;
+    int *status;
+};
+
+__device__ __forceinline__ long long tc_seg_begin(const TcParams &p, int c)
+{
+    return (long long)c * p.total / p.P;
+}
+
+__device__ __forceinline__ int tc_cta_of(const TcParams &p, long long t)
+{
+    return (int)(((t + 1) * (long long)p.P - 1) / p.total);
+}
+
+// MN-major (N contiguous) 128-byte-swizzled operand: lbo = stride between
+// 64-element column atoms, sbo = stride between groups of 8 K rows.
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t lbo, uint32_t sbo)
+{
+    return smem_desc_sw128(addr, lbo, sbo);
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
+    __shared__ __align__(8) uint64_t q_full, o_free, drain_bar, epi_written, epi_ticket;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+    __shared__ int ticket;
+
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sQ = smem;
+    uint8_t *sKV = smem + kQBytes;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = blockIdx.x;
+    const long long t0 = tc_seg_begin(p, c), t1 = tc_seg_begin(p, c + 1);
+    const long long n_tiles = t1 - t0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&s_full[b], 1);
+            mbar_init(&s_free[b], 4);
+            mbar_init(&p_full[b], 4);
+            mbar_init(&pv_done[b], 1);
+        }
+        mbar_init(&q_full, 4);
+        mbar_init(&o_free, 4);
+        mbar_init(&drain_bar, 1);
+        mbar_init(&epi_written, 4);
+        mbar_init(&epi_ticket, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&p.tmap_k);
+        prefetch_tmap(&p.tmap_v);
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            long long issued = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
+                const int s = (int)(it % kStages);
+                const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+                if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
+                    break;
+                const long long t = t0 + it;
+                const int u = (int)(t / p.T);
+                const int j = (int)(t % p.T);
+                const int head = (u / p.row_blocks) % p.Hkv;
+                const int layer = p.layer_begin + u / (p.row_blocks * p.Hkv);
+                uint8_t *sk = sKV + (size_t)s * kStage;
+                uint8_t *sv = sk + kTile;
+                mbar_arrive_expect_tx(&full_bar[s], kStage);
+                tma_load_4d(sk, &p.tmap_k, &full_bar[s], 0, j * kBN, head, layer);
+                tma_load_4d(sk + kAtom, &p.tmap_k, &full_bar[s], 64, j * kBN, head, layer);
+                tma_load_4d(sv, &p.tmap_v, &full_bar[s], 0, j * kBN, head, layer);
+                tma_load_4d(sv + kAtom, &p.tmap_v, &full_bar[s], 64, j * kBN, head, layer);
+                issued = it + 1;
+            }
+            if (issued < n_tiles)
+                for (long long it = (issued > kStages ? issued - kStages : 0); it < issued; ++it)
+                    mbar_wait_drain(&full_bar[it % kStages], (uint32_t)(it / kStages) & 1u);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc_s = idesc_bf16_f32(128, kBN);
+            const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
+            const uint32_t q_base = smem_u32(sQ);
+            int sg = -1;
+            // the pending O += P V (tile it - 1)
+            bool pend = false, pend_first = false;
+            int pend_sg = 0;
+            long long pend_it = 0;
+            bool ok = true;
+            auto issue_pv = [&](long long j, bool first, int seg) -> bool {
+                const int bj = (int)(j & 1);
+                if (!mbar_wait_bounded(&p_full[bj], (uint32_t)(j >> 1) & 1u, &abort_flag, p.status))
+                    return false;
+                if (first && seg > 0 &&
+                    !mbar_wait_bounded(&o_free, (uint32_t)(seg - 1) & 1u, &abort_flag, p.status))
+                    return false;
+                tc_fence_after();
+                const uint32_t v_base = smem_u32(sKV + (size_t)(j % kStages) * kStage + kTile);
+                const uint32_t p_col = bj ? kColP1 : kColP0;
+#pragma unroll
+                for (int ks = 0; ks < kBN / 16; ++ks) {
+                    const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
+                    tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
+                }
+                tc_commit(&empty_bar[j % kStages]);
+                tc_commit(&pv_done[bj]);
+                return true;
+            };
+            for (long long it = 0; it < n_tiles && ok; ++it) {
+                const long long t = t0 + it;
+                const bool first = (it == 0) || (t % p.T == 0);
+                if (first)
+                    ++sg;
+                const int s = (int)(it % kStages);
+                const int b = (int)(it & 1);
+                if (first && pend) {
+                    // finish the previous unit first: its epilogue frees O for this one
+                    if (!issue_pv(pend_it, pend_first, pend_sg)) {
+                        ok = false;
+                        break;
+                    }
+                    pend = false;
+                }
+                if (!mbar_wait_bounded(&full_bar[s], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status) ||
+                    !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
+                    (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status))) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t k_base = smem_u32(sKV + (size_t)s * kStage);
+                const uint32_t s_col = b ? kColS1 : kColS0;
+#pragma unroll
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                    const uint32_t off = (uint32_t)(kk >> 2) * kAtom + (uint32_t)(kk & 3) * 32;
+                    const uint64_t adesc = smem_desc_sw128(q_base + off, 0, 1024);
+                    const uint64_t bdesc = smem_desc_sw128(k_base + off, 0, 1024);
+                    tc_mma_f16_ss(tmem + s_col, adesc, bdesc, idesc_s, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(&s_full[b]);
+                if (pend && !issue_pv(pend_it, pend_first, pend_sg)) {
+                    ok = false;
+                    break;
+                }
+                pend = true;
+                pend_it = it;
+                pend_first = first;
+                pend_sg = sg;
+            }
+            if (ok && pend)
+                issue_pv(pend_it, pend_first, pend_sg);
+            // arrives when every MMA issued above has retired (waited for before TMEM is released)
+            tc_commit(&drain_bar);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax / epilogue (warps 2-5)
+        const int q4 = warp & 3;  // TMEM lane quadrant of this warp
+        const uint32_t lane_addr = tmem + ((uint32_t)(32 * q4) << 16);
+        const int rloc = 4 * lane + q4;  // query row of this thread within the block
+        const int arow = 32 * q4 + lane;  // its A-operand row (= TMEM lane)
+
+        struct Seg {
+            long long start, end, u_first, u_last;
+            int u, rb, head, layer_rel, rows_here, node, qh;
+            bool valid;
+            uint64_t anc;
+        };
+        auto describe = [&](long long t) {
+            Seg g;
+            g.start = t;
+            g.u = (int)(t / p.T);
+            g.u_first = (long long)g.u * p.T;
+            g.u_last = g.u_first + p.T;
+            g.end = t1 < g.u_last ? t1 : g.u_last;
+            g.rb = g.u % p.row_blocks;
+            g.head = (g.u / p.row_blocks) % p.Hkv;
+            g.layer_rel = g.u / (p.row_blocks * p.Hkv);
+            g.rows_here = min(128, p.rows - g.rb * 128);
+            g.valid = rloc < g.rows_here;
+            const int grow = g.rb * 128 + rloc;
+            g.node = g.valid ? grow / p.group : 0;
+            g.qh = g.head * p.group + grow % p.group;
+            g.anc = g.valid ? p.tree->anc[g.node] : 0ull;
+            return g;
+        };
+        // Q row of this thread -> shared memory (A-row arow, 128-byte swizzle); zeros for padding rows
+        auto write_q = [&](const Seg &g) {
+            const uint4 *src =
+                reinterpret_cast<const uint4 *>(p.q + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+#pragma unroll
+            for (int ch = 0; ch < 16; ++ch) {
+                const uint4 v = g.valid ? src[ch] : make_uint4(0, 0, 0, 0);
+                const int h = ch >> 3, cc = ch & 7;
+                *reinterpret_cast<uint4 *>(sQ + h * kAtom + arow * 128 + ((cc ^ (arow & 7)) << 4)) = v;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&q_full);
+        };
+        long long it = 0;
+        int n_partial = 0;  // partial segments so far (phase of epi_written / epi_ticket)
+        bool aborted = (n_tiles == 0);
+        Seg g;
+        if (!aborted) {
+            g = describe(t0);
+            write_q(g);
+        }
+        while (!aborted) {
+            float m_ref = -INFINITY, l = 0.f;
+            for (long long t = g.start; t < g.end; ++t, ++it) {
+                const int b = (int)(it & 1);
+                if (!mbar_wait_bounded(&s_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status)) {
+                    aborted = true;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = lane_addr + (b ? kColS1 : kColS0);
+                const int key0 = (int)(t - g.u_first) * kBN;
+                const bool masked = key0 + kBN > p.L;
+
+                // pass 1: the whole S row (4 loads, one wait), masked row max
+                float sc[kBN];
+                {
+                    uint32_t *r = reinterpret_cast<uint32_t *>(sc);
+                    tmem_ld_32x32b_x32(sa, r);
+                    tmem_ld_32x32b_x32(sa + 32, r + 32);
+                    tmem_ld_32x32b_x32(sa + 64, r + 64);
+                    tmem_ld_32x32b_x32(sa + 96, r + 96);
+                    tmem_ld_wait();
+                }
+                float mx = -INFINITY;
+                if (masked) {
+#pragma unroll
+                    for (int x = 0; x < kBN; ++x) {
+                        const int tj = key0 + x - p.L;
+                        const bool ok = tj < 0 || (tj < p.N && ((g.anc >> tj) & 1ull));
+                        sc[x] = ok ? sc[x] : -INFINITY;
+                        mx = fmaxf(mx, sc[x]);
+                    }
+                } else {
+#pragma unroll
+                    for (int x = 0; x < kBN; ++x)
+                        mx = fmaxf(mx, sc[x]);
+                }
+                mx *= p.scale_log2;  // row max in log2 units (scale > 0)
+
+                // lazily rescaled reference maximum
+                float alpha = 1.f;
+                bool rescale = false;
+                if (t == g.start) {
+                    m_ref = mx;
+                } else if (mx > m_ref + kRescaleLog2) {
+                    alpha = (m_ref == -INFINITY) ? 0.f : ex2_approx(m_ref - mx);
+                    m_ref = mx;
+                    rescale = true;
+                }
+                if (__any_sync(0xffffffffu, rescale)) {
+                    // O holds the previous tiles' P V: wait for the last one, then scale in place
+                    const long long jp = it - 1;
+                    if (!mbar_wait_bounded(&pv_done[jp & 1], (uint32_t)(jp >> 1) & 1u, &abort_flag, p.status)) {
+                        aborted = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    l *= alpha;
+#pragma unroll 1
+                    for (int c0 = 0; c0 < kD; c0 += 32) {
+                        uint32_t o[32];
+                        tmem_ld_32x32b_x32(lane_addr + kColO + c0, o);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int x = 0; x < 32; ++x)
+                            o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
+                        tmem_st_32x32b_x32(lane_addr + kColO + c0, o);
+                    }
+                    tmem_st_wait();
+                }
+                // P buffer b was last read by O += P V of tile it - 2
+                if (it >= 2 &&
+                    !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) {
+                    aborted = true;
+                    break;
+                }
+                tc_fence_after();
+
+                // pass 2: P = 2^(s * scale - m_ref) as bf16 pairs into TMEM (masked entries are
+                // -inf and give 0), row sum into l
+                const float mu = (m_ref == -INFINITY) ? 0.f : m_ref;
+                const uint32_t pa = lane_addr + (b ? kColP1 : kColP0);
+                float rs = 0.f;
+#pragma unroll
+                for (int c0 = 0; c0 < kBN; c0 += 32) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) {
+                        const float p0 = ex2_approx(fmaf(sc[c0 + 2 * x], p.scale_log2, -mu));
+                        const float p1 = ex2_approx(fmaf(sc[c0 + 2 * x + 1], p.scale_log2, -mu));
+                        rs += p0 + p1;
+                        pk[x] = pack_bf16x2(p0, p1);
+                    }
+                    tmem_st_32x32b_x16(pa + c0 / 2, pk);
+                }
+                l += rs;
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&s_free[b]);
+                    mbar_arrive(&p_full[b]);
+                }
+            }
+            if (aborted)
+                break;
+
+            // Every QK^T of this segment has been consumed, so Q can take the next unit's rows
+            // now, letting the next segment's first QK^T overlap this epilogue.
+            const bool has_next = g.end < t1;
+            Seg nx;
+            if (has_next) {
+                nx = describe(g.end);
+                write_q(nx);
+            }
+
+            // ---------------------------------------------------- segment epilogue
+            const long long jl = it - 1;
+            if (!mbar_wait_bounded(&pv_done[jl & 1], (uint32_t)(jl >> 1) & 1u, &abort_flag, p.status))
+                break;
+            tc_fence_after();
+            const bool whole = (g.start == g.u_first && g.end == g.u_last);
+            float *slot = p.part + ((size_t)c * 2 + (g.start == t0 ? 0 : 1)) * kSlot;
+            {
+                const float inv = 1.f / l;
+                uint4 *dst =
+                    reinterpret_cast<uint4 *>(p.out + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+                float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
+#pragma unroll 1
+                for (int c0 = 0; c0 < kD; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32b_x32(lane_addr + kColO + c0, r);
+                    tmem_ld_wait();
+                    if (!g.valid)
+                        continue;
+                    if (whole) {
+#pragma unroll
+                        for (int ch = 0; ch < 4; ++ch) {
+                            uint4 v;
+                            v.x = pack_bf16x2(__uint_as_float(r[8 * ch + 0]) * inv, __uint_as_float(r[8 * ch + 1]) * inv);
+                            v.y = pack_bf16x2(__uint_as_float(r[8 * ch + 2]) * inv, __uint_as_float(r[8 * ch + 3]) * inv);
+                            v.z = pack_bf16x2(__uint_as_float(r[8 * ch + 4]) * inv, __uint_as_float(r[8 * ch + 5]) * inv);
+                            v.w = pack_bf16x2(__uint_as_float(r[8 * ch + 6]) * inv, __uint_as_float(r[8 * ch + 7]) * inv);
+                            dst[c0 / 8 + ch] = v;
+                        }
+                    } else {
+#pragma unroll
+                        for (int x = 0; x < 8; ++x)
+                            pdst[c0 / 4 + x] = make_float4(__uint_as_float(r[4 * x]), __uint_as_float(r[4 * x + 1]),
+                                                           __uint_as_float(r[4 * x + 2]), __uint_as_float(r[4 * x + 3]));
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&o_free);
+
+            if (!whole) {
+                // partial (O, m_ref, l) is in this CTA's slot; take the unit's arrival ticket
+                if (g.valid) {
+                    slot[128 * kD + rloc] = m_ref;
+                    slot[128 * kD + 128 + rloc] = l;
+                }
+                // all four warps' rows written -> one ticket for the CTA -> broadcast
+                __threadfence();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&epi_written);
+                const int c_lo = tc_cta_of(p, g.u_first), c_hi = tc_cta_of(p, g.u_last - 1);
+                const uint32_t eph = (uint32_t)n_partial & 1u;
+                ++n_partial;
+                if (warp == 2 && lane == 0) {
+                    if (mbar_wait_bounded(&epi_written, eph, &abort_flag, p.status))
+                        ticket = atomicAdd(&p.counters[g.u], 1);
+                    mbar_arrive(&epi_ticket);
+                }
+                if (!mbar_wait_bounded(&epi_ticket, eph, &abort_flag, p.status))
+                    break;
+                const bool last = (ticket == c_hi - c_lo);
+                if (last) {
+                    __threadfence();
+                    if (g.valid) {
+                        float M = -INFINITY;
+                        for (int cc = c_lo; cc <= c_hi; ++cc) {
+                            const float *sl =
+                                p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
+                            M = fmaxf(M, __ldcg(sl + 128 * kD + rloc));
+                        }
+                        float lsum = 0.f;
+                        for (int cc = c_lo; cc <= c_hi; ++cc) {
+                            const float *sl =
+                                p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
+                            const float ms = __ldcg(sl + 128 * kD + rloc);
+                            lsum += (ms == -INFINITY) ? 0.f : ex2_approx(ms - M) * __ldcg(sl + 128 * kD + 128 + rloc);
+                        }
+                        const float inv = 1.f / lsum;
+                        uint4 *dst = reinterpret_cast<uint4 *>(
+                            p.out + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+#pragma unroll 1
+                        for (int c0 = 0; c0 < kD; c0 += 32) {
+                            float acc[32];
+#pragma unroll
+                            for (int x = 0; x < 32; ++x)
+                                acc[x] = 0.f;
+                            for (int cc = c_lo; cc <= c_hi; ++cc) {
+                                const float *sl =
+                                    p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
+                                const float ms = __ldcg(sl + 128 * kD + rloc);
+                                const float w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M) * inv;
+                                const float4 *src = reinterpret_cast<const float4 *>(sl + rloc * kD + c0);
+#pragma unroll
+                                for (int x = 0; x < 8; ++x) {
+                                    const float4 v = __ldcg(src + x);
+                                    acc[4 * x] += w * v.x;
+                                    acc[4 * x + 1] += w * v.y;
+                                    acc[4 * x + 2] += w * v.z;
+                                    acc[4 * x + 3] += w * v.w;
+                                }
+                            }
+#pragma unroll
+                            for (int ch = 0; ch < 4; ++ch) {
+                                uint4 v;
+                                v.x = pack_bf16x2(acc[8 * ch + 0], acc[8 * ch + 1]);
+                                v.y = pack_bf16x2(acc[8 * ch + 2], acc[8 * ch + 3]);
+                                v.z = pack_bf16x2(acc[8 * ch + 4], acc[8 * ch + 5]);
+                                v.w = pack_bf16x2(acc[8 * ch + 6], acc[8 * ch + 7]);
+                                dst[c0 / 8 + ch] = v;
+                            }
+                        }
+                    }
+                    if (warp == 2 && lane == 0)
+                        p.counters[g.u] = 0;
+                }
+            }
+            if (!has_next)
+                break;
+            g = nx;
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        if (lane == 0)
+            mbar_wait_drain(&drain_bar, 0);
+        __syncwarp();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// ----------------------------------------------------------------------------
+// host side
+
+static size_t tc_smem_bytes()
+{
+    return (size_t)kQBytes + (size_t)kStages * kStage + 1024;
+}
+
+bool attn_tc_supported(int d, int rows)
+{
+    (void)rows;
+    return d == kD;
+}
+
+AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm)
+{
+    AttnPlan pl{};
+    pl.group = Hq / Hkv;
+    pl.rows = N * pl.group;
+    pl.row_blocks = (pl.rows + 127) / 128;
+    pl.T = (L + N + kBN - 1) / kBN;
+    pl.n_units = n_layers * Hkv * pl.row_blocks;
+    pl.total = (long long)pl.n_units * pl.T;
+    long long P = n_sm;
+    if (P > pl.total)
+        P = pl.total;
+    pl.P = (int)P;
+    return pl;
+}
+
+size_t attn_tc_slot_floats()
+{
+    return (size_t)kSlot;
+}
+
+cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
+                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                           cudaStream_t stream, const char **err)
+{
+    const AttnPlan pl = attn_tc_plan(kv->L, N, Hq, kv->n_kv_heads, n_layers, n_sm);
+    TcParams p{};
+    if (!make_tmap_kv(&p.tmap_k, kv->k, kD, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+                      kv->layer_stride, kBN, err))
+        return cudaErrorInvalidValue;
+    if (!make_tmap_kv(&p.tmap_v, kv->v, kD, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+                      kv->layer_stride, kBN, err))
+        return cudaErrorInvalidValue;
+    p.q = static_cast<const __nv_bfloat16 *>(q);
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.tree = d_tree;
+    p.L = kv->L;
+    p.N = N;
+    p.Hq = Hq;
+    p.Hkv = kv->n_kv_heads;
+    p.group = pl.group;
+    p.layer_begin = layer_begin;
+    p.n_layers = n_layers;
+    p.rows = pl.rows;
+    p.row_blocks = pl.row_blocks;
+    p.T = pl.T;
+    p.n_units = pl.n_units;
+    p.total = pl.total;
+    p.P = pl.P;
+    p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
+    p.part = part;
+    p.counters = counters;
+    p.status = status;
+    cudaError_t e = allow_max_smem((const void *)k1_tree_attention_tc);
+    if (e != cudaSuccess)
+        return e;
+    k1_tree_attention_tc<<<pl.P, 192, tc_smem_bytes(), stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace tv

@@ -27,6 +27,14 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
                         const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
                         cudaStream_t stream, const char **err);
 
+// tree attention on tcgen05 (attention_tc.cu): head_dim 128
+bool attn_tc_supported(int d, int rows);
+AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
+size_t attn_tc_slot_floats();
+cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
+                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                           cudaStream_t stream, const char **err);
+
 // acceptance + compaction (accept.cu)
 struct AcceptParams {
     const TreeDesc *tree;
@@ -45,6 +53,10 @@ struct AcceptParams {
 };
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
 
+// Raises a kernel's dynamic shared-memory limit to the device maximum, once
+// per (kernel, device) (treeverify.cu).
+cudaError_t allow_max_smem(const void *kernel);
+
 // sets the message returned by tb_last_error() on this thread (treeverify.cu)
 tb_status record_error(tb_status st, const char *fmt, ...);
 
@@ -52,6 +64,6 @@ tb_status record_error(tb_status st, const char *fmt, ...);
 bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                   uint32_t box_inner, uint32_t box_outer, const char **err);
 bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_heads, int n_layers,
-                  int64_t head_stride, int64_t layer_stride, const char **err);
+                  int64_t head_stride, int64_t layer_stride, int box_keys, const char **err);
 
 }  // namespace tv

@@ -81,14 +81,6 @@ __device__ __forceinline__ RowStat stat_shfl_xor(RowStat a, int mask)
     return b;
 }
 
-__device__ __forceinline__ RowStat warp_merge(RowStat a)
-{
-#pragma unroll
-    for (int m = 16; m >= 1; m >>= 1)
-        a = stat_merge(a, stat_shfl_xor(a, m));
-    return a;
-}
-
 __device__ __forceinline__ float4 stat_pack(RowStat a)
 {
     return make_float4(a.m, __int_as_float(a.idx), a.s, a.t);
@@ -99,28 +91,69 @@ __device__ __forceinline__ RowStat stat_unpack(float4 v)
     return RowStat{v.x, __float_as_int(v.y), v.z, v.w};
 }
 
-// Copies count x R_pad partials (global, written by other CTAs) into shared
-// memory, then each warp merges rows warp, warp+4, ...  Writes either the
-// merged partial (dst != nullptr) or the final per-row outputs.
+// Threads per row for per-row scans by the 128 threads of a CTA: the largest
+// power of two with tpr x R_pad <= 128 (at least 1).
+__device__ __forceinline__ int threads_per_row(int R_pad)
+{
+    int tpr = 1;
+    while (tpr * 2 * R_pad <= 128)
+        tpr *= 2;
+    return tpr;
+}
+
+// Combines the statistics held by the tpr consecutive lanes of each row group.
+__device__ __forceinline__ RowStat group_merge(RowStat st, int tpr)
+{
+    for (int m = 1; m < tpr; m <<= 1)
+        st = stat_merge(st, stat_shfl_xor(st, m));
+    return st;
+}
+
+// Merges count x R_pad partials (global, written by other CTAs): they are
+// staged in shared memory, then every row is reduced by `tpr` threads in two
+// independent passes (max / first argmax, then the rescaled sums), so there is
+// no serial dependency chain per row.  Writes the merged partial (dst) or the
+// final per-row outputs.
 __device__ void merge_partials(const LmParams &p, const float4 *src, int count, float4 *sbuf, float4 *dst)
 {
     const int n = count * p.R_pad;
     for (int i = threadIdx.x; i < n; i += blockDim.x)
         sbuf[i] = __ldcg(src + i);
     __syncthreads();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int r = warp; r < p.R; r += 4) {
-        RowStat acc = stat_empty();
-        for (int k = lane; k < count; k += 32)
-            acc = stat_merge(acc, stat_unpack(sbuf[k * p.R_pad + r]));
-        acc = warp_merge(acc);
-        if (lane == 0) {
+    const int tpr = threads_per_row(p.R_pad);
+    const int sub = threadIdx.x % tpr;
+    for (int r0 = 0; r0 < p.R; r0 += 128 / tpr) {
+        const int r = r0 + threadIdx.x / tpr;
+        RowStat st = stat_empty();
+        if (r < p.R) {
+            for (int k = sub; k < count; k += tpr) {
+                const float4 v = sbuf[k * p.R_pad + r];
+                const int idx = __float_as_int(v.y);
+                if (v.z > 0.f && (v.x > st.m || (v.x == st.m && idx < st.idx))) {
+                    st.m = v.x;
+                    st.idx = idx;
+                }
+            }
+            if (st.idx != 0x7fffffff) {
+                for (int k = sub; k < count; k += tpr) {
+                    const float4 v = sbuf[k * p.R_pad + r];
+                    if (v.z > 0.f) {
+                        const float delta = v.x - st.m;
+                        const float e = ex2_approx(delta * kLog2e);
+                        st.s += v.z * e;
+                        st.t += (v.w + delta * v.z) * e;
+                    }
+                }
+            }
+        }
+        st = group_merge(st, tpr);
+        if (sub == 0 && r < p.R) {
             if (dst) {
-                dst[r] = stat_pack(acc);
+                dst[r] = stat_pack(st);
             } else {
-                p.argmax[r] = acc.idx;
-                p.top1[r] = 1.0f / acc.s;
-                p.entropy[r] = logf(acc.s) - acc.t / acc.s;
+                p.argmax[r] = st.idx;
+                p.top1[r] = 1.0f / st.s;
+                p.entropy[r] = logf(st.s) - st.t / st.s;
             }
         }
     }
@@ -228,7 +261,11 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     tc_fence_after();
     __syncthreads();
     const bool ok = (abort_flag == 0);
-    float *logits = reinterpret_cast<float *>(smem);  // [R_pad][128], aliases the drained ring
+    // logits[r][v] at r * ld + v; the row stride 128 + tpr keeps both the
+    // column writes below and the per-row scans free of bank conflicts.
+    const int tpr = threads_per_row(p.R_pad);
+    const int ld = 128 + tpr;
+    float *logits = reinterpret_cast<float *>(smem);  // aliases the drained ring
     if (ok) {
         const uint32_t row_addr = tmem + ((uint32_t)(32 * warp) << 16);
         for (int c0 = 0; c0 < p.R_pad; c0 += 16) {
@@ -237,7 +274,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             tmem_ld_wait();
 #pragma unroll
             for (int j = 0; j < 16; ++j)
-                logits[(c0 + j) * 128 + 32 * warp + lane] = __uint_as_float(r[j]);
+                logits[(c0 + j) * ld + 32 * warp + lane] = __uint_as_float(r[j]);
         }
     } else if (warp == 1 && lane == 0) {
         mbar_wait_drain(&acc_bar, 0);  // MMAs issued before giving up must finish before dealloc
@@ -249,33 +286,33 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     if (!ok)
         return;
 
-    for (int r = warp; r < p.R; r += 4) {
-        RowStat st = stat_empty();
-        float z[4];
-        bool valid[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int j = lane + 32 * k;
-            z[k] = logits[r * 128 + j];
-            valid[k] = (v0 + j) < p.V;
-            if (valid[k] && z[k] > st.m) {
-                st.m = z[k];
-                st.idx = v0 + j;
-            }
-        }
-        if (st.idx != 0x7fffffff) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-                if (valid[k]) {
-                    const float dz = z[k] - st.m;
+    // per-row statistics of this tile: tpr threads per row, two passes
+    {
+        const int sub = threadIdx.x % tpr;
+        const int nvalid = min(128, p.V - v0);
+        for (int r0 = 0; r0 < p.R; r0 += 128 / tpr) {
+            const int r = r0 + threadIdx.x / tpr;
+            RowStat st = stat_empty();
+            if (r < p.R) {
+                const float *row = logits + r * ld;
+                for (int j = sub; j < nvalid; j += tpr) {
+                    const float z = row[j];
+                    if (z > st.m) {
+                        st.m = z;
+                        st.idx = v0 + j;
+                    }
+                }
+                for (int j = sub; j < nvalid; j += tpr) {
+                    const float dz = row[j] - st.m;
                     const float e = ex2_approx(dz * kLog2e);
                     st.s += e;
                     st.t += e * dz;
                 }
+            }
+            st = group_merge(st, tpr);
+            if (sub == 0 && r < p.R)
+                p.part_tile[(size_t)tile * p.R_pad + r] = stat_pack(st);
         }
-        st = warp_merge(st);
-        if (lane == 0)
-            p.part_tile[(size_t)tile * p.R_pad + r] = stat_pack(st);
     }
 
     // ---------------- two-level merge by arrival tickets
@@ -315,13 +352,12 @@ static int ceil_div(int a, int b)
     return (a + b - 1) / b;
 }
 
-// Boxes per stage: the widest contiguous W run per row that still leaves two
-// stages per CTA and two CTAs per SM.
+// 64-column boxes per pipeline stage.  Measured on GB300 (V=32000 and 128256,
+// 26-200 rows): one or two boxes per stage are within 3%; four boxes cost
+// stages and lose; so one box, the deepest ring.
 static int lm_boxes_per_stage(int R_pad)
 {
-    const char *env = getenv("TV_LM_BPS");
-    if (env && atoi(env) >= 1 && atoi(env) <= 4)
-        return atoi(env);
+    (void)R_pad;
     return 1;
 }
 
@@ -348,7 +384,7 @@ LmPlan lm_plan(int R, int D, int V)
     pl.group_size = gs;
     pl.n_groups = ceil_div(pl.n_tiles, gs);
     size_t pipe = (size_t)pl.stages * stage_bytes;
-    size_t tr = (size_t)pl.R_pad * 128 * 4;
+    size_t tr = (size_t)pl.R_pad * (128 + 8) * 4;
     size_t mg = (size_t)(gs > pl.n_groups ? gs : pl.n_groups) * pl.R_pad * 16;
     size_t sm = pipe;
     if (tr > sm)
@@ -388,7 +424,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.argmax = argmax;
     p.top1 = top1;
     p.entropy = entropy;
-    cudaError_t e = cudaFuncSetAttribute(k2_lm_head, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.smem_bytes);
+    cudaError_t e = allow_max_smem((const void *)k2_lm_head);
     if (e != cudaSuccess)
         return e;
     k2_lm_head<<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);

@@ -6,6 +6,7 @@
 #include <atomic>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -26,6 +27,31 @@ static tb_status fail(tb_status st, const char *fmt, ...)
     vsnprintf(g_err, sizeof g_err, fmt, ap);
     va_end(ap);
     return st;
+}
+
+cudaError_t allow_max_smem(const void *kernel)
+{
+    static std::mutex mu;
+    static std::vector<std::pair<const void *, int>> done;
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    std::lock_guard<std::mutex> lk(mu);
+    for (auto &kd : done)
+        if (kd.first == kernel && kd.second == dev)
+            return cudaSuccess;
+    int max_optin = 0;
+    if ((e = cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
+        return e;
+    cudaFuncAttributes attr;
+    if ((e = cudaFuncGetAttributes(&attr, kernel)) != cudaSuccess)
+        return e;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             max_optin - (int)attr.sharedSizeBytes);
+    if (e == cudaSuccess)
+        done.emplace_back(kernel, dev);
+    return e;
 }
 
 tb_status record_error(tb_status st, const char *fmt, ...)
@@ -90,13 +116,13 @@ bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t o
 }
 
 bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_heads, int n_layers,
-                  int64_t head_stride, int64_t layer_stride, const char **err)
+                  int64_t head_stride, int64_t layer_stride, int box_keys, const char **err)
 {
     if (!get_encode(err))
         return false;
     cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)n_keys, (cuuint64_t)n_heads, (cuuint64_t)n_layers};
     cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)head_stride * 2, (cuuint64_t)layer_stride * 2};
-    cuuint32_t box[4] = {64, 64, 1, 1};
+    cuuint32_t box[4] = {64, (cuuint32_t)box_keys, 1, 1};
     cuuint32_t estr[4] = {1, 1, 1, 1};
     CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box,
                           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -128,9 +154,19 @@ static size_t align256(size_t x)
     return (x + 255) / 256 * 256;
 }
 
-static size_t attn_part_bytes(int P, int d)
+// Partial slots of the split-L merge: two per CTA of whichever attention
+// kernel runs (the tcgen05 one for head_dim 128, else the mma.sync one).
+static size_t attn_part_bytes(int n_sm, int d)
 {
-    return align256((size_t)P * 2 * attn_slot_floats(d) * 4);
+    const size_t mma = (size_t)2 * n_sm * 2 * attn_slot_floats(d) * 4;
+    const size_t tc = attn_tc_supported(d, 0) ? (size_t)n_sm * 2 * attn_tc_slot_floats() * 4 : 0;
+    return align256(mma > tc ? mma : tc);
+}
+
+// head_dim 128 runs on the tcgen05 kernel; head_dim 64 on the mma.sync one.
+static bool use_tc_attention(int d, int rows)
+{
+    return attn_tc_supported(d, rows);
 }
 
 static int sm_count(int device)
@@ -370,7 +406,7 @@ extern "C" size_t tb_workspace_size(int max_rows, int n_layers, int n_kv_heads, 
         return 0;
     size_t bytes = kPartBase;
     if (head_dim > 0)
-        bytes += attn_part_bytes(2 * nsm, head_dim);
+        bytes += attn_part_bytes(nsm, head_dim);
     if (max_rows > 0 && vocab > 0)
         bytes += align256(lm_plan(max_rows, 64, vocab).ws_bytes);
     return bytes;
@@ -477,7 +513,9 @@ static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan
         return fail(TB_EUNSUPPORTED, "%s: N * group = %d > 256 query rows per kv head", fn,
                     N * (a.Hq / a.kv->n_kv_heads));
     const int nsm = sm_count(a.bank->device);
-    *plan = attn_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
+    const int rows = N * (a.Hq / a.kv->n_kv_heads);
+    *plan = use_tc_attention(a.kv->head_dim, rows) ? attn_tc_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm)
+                                                   : attn_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
     if (plan->n_units > kMaxAttnUnits)
         return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, plan->n_units, kMaxAttnUnits);
     return TB_OK;
@@ -487,9 +525,11 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
-    cudaError_t e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
-                                reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                                reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
+    const int rows = N * (a.Hq / a.kv->n_kv_heads);
+    auto launch = use_tc_attention(a.kv->head_dim, rows) ? attn_tc_launch : attn_launch;
+    cudaError_t e = launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
+                           reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
+                           reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -569,7 +609,7 @@ extern "C" tb_status tree_attention(const tb_bank *bank, int bank_id, const tb_k
     tb_status st = attn_validate(a, fn, &plan);
     if (st != TB_OK)
         return st;
-    const size_t need = kPartBase + attn_part_bytes(plan.P, kv->head_dim);
+    const size_t need = kPartBase + attn_part_bytes(sm_count(bank->device), kv->head_dim);
     if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
         return st;
     if ((st = attn_enqueue(a, static_cast<uint8_t *>(workspace), kPartBase, (cudaStream_t)stream, fn)) != TB_OK)
@@ -648,7 +688,7 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
         return st;
     if (!draft_tokens || !result)
         return fail(TB_EINVAL, "%s: draft_tokens / result is NULL", fn);
-    const size_t attn_bytes = attn_part_bytes(aplan.P, kv->head_dim);
+    const size_t attn_bytes = attn_part_bytes(sm_count(bank->device), kv->head_dim);
     const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
     if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
         return st;
