@@ -7,8 +7,9 @@
 // merge of split units), with the contractions on tcgen05:
 //
 //   S   = Q K^T   tcgen05.mma kind::f16, M = 128 query rows, N = 128 keys,
-//                 K = 128 = head_dim; Q and the K tile are 128-byte-swizzled
-//                 K-major shared-memory operands; S accumulates in TMEM.
+//                 K = 128 = head_dim; Q (bf16) is the TMEM A operand, the K
+//                 tile a 128-byte-swizzled K-major shared-memory operand; S
+//                 accumulates in TMEM.
 //   O  += P V     M = 128 rows, N = 128 = head_dim, K = 128 keys; P (bf16)
 //                 is the TMEM A operand, the V tile an MN-major shared-memory
 //                 operand; O accumulates in TMEM.
@@ -24,10 +25,12 @@
 //                when the maximum grows by more than 2^8), P written back to
 //                TMEM, and the segment epilogue (normalise, or write a partial
 //                for the merge).
-// TMEM columns: S0 [0,128), S1 [128,256), P0 [256,320), P1 [320,384),
-// O [384,512).  Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that
-// the rows are spread over the four lane quadrants (all four SM sub-partitions
-// share the softmax).
+// TMEM columns: S0 [0,128), S1 [128,256) with P0 / P1 aliased onto their first
+// halves, O [256,384), Q [384,448).  Both QK^T and P V take their A operand
+// from TMEM, so each MMA reads only the 128 x 16 B operand from shared memory.
+// Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that the rows
+// are spread over the four lane quadrants (all four SM sub-partitions share
+// the softmax).
 #include "kernels.cuh"
 
 namespace tv {
@@ -40,9 +43,10 @@ constexpr int kStages = 3;
 constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
 constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
 constexpr int kStage = 2 * kTile;  // K + V
-constexpr int kQBytes = 2 * kAtom;
 constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
-constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 256, kColP1 = 320, kColO = 384;
+// TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
+// softmax has read S_b into registers; Q (bf16 pairs) is the A operand of QK^T.
+constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 0, kColP1 = 128, kColO = 256, kColQ = 384;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
 
 struct TcParams {
@@ -91,8 +95,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
     __shared__ int ticket;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sQ = smem;
-    uint8_t *sKV = smem + kQBytes;
+    uint8_t *sKV = smem;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
@@ -161,7 +164,6 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         if (lane == 0) {
             const uint32_t idesc_s = idesc_bf16_f32(128, kBN);
             const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
-            const uint32_t q_base = smem_u32(sQ);
             int sg = -1;
             // the pending O += P V (tile it - 1)
             bool pend = false, pend_first = false;
@@ -214,9 +216,8 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
                     const uint32_t off = (uint32_t)(kk >> 2) * kAtom + (uint32_t)(kk & 3) * 32;
-                    const uint64_t adesc = smem_desc_sw128(q_base + off, 0, 1024);
                     const uint64_t bdesc = smem_desc_sw128(k_base + off, 0, 1024);
-                    tc_mma_f16_ss(tmem + s_col, adesc, bdesc, idesc_s, kk > 0 ? 1u : 0u);
+                    tc_mma_f16_ts(tmem + s_col, tmem + kColQ + kk * 8, bdesc, idesc_s, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[b]);
                 if (pend && !issue_pv(pend_it, pend_first, pend_sg)) {
@@ -238,7 +239,6 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         const int q4 = warp & 3;  // TMEM lane quadrant of this warp
         const uint32_t lane_addr = tmem + ((uint32_t)(32 * q4) << 16);
         const int rloc = 4 * lane + q4;  // query row of this thread within the block
-        const int arow = 32 * q4 + lane;  // its A-operand row (= TMEM lane)
 
         struct Seg {
             long long start, end, u_first, u_last;
@@ -264,17 +264,26 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             g.anc = g.valid ? p.tree->anc[g.node] : 0ull;
             return g;
         };
-        // Q row of this thread -> shared memory (A-row arow, 128-byte swizzle); zeros for padding rows
+        // Q row of this thread -> its TMEM lane as 64 columns of bf16 pairs (the A
+        // operand of QK^T); zeros for padding rows
         auto write_q = [&](const Seg &g) {
             const uint4 *src =
                 reinterpret_cast<const uint4 *>(p.q + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+#pragma unroll 1
+            for (int qc = 0; qc < 4; ++qc) {
+                uint32_t w[16];
 #pragma unroll
-            for (int ch = 0; ch < 16; ++ch) {
-                const uint4 v = g.valid ? src[ch] : make_uint4(0, 0, 0, 0);
-                const int h = ch >> 3, cc = ch & 7;
-                *reinterpret_cast<uint4 *>(sQ + h * kAtom + arow * 128 + ((cc ^ (arow & 7)) << 4)) = v;
+                for (int ch = 0; ch < 4; ++ch) {
+                    const uint4 v = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
+                    w[4 * ch] = v.x;
+                    w[4 * ch + 1] = v.y;
+                    w[4 * ch + 2] = v.z;
+                    w[4 * ch + 3] = v.w;
+                }
+                tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, w);
             }
-            fence_proxy_async_smem();
+            tmem_st_wait();
+            tc_fence_before();
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&q_full);
@@ -544,7 +553,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 
 static size_t tc_smem_bytes()
 {
-    return (size_t)kQBytes + (size_t)kStages * kStage + 1024;
+    return (size_t)kStages * kStage + 1024;
 }
 
 bool attn_tc_supported(int d, int rows)
