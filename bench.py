@@ -270,6 +270,7 @@ def run_gpu(args):
     if rank != 0:
         return
 
+    k1_name = "k1_tree_attention_tc" if d == 128 else "k1_tree_attention"
     peaks, peak_src = load_peaks()
     hbm = float(peaks["hbm_gbs"])
     ms = elapsed_ms / args.steps
@@ -296,10 +297,10 @@ def run_gpu(args):
         "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
                          "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
                          "peak_gbs": hbm, "peak_src": peak_src},
-        "roofline": {"kernel": "k1_tree_attention", "bound": "hbm", "achieved": round(at_gbs, 1), "peak": hbm,
-                     "unit": "GB/s", "frac": round(at_gbs / hbm, 4), "traffic": traffic_from_profiles("k1_tree_attention"),
+        "roofline": {"kernel": k1_name, "bound": "hbm", "achieved": round(at_gbs, 1), "peak": hbm,
+                     "unit": "GB/s", "frac": round(at_gbs / hbm, 4), "traffic": traffic_from_profiles(k1_name),
                      "algorithmic_bytes": kv_bytes, "avg_launch_ms": round(t_at, 4)},
-        "kernels_ms": {"k2_lm_head": round(t_lm, 4), "k1_tree_attention": round(t_at, 4),
+        "kernels_ms": {"k2_lm_head": round(t_lm, 4), k1_name: round(t_at, 4),
                        "k3_accept_compact": round(t_ac, 4)},
         "lm_head_gbs": round(w_bytes / (t_lm * 1e-3) / 1e9, 1),
         "accept_len_last": r["accept_len"],
