@@ -316,6 +316,110 @@ def run_gpu(args):
     print(json.dumps(line), flush=True)
 
 
+def run_gpu_batched(args):
+    """The ragged batch (verify_step_batched): 8 sequences, GQA 32/8 x 128,
+    L ~ U[512, 8192], trees of 4-64 nodes, one LM head of 4096 x 128256."""
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_27550_gb300 as tv
+    from paper_2606_27550_gb300 import build as tvbuild
+
+    world, rank, local = dist_info()
+    tvbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    sh = synth.batch_c5(seed=5)
+    Hq, Hkv, d, D, V = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_model, sh.vocab
+    bf = torch.bfloat16
+    seed = 4321 + rank
+    bank = tv.Bank(16, local)
+    W = synth.device_normal_bf16_(torch.empty((V, D), dtype=bf, device=dev), seed, std=sh.w_std)
+    R = sum(sh.Ns)
+    hidden = synth.device_normal_bf16_(torch.empty((R, D), dtype=bf, device=dev), seed + 1)
+    am = torch.empty(R, dtype=torch.int32, device=dev)
+    t1 = torch.empty(R, dtype=torch.float32, device=dev)
+    en = torch.empty(R, dtype=torch.float32, device=dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(R, 1, Hkv, Hq, d, V, local), dev)
+    # drafts from an untimed LM-head pass (rows in chunks of 256)
+    for r0 in range(0, R, 256):
+        r1 = min(R, r0 + 256)
+        tv.lm_head_stats(hidden[r0:r1], W, am[r0:r1], t1[r0:r1], en[r0:r1], ws)
+    torch.cuda.synchronize()
+    am_h = am.cpu().numpy()
+    seqs, kv_bytes, r0 = [], 0, 0
+    for b, (parent, L, pm) in enumerate(zip(sh.parents, sh.Ls, sh.p_match)):
+        N = len(parent)
+        bid, _ = bank.add(parent)
+        k = synth.device_normal_bf16_(torch.empty((1, Hkv, L + N, d), dtype=bf, device=dev), seed + 10 + 2 * b)
+        v = synth.device_normal_bf16_(torch.empty((1, Hkv, L + N, d), dtype=bf, device=dev), seed + 11 + 2 * b)
+        q = synth.device_normal_bf16_(torch.empty((1, N, Hq, d), dtype=bf, device=dev), seed + 100 + b)
+        drafts = torch.from_numpy(synth.gen_drafts(seed + b, parent, am_h[r0:r0 + N], V, pm)).to(dev)
+        seqs.append(tv.Seq(bid, tv.KvCache(k, v, L), q, drafts, torch.empty((1, N, Hq, d), dtype=bf, device=dev),
+                           tv.make_result(dev)))
+        kv_bytes += 2 * (L + N) * Hkv * d * 2
+        r0 += N
+    w_bytes = V * D * 2
+    flops = 2 * R * D * V + sum(4 * len(p) * (L + len(p)) * d * Hq for p, L in zip(sh.parents, sh.Ls))
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # KV (~0.1 GB) fits in L2: flush between steps
+    stream = torch.cuda.current_stream()
+
+    def step():
+        tv.verify_step_batched(bank, seqs, hidden, W, am, t1, en, ws, tv.TB_NO_COMPACT, stream)
+
+    sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]
+                           if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
+    sampler.start()
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    elapsed_ms = sum(a.elapsed_time(b) for a, b in ev)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    clocks = sampler.stop()
+    if world > 1:
+        dist.destroy_process_group()
+    bank.close()
+    if rank != 0:
+        return
+    peaks, peak_src = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    tflops = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    ms = elapsed_ms / args.steps
+    value = world * args.steps / (elapsed_ms / 1e3)
+    t_mem = (kv_bytes + w_bytes) / (hbm * 1e9) * 1e3
+    t_comp = flops / (tflops * 1e12) * 1e3
+    line = {
+        "metric": "verify-steps/s", "value": round(value, 3), "unit": "verify-steps/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded)",
+        "config": {"workload": sh.name, "batch": len(sh.parents), "tree_nodes": sh.Ns, "L": sh.Ls, "q_heads": Hq,
+                   "kv_heads": Hkv, "head_dim": d, "d_model": D, "vocab": V,
+                   "l2": "256 MB flush before every step (the batch's KV fits in L2)"},
+        "tree_tokens_per_s": round(value * R, 1),
+        "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
+                     "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
+                     "flops_per_step": flops, "peak_gbs": hbm, "peak_tflops_sustained": tflops, "peak_src": peak_src},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+
+
 # ----------------------------------------------------------------------------- CPU oracle (reference arm)
 
 
@@ -411,7 +515,7 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c4"])
+    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c4", "c5"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
@@ -421,6 +525,8 @@ def main(argv=None):
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.config == "c5":
+        run_gpu_batched(args)
     else:
         run_gpu(args)
 

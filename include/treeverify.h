@@ -42,6 +42,7 @@ extern "C" {
 #endif
 
 #define TB_MAX_NODES 64 /* nodes per draft tree, root included */
+#define TB_MAX_BATCH 16 /* sequences per verify_step_batched call */
 
 typedef enum {
     TB_OK = 0,
@@ -209,6 +210,31 @@ TB_API tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, 
                       int vocab, const int32_t *draft_tokens, void *attn_out, int32_t *argmax,
                       float *top1, float *entropy, tb_result *result, void *workspace,
                       size_t workspace_bytes, int flags, tb_stream stream);
+
+/* One sequence of a batched verification step. */
+typedef struct tb_seq {
+    int32_t bank_id;              /* its draft-tree topology */
+    int32_t reserved;             /* 0 */
+    tb_kv kv;                     /* its KV cache and prefix length (all sequences of a batch share
+                                     n_layers, n_kv_heads and head_dim) */
+    const void *q;                /* bf16 [kv.n_layers][N_b][n_q_heads][head_dim] */
+    const int32_t *draft_tokens;  /* device int32 [N_b] */
+    void *attn_out;               /* bf16 [kv.n_layers][N_b][n_q_heads][head_dim] */
+    tb_result *result;            /* device */
+} tb_seq;
+
+/* verify_step for a batch of 1..TB_MAX_BATCH independent sequences, each with
+ * its own topology, prefix length and KV cache (ragged batch).  The LM head
+ * reads W once for the whole batch: hidden holds the rows of every sequence,
+ * sequence 0 first (sum of N_b rows, at most 1024); argmax / top1 / entropy
+ * follow the same row order.  Tree attention of every sequence runs in one
+ * launch (head_dim 128) whose work is balanced over the GPU whatever the
+ * prefix lengths; acceptance and compaction run in one launch.  `seqs` is a
+ * host array; everything else is as for verify_step. */
+TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                     const void *hidden, const void *lm_head, int d_model, int vocab, int32_t *argmax,
+                                     float *top1, float *entropy, void *workspace, size_t workspace_bytes, int flags,
+                                     tb_stream stream);
 
 /* lm_head_stats for callers that cannot allocate device memory.  Code that
  * runs inside a host framework which owns every device allocation, in a

@@ -28,7 +28,7 @@ RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
-       "kv_compact", "verify_step", "lm_head_stats_noalloc", "tb_last_error")
+       "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error")
 
 
 class TreeVerifyError(RuntimeError):
@@ -42,6 +42,13 @@ class TbKv(ctypes.Structure):
                 ("head_stride", ctypes.c_int64), ("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("L", ctypes.c_int32), ("L_cap", ctypes.c_int32)]
 
+
+class TbSeq(ctypes.Structure):
+    _fields_ = [("bank_id", ctypes.c_int32), ("reserved", ctypes.c_int32), ("kv", TbKv), ("q", ctypes.c_void_p),
+                ("draft_tokens", ctypes.c_void_p), ("attn_out", ctypes.c_void_p), ("result", ctypes.c_void_p)]
+
+
+TB_MAX_BATCH = 16
 
 _lib = None
 
@@ -70,6 +77,7 @@ def load(path: str = LIB_PATH):
         "kv_compact": [P, P, P],
         "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
         "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, P],
+        "verify_step_batched": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, sz, i32, P],
         "tb_last_error": [],
     }
     for name, args in sig.items():
@@ -261,3 +269,27 @@ def lm_head_stats_noalloc(hidden, lm_head, argmax, top1, entropy, stream=None):
     R, D = hidden.shape
     _check(load().lm_head_stats_noalloc(_ptr(hidden), R, _ptr(lm_head), D, lm_head.shape[0], _ptr(argmax),
                                         _ptr(top1), _ptr(entropy), _stream(stream)), "lm_head_stats_noalloc")
+
+
+@dataclass
+class Seq:
+    """One sequence of verify_step_batched."""
+
+    bank_id: int
+    kv: KvCache
+    q: object
+    draft_tokens: object
+    attn_out: object
+    result: object
+
+    def as_c(self) -> TbSeq:
+        return TbSeq(self.bank_id, 0, self.kv.as_c(), _ptr(self.q), _ptr(self.draft_tokens), _ptr(self.attn_out),
+                     _ptr(self.result))
+
+
+def verify_step_batched(bank: Bank, seqs, hidden, lm_head, argmax, top1, entropy, ws, flags: int = 0, stream=None):
+    """hidden bf16 [sum N_b][d_model] (sequence 0 first); argmax/top1/entropy [sum N_b]."""
+    arr = (TbSeq * len(seqs))(*[s.as_c() for s in seqs])
+    _check(load().verify_step_batched(bank.handle, len(seqs), arr, seqs[0].q.shape[2], _ptr(hidden), _ptr(lm_head),
+                                      hidden.shape[1], lm_head.shape[0], _ptr(argmax), _ptr(top1), _ptr(entropy),
+                                      _ptr(ws), ws.numel(), flags, _stream(stream)), "verify_step_batched")

@@ -37,8 +37,14 @@ __device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k,
     }
 }
 
-__global__ void __launch_bounds__(256) k3_accept_compact(const AcceptParams p)
+struct AcceptBatch {
+    AcceptParams seq[TB_MAX_BATCH];
+};
+
+// blockIdx.y selects the sequence; every CTA of a sequence recomputes its acceptance.
+__global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__ AcceptBatch pb)
 {
+    const AcceptParams &p = pb.seq[blockIdx.y];
     __shared__ int s_path[kMaxNodes];
     __shared__ int s_len;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -134,19 +140,31 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const AcceptParams p)
     }
 }
 
+cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream)
+{
+    if (n < 1 || n > TB_MAX_BATCH)
+        return cudaErrorInvalidValue;
+    AcceptBatch pb{};
+    int grid = 1;
+    for (int b = 0; b < n; ++b) {
+        pb.seq[b] = ps[b];
+        if (ps[b].n_layers > 0) {
+            const int units = ps[b].n_layers * ps[b].n_kv_heads * 2;
+            int gx = (units + 7) / 8;
+            const int cap = (2 * n_sm + n - 1) / n;
+            if (gx > cap)
+                gx = cap;
+            if (gx > grid)
+                grid = gx;
+        }
+    }
+    k3_accept_compact<<<dim3(grid, n), 256, 0, stream>>>(pb);
+    return cudaGetLastError();
+}
+
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream)
 {
-    int grid = 1;
-    if (p.n_layers > 0) {
-        const int units = p.n_layers * p.n_kv_heads * 2;
-        grid = (units + 7) / 8;
-        if (grid > 2 * n_sm)
-            grid = 2 * n_sm;
-        if (grid < 1)
-            grid = 1;
-    }
-    k3_accept_compact<<<grid, 256, 0, stream>>>(p);
-    return cudaGetLastError();
+    return accept_launch_batch(&p, 1, n_sm, stream);
 }
 
 }  // namespace tv

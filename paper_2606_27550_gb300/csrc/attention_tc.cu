@@ -49,14 +49,21 @@ constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], 
 constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 0, kColP1 = 128, kColO = 256, kColQ = 384;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
 
-struct TcParams {
-    CUtensorMap tmap_k;  // (128, L + N, Hkv, layers), box (64, 128, 1, 1), 128B swizzle
-    CUtensorMap tmap_v;
-    const __nv_bfloat16 *q;
-    __nv_bfloat16 *out;
+// One sequence of a (possibly batched) launch: its own KV cache (tensor maps),
+// prefix length, tree, queries and outputs.  Its tiles occupy
+// [tile_base, tile_base + n_units * T) of the flattened tile space.
+struct TcSeq {
+    long long tile_base;
+    const __nv_bfloat16 *q;  // [n_layers][N][Hq][128]
+    __nv_bfloat16 *out;      // same layout
     const TreeDesc *tree;
-    int L, N, Hq, Hkv, group, layer_begin, n_layers;
-    int rows, row_blocks, T, n_units;
+    int L, N, rows, row_blocks, T, unit_base;
+};
+
+struct TcParams {
+    CUtensorMap tmap[2 * kMaxSeqPerLaunch];  // K, V of each sequence: (128, L + N, Hkv, layers), box (64, 128, 1, 1)
+    TcSeq seq[kMaxSeqPerLaunch];
+    int n_seq, Hq, Hkv, group, layer_begin;
     long long total;
     int P;
     float scale_log2;
@@ -64,6 +71,15 @@ struct TcParams {
     int *counters;
     int *status;
 };
+
+// Sequence holding flattened tile t, searching forward from `b` (tiles are
+// visited in increasing order by every role).
+__device__ __forceinline__ int seq_at(const TcParams &p, long long t, int b)
+{
+    while (b + 1 < p.n_seq && t >= p.seq[b + 1].tile_base)
+        ++b;
+    return b;
+}
 
 __device__ __forceinline__ long long tc_seg_begin(const TcParams &p, int c)
 {
@@ -120,8 +136,10 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         mbar_init(&epi_ticket, 1);
         abort_flag = 0;
         fence_mbar_init();
-        prefetch_tmap(&p.tmap_k);
-        prefetch_tmap(&p.tmap_v);
+        for (int b = 0; b < p.n_seq; ++b) {
+            prefetch_tmap(&p.tmap[2 * b]);
+            prefetch_tmap(&p.tmap[2 * b + 1]);
+        }
     }
     if (warp == 1) {
         tmem_alloc(&tmem_slot, 512);
@@ -136,23 +154,28 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             long long issued = 0;
+            int sb = 0;
             for (long long it = 0; it < n_tiles; ++it) {
                 const int s = (int)(it % kStages);
                 const uint32_t ph = (uint32_t)(it / kStages) & 1u;
                 if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
                     break;
                 const long long t = t0 + it;
-                const int u = (int)(t / p.T);
-                const int j = (int)(t % p.T);
-                const int head = (u / p.row_blocks) % p.Hkv;
-                const int layer = p.layer_begin + u / (p.row_blocks * p.Hkv);
+                sb = seq_at(p, t, sb);
+                const TcSeq &sq = p.seq[sb];
+                const long long tl = t - sq.tile_base;
+                const int u = (int)(tl / sq.T);
+                const int j = (int)(tl % sq.T);
+                const int head = (u / sq.row_blocks) % p.Hkv;
+                const int layer = p.layer_begin + u / (sq.row_blocks * p.Hkv);
+                const CUtensorMap *mk = &p.tmap[2 * sb], *mv = &p.tmap[2 * sb + 1];
                 uint8_t *sk = sKV + (size_t)s * kStage;
                 uint8_t *sv = sk + kTile;
                 mbar_arrive_expect_tx(&full_bar[s], kStage);
-                tma_load_4d(sk, &p.tmap_k, &full_bar[s], 0, j * kBN, head, layer);
-                tma_load_4d(sk + kAtom, &p.tmap_k, &full_bar[s], 64, j * kBN, head, layer);
-                tma_load_4d(sv, &p.tmap_v, &full_bar[s], 0, j * kBN, head, layer);
-                tma_load_4d(sv + kAtom, &p.tmap_v, &full_bar[s], 64, j * kBN, head, layer);
+                tma_load_4d(sk, mk, &full_bar[s], 0, j * kBN, head, layer);
+                tma_load_4d(sk + kAtom, mk, &full_bar[s], 64, j * kBN, head, layer);
+                tma_load_4d(sv, mv, &full_bar[s], 0, j * kBN, head, layer);
+                tma_load_4d(sv + kAtom, mv, &full_bar[s], 64, j * kBN, head, layer);
                 issued = it + 1;
             }
             if (issued < n_tiles)
@@ -189,9 +212,11 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 tc_commit(&pv_done[bj]);
                 return true;
             };
+            int sb = 0;
             for (long long it = 0; it < n_tiles && ok; ++it) {
                 const long long t = t0 + it;
-                const bool first = (it == 0) || (t % p.T == 0);
+                sb = seq_at(p, t, sb);
+                const bool first = (it == 0) || ((t - p.seq[sb].tile_base) % p.seq[sb].T == 0);
                 if (first)
                     ++sg;
                 const int s = (int)(it % kStages);
@@ -241,34 +266,45 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         const int rloc = 4 * lane + q4;  // query row of this thread within the block
 
         struct Seg {
-            long long start, end, u_first, u_last;
-            int u, rb, head, layer_rel, rows_here, node, qh;
+            long long start, end, u_first, u_last;  // flattened tile indices
+            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N;
             bool valid;
             uint64_t anc;
+            const __nv_bfloat16 *q;
+            __nv_bfloat16 *out;
         };
+        int sb = 0;
         auto describe = [&](long long t) {
             Seg g;
+            sb = seq_at(p, t, sb);
+            const TcSeq &sq = p.seq[sb];
+            g.b = sb;
             g.start = t;
-            g.u = (int)(t / p.T);
-            g.u_first = (long long)g.u * p.T;
-            g.u_last = g.u_first + p.T;
+            g.u = (int)((t - sq.tile_base) / sq.T);
+            g.ucount = sq.unit_base + g.u;
+            g.u_first = sq.tile_base + (long long)g.u * sq.T;
+            g.u_last = g.u_first + sq.T;
             g.end = t1 < g.u_last ? t1 : g.u_last;
-            g.rb = g.u % p.row_blocks;
-            g.head = (g.u / p.row_blocks) % p.Hkv;
-            g.layer_rel = g.u / (p.row_blocks * p.Hkv);
-            g.rows_here = min(128, p.rows - g.rb * 128);
+            g.rb = g.u % sq.row_blocks;
+            g.head = (g.u / sq.row_blocks) % p.Hkv;
+            g.layer_rel = g.u / (sq.row_blocks * p.Hkv);
+            g.rows_here = min(128, sq.rows - g.rb * 128);
             g.valid = rloc < g.rows_here;
             const int grow = g.rb * 128 + rloc;
             g.node = g.valid ? grow / p.group : 0;
             g.qh = g.head * p.group + grow % p.group;
-            g.anc = g.valid ? p.tree->anc[g.node] : 0ull;
+            g.anc = g.valid ? sq.tree->anc[g.node] : 0ull;
+            g.L = sq.L;
+            g.N = sq.N;
+            g.q = sq.q;
+            g.out = sq.out;
             return g;
         };
         // Q row of this thread -> its TMEM lane as 64 columns of bf16 pairs (the A
         // operand of QK^T); zeros for padding rows
         auto write_q = [&](const Seg &g) {
             const uint4 *src =
-                reinterpret_cast<const uint4 *>(p.q + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+                reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
 #pragma unroll 1
             for (int qc = 0; qc < 4; ++qc) {
                 uint32_t w[16];
@@ -307,7 +343,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 tc_fence_after();
                 const uint32_t sa = lane_addr + (b ? kColS1 : kColS0);
                 const int key0 = (int)(t - g.u_first) * kBN;
-                const bool masked = key0 + kBN > p.L;
+                const bool masked = key0 + kBN > g.L;
 
                 // pass 1: the whole S row (4 loads, one wait), masked row max
                 float sc[kBN];
@@ -323,8 +359,8 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 if (masked) {
 #pragma unroll
                     for (int x = 0; x < kBN; ++x) {
-                        const int tj = key0 + x - p.L;
-                        const bool ok = tj < 0 || (tj < p.N && ((g.anc >> tj) & 1ull));
+                        const int tj = key0 + x - g.L;
+                        const bool ok = tj < 0 || (tj < g.N && ((g.anc >> tj) & 1ull));
                         sc[x] = ok ? sc[x] : -INFINITY;
                         mx = fmaxf(mx, sc[x]);
                     }
@@ -422,7 +458,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             {
                 const float inv = 1.f / l;
                 uint4 *dst =
-                    reinterpret_cast<uint4 *>(p.out + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
                 float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
 #pragma unroll 1
                 for (int c0 = 0; c0 < kD; c0 += 32) {
@@ -470,7 +506,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 ++n_partial;
                 if (warp == 2 && lane == 0) {
                     if (mbar_wait_bounded(&epi_written, eph, &abort_flag, p.status))
-                        ticket = atomicAdd(&p.counters[g.u], 1);
+                        ticket = atomicAdd(&p.counters[g.ucount], 1);
                     mbar_arrive(&epi_ticket);
                 }
                 if (!mbar_wait_bounded(&epi_ticket, eph, &abort_flag, p.status))
@@ -494,7 +530,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                         }
                         const float inv = 1.f / lsum;
                         uint4 *dst = reinterpret_cast<uint4 *>(
-                            p.out + (((size_t)g.layer_rel * p.N + g.node) * p.Hq + g.qh) * kD);
+                            g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
 #pragma unroll 1
                         for (int c0 = 0; c0 < kD; c0 += 32) {
                             float acc[32];
@@ -528,7 +564,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                         }
                     }
                     if (warp == 2 && lane == 0)
-                        p.counters[g.u] = 0;
+                        p.counters[g.ucount] = 0;
                 }
             }
             if (!has_next)
@@ -583,34 +619,54 @@ size_t attn_tc_slot_floats()
     return (size_t)kSlot;
 }
 
-cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
-                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                           cudaStream_t stream, const char **err)
+int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers)
 {
-    const AttnPlan pl = attn_tc_plan(kv->L, N, Hq, kv->n_kv_heads, n_layers, n_sm);
+    int units = 0;
+    for (int b = 0; b < n_seq; ++b)
+        units += attn_tc_plan(seqs[b].kv->L, seqs[b].N, Hq, Hkv, n_layers, 1).n_units;
+    return units;
+}
+
+cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
+                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err)
+{
+    if (n_seq < 1 || n_seq > kMaxSeqPerLaunch) {
+        *err = "too many sequences for one attention launch";
+        return cudaErrorInvalidValue;
+    }
     TcParams p{};
-    if (!make_tmap_kv(&p.tmap_k, kv->k, kD, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
-                      kv->layer_stride, kBN, err))
-        return cudaErrorInvalidValue;
-    if (!make_tmap_kv(&p.tmap_v, kv->v, kD, kv->L + N, kv->n_kv_heads, kv->n_layers, kv->head_stride,
-                      kv->layer_stride, kBN, err))
-        return cudaErrorInvalidValue;
-    p.q = static_cast<const __nv_bfloat16 *>(q);
-    p.out = static_cast<__nv_bfloat16 *>(out);
-    p.tree = d_tree;
-    p.L = kv->L;
-    p.N = N;
+    long long tiles = 0;
+    int units = 0;
+    const int Hkv = seqs[0].kv->n_kv_heads;
+    for (int b = 0; b < n_seq; ++b) {
+        const tb_kv *kv = seqs[b].kv;
+        const AttnPlan pl = attn_tc_plan(kv->L, seqs[b].N, Hq, Hkv, n_layers, n_sm);
+        if (!make_tmap_kv(&p.tmap[2 * b], kv->k, kD, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
+                          kv->head_stride, kv->layer_stride, kBN, err) ||
+            !make_tmap_kv(&p.tmap[2 * b + 1], kv->v, kD, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
+                          kv->head_stride, kv->layer_stride, kBN, err))
+            return cudaErrorInvalidValue;
+        TcSeq &sq = p.seq[b];
+        sq.tile_base = tiles;
+        sq.q = static_cast<const __nv_bfloat16 *>(seqs[b].q);
+        sq.out = static_cast<__nv_bfloat16 *>(seqs[b].out);
+        sq.tree = seqs[b].tree;
+        sq.L = kv->L;
+        sq.N = seqs[b].N;
+        sq.rows = pl.rows;
+        sq.row_blocks = pl.row_blocks;
+        sq.T = pl.T;
+        sq.unit_base = units;
+        tiles += pl.total;
+        units += pl.n_units;
+    }
+    p.n_seq = n_seq;
     p.Hq = Hq;
-    p.Hkv = kv->n_kv_heads;
-    p.group = pl.group;
+    p.Hkv = Hkv;
+    p.group = Hq / Hkv;
     p.layer_begin = layer_begin;
-    p.n_layers = n_layers;
-    p.rows = pl.rows;
-    p.row_blocks = pl.row_blocks;
-    p.T = pl.T;
-    p.n_units = pl.n_units;
-    p.total = pl.total;
-    p.P = pl.P;
+    p.total = tiles;
+    p.P = (int)(tiles < n_sm ? tiles : n_sm);
     p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
     p.part = part;
     p.counters = counters;
@@ -618,8 +674,16 @@ cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int l
     cudaError_t e = allow_max_smem((const void *)k1_tree_attention_tc);
     if (e != cudaSuccess)
         return e;
-    k1_tree_attention_tc<<<pl.P, 192, tc_smem_bytes(), stream>>>(p);
+    k1_tree_attention_tc<<<p.P, 192, tc_smem_bytes(), stream>>>(p);
     return cudaGetLastError();
+}
+
+cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
+                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                           cudaStream_t stream, const char **err)
+{
+    AttnSeq one{kv, d_tree, N, q, out};
+    return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, counters, status, n_sm, stream, err);
 }
 
 }  // namespace tv

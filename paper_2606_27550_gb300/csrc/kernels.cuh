@@ -27,7 +27,19 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
                         const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
                         cudaStream_t stream, const char **err);
 
-// tree attention on tcgen05 (attention_tc.cu): head_dim 128
+// tree attention on tcgen05 (attention_tc.cu): head_dim 128, one or several
+// sequences (each with its own cache, prefix length and tree) per launch
+constexpr int kMaxSeqPerLaunch = TB_MAX_BATCH;
+struct AttnSeq {
+    const tb_kv *kv;
+    const TreeDesc *tree;
+    int N;
+    const void *q;
+    void *out;
+};
+int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers);
+cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
+                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err);
 bool attn_tc_supported(int d, int rows);
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
 size_t attn_tc_slot_floats();
@@ -52,6 +64,7 @@ struct AcceptParams {
     int from_result;  // compaction driven by an existing result (kv_compact): no acceptance
 };
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
+cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once
 // per (kernel, device) (treeverify.cu).

@@ -407,8 +407,8 @@ extern "C" size_t tb_workspace_size(int max_rows, int n_layers, int n_kv_heads, 
     size_t bytes = kPartBase;
     if (head_dim > 0)
         bytes += attn_part_bytes(nsm, head_dim);
-    if (max_rows > 0 && vocab > 0)
-        bytes += align256(lm_plan(max_rows, 64, vocab).ws_bytes);
+    if (max_rows > 0 && vocab > 0)  // batched calls run the LM head in chunks of 256 rows
+        bytes += align256(lm_plan(max_rows < 256 ? max_rows : 256, 64, vocab).ws_bytes);
     return bytes;
 }
 
@@ -704,6 +704,112 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
     if (!(flags & TB_NO_COMPACT))
         add_compaction(p, kv);
     cudaError_t e = accept_launch(p, sm_count(bank->device), s);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
+}
+
+extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                         const void *hidden, const void *lm_head, int d_model, int vocab,
+                                         int32_t *argmax, float *top1, float *entropy, void *workspace,
+                                         size_t workspace_bytes, int flags, tb_stream stream)
+{
+    const char *fn = "verify_step_batched";
+    if (!bank)
+        return fail(TB_EINVAL, "%s: bank is NULL", fn);
+    if (batch < 1 || batch > TB_MAX_BATCH || !seqs)
+        return fail(TB_EINVAL, "%s: batch %d outside 1..%d (or seqs NULL)", fn, batch, TB_MAX_BATCH);
+    tb_status st;
+    int rows_total = 0;
+    int Ns[TB_MAX_BATCH];
+    for (int b = 0; b < batch; ++b) {
+        const tb_seq &sq = seqs[b];
+        if ((st = check_bank(bank, sq.bank_id, fn)) != TB_OK)
+            return st;
+        Ns[b] = bank->h_desc[sq.bank_id].n;
+        if ((st = check_kv(&sq.kv, Ns[b], fn)) != TB_OK)
+            return st;
+        if (sq.kv.n_layers != seqs[0].kv.n_layers || sq.kv.n_kv_heads != seqs[0].kv.n_kv_heads ||
+            sq.kv.head_dim != seqs[0].kv.head_dim)
+            return fail(TB_EINVAL, "%s: sequence %d has another layer / head / head_dim count than sequence 0", fn,
+                        b);
+        if (!sq.q || !sq.attn_out || !sq.draft_tokens || !sq.result || !aligned16(sq.q) || !aligned16(sq.attn_out))
+            return fail(TB_EINVAL, "%s: sequence %d: NULL or unaligned q / attn_out / draft_tokens / result", fn, b);
+        rows_total += Ns[b];
+    }
+    const tb_kv &kv0 = seqs[0].kv;
+    if (n_q_heads < kv0.n_kv_heads || n_q_heads % kv0.n_kv_heads)
+        return fail(TB_EINVAL, "%s: n_q_heads %d not a multiple of n_kv_heads %d", fn, n_q_heads, kv0.n_kv_heads);
+    const int group = n_q_heads / kv0.n_kv_heads;
+    for (int b = 0; b < batch; ++b)
+        if (Ns[b] * group > 256)
+            return fail(TB_EUNSUPPORTED, "%s: sequence %d: N * group = %d > 256", fn, b, Ns[b] * group);
+    if (rows_total > 4 * 256)
+        return fail(TB_EUNSUPPORTED, "%s: %d LM-head rows > 1024", fn, rows_total);
+    LmPlan lplan;
+    const int chunk = rows_total < 256 ? rows_total : 256;
+    if ((st = lm_validate(hidden, chunk, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
+        return st;
+    const int nsm = sm_count(bank->device);
+    const bool tc = use_tc_attention(kv0.head_dim, 0);
+    if (tc) {
+        AttnSeq as[TB_MAX_BATCH];
+        for (int b = 0; b < batch; ++b)
+            as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
+        const int units = attn_tc_units(as, batch, n_q_heads, kv0.n_kv_heads, kv0.n_layers);
+        if (units > kMaxAttnUnits)
+            return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, units, kMaxAttnUnits);
+    }
+    const size_t attn_bytes = attn_part_bytes(nsm, kv0.head_dim);
+    const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
+    if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
+        return st;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = (cudaStream_t)stream;
+
+    // LM head over every row of the batch, in chunks of up to 256 rows
+    const uint8_t *h8 = static_cast<const uint8_t *>(hidden);
+    for (int r0 = 0; r0 < rows_total; r0 += 256) {
+        const int rc = rows_total - r0 < 256 ? rows_total - r0 : 256;
+        if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
+                             entropy + r0, ws, kPartBase + attn_bytes, s, fn)) != TB_OK)
+            return st;
+    }
+    // tree attention of every sequence
+    if (tc) {
+        AttnSeq as[TB_MAX_BATCH];
+        for (int b = 0; b < batch; ++b)
+            as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
+        const char *err = "";
+        cudaError_t e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads,
+                                             reinterpret_cast<float *>(ws + kPartBase),
+                                             reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws),
+                                             nsm, s, &err);
+        if (e == cudaErrorInvalidValue && err[0])
+            return fail(TB_EINVAL, "%s: %s", fn, err);
+        if (e != cudaSuccess)
+            return cuda_fail(e, fn);
+    } else {
+        for (int b = 0; b < batch; ++b) {
+            AttnArgs a{bank, seqs[b].bank_id, &seqs[b].kv, 0, kv0.n_layers, seqs[b].q, n_q_heads, seqs[b].attn_out};
+            AttnPlan plan;
+            if ((st = attn_validate(a, fn, &plan)) != TB_OK)
+                return st;
+            if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+                return st;
+        }
+    }
+    // acceptance + compaction, one launch
+    AcceptParams ps[TB_MAX_BATCH];
+    int r0 = 0;
+    for (int b = 0; b < batch; ++b) {
+        ps[b] = accept_params(bank, seqs[b].bank_id, seqs[b].draft_tokens, argmax + r0, vocab, seqs[b].kv.L,
+                              seqs[b].result, reinterpret_cast<const int *>(ws));
+        if (!(flags & TB_NO_COMPACT))
+            add_compaction(ps[b], &seqs[b].kv);
+        r0 += Ns[b];
+    }
+    cudaError_t e = accept_launch_batch(ps, batch, nsm, s);
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();

@@ -178,6 +178,38 @@ def shape_c4() -> Shape:
                  rank_product_tree(BANK_BRANCHING, 64), 0.5)
 
 
+@dataclass
+class BatchShape:
+    """Ragged batch: one (tree, L, p_match) per sequence, shared model shapes."""
+    name: str
+    n_layers: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    d_model: int
+    vocab: int
+    parents: list
+    Ls: list
+    p_match: list
+    w_std: float = 0.02
+
+    @property
+    def Ns(self):
+        return [len(p) for p in self.parents]
+
+
+def batch_c5(seed: int = 5, batch: int = 8, vocab: int = 128256, L_range=(512, 8192)) -> BatchShape:
+    """Ragged batched verify: GQA 32 q / 8 kv heads x 128, d_model 4096; each
+    sequence draws its tree from the bank sizes >= 4, L ~ U[512, 8192] and its
+    draft-match probability ~ U[0.3, 0.9]."""
+    g = rng(seed, 7)
+    trees = [t for t in bank_trees() if len(t) >= 4]
+    parents = [trees[int(g.integers(0, len(trees)))] for _ in range(batch)]
+    Ls = [int(g.integers(L_range[0], L_range[1] + 1)) for _ in range(batch)]
+    ps = [float(g.uniform(0.3, 0.9)) for _ in range(batch)]
+    return BatchShape(f"7b-gqa32x8-batch{batch}-V{vocab}-ragged", 1, 32, 8, 128, 4096, vocab, parents, Ls, ps)
+
+
 SHAPES = {"c1": shape_c1, "c2": shape_c2, "c3": shape_c3, "c4": shape_c4}
 
 
