@@ -420,6 +420,104 @@ def run_gpu_batched(args):
     print(json.dumps(line), flush=True)
 
 
+def run_gpu_bank_loop(args):
+    """The bank-switching loop: 7B single-layer shapes, the 8-tree bank, L from
+    2048 growing by accept_len, 1000 steps; each step's tree comes from the
+    hysteretic step ladder (up below 1.5 nats, down above 2.5 nats) over a
+    seeded AR(1) entropy trace; KV compaction every step; the host reads the
+    step's result (new prefix length) once per step."""
+    import torch
+
+    import paper_2606_27550_gb300 as tv
+    from paper_2606_27550_gb300 import build as tvbuild
+
+    world, rank, local = dist_info()
+    tvbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    sh = synth.shape_c3()
+    steps = sh.extra["steps"] if args.steps == 200 else args.steps
+    H, d, D, V, L0 = sh.n_q_heads, sh.head_dim, sh.d_model, sh.vocab, sh.L
+    bf = torch.bfloat16
+    seed = 777 + rank
+    trees = synth.bank_trees()
+    bank = tv.Bank(16, local)
+    ids = [bank.add(t)[0] for t in trees]
+    k = synth.device_normal_bf16_(torch.empty((1, H, sh.L_cap, d), dtype=bf, device=dev), seed)
+    v = synth.device_normal_bf16_(torch.empty((1, H, sh.L_cap, d), dtype=bf, device=dev), seed + 1)
+    W = synth.device_normal_bf16_(torch.empty((V, D), dtype=bf, device=dev), seed + 2, std=sh.w_std)
+    pool = 16
+    qs = synth.device_normal_bf16_(torch.empty((pool, 1, 64, H, d), dtype=bf, device=dev), seed + 3)
+    hs = synth.device_normal_bf16_(torch.empty((pool, 64, D), dtype=bf, device=dev), seed + 4)
+    am = torch.empty(64, dtype=torch.int32, device=dev)
+    t1 = torch.empty(64, dtype=torch.float32, device=dev)
+    en = torch.empty(64, dtype=torch.float32, device=dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(64, 1, H, H, d, V, local), dev)
+    drafts = {}
+    for i in range(pool):  # untimed: each pool entry's greedy tokens -> drafts for every bank tree
+        tv.lm_head_stats(hs[i], W, am, t1, en, ws)
+        a = am.cpu().numpy()
+        for j, t in enumerate(trees):
+            drafts[(i, j)] = torch.from_numpy(synth.gen_drafts(seed + 100 * i + j, t, a[:len(t)], V, sh.p_match)).to(dev)
+    outs = [torch.empty((1, len(t), H, d), dtype=bf, device=dev) for t in trees]
+    res = tv.make_result(dev)
+    res_h = torch.empty(tv.RESULT_INTS, dtype=torch.int32, pin_memory=True)
+    trace = synth.ar1_entropy_trace(0, steps + args.warmup, hmax=float(np.log(V)))
+    stream = torch.cuda.current_stream()
+
+    def loop(t_from, t_to, L, kix):
+        toks = kv_b = 0
+        accepted = []
+        hist = [0] * len(trees)
+        for t in range(t_from, t_to):
+            kix = tv.tb_schedule_hysteretic_ladder(kix, len(trees), float(trace[t]), 1.5, 2.5)
+            n = len(trees[kix])
+            i = t % pool
+            kv = tv.KvCache(k, v, L)
+            tv.verify_step(bank, ids[kix], kv, qs[i][:, :n], hs[i][:n], W, drafts[(i, kix)], outs[kix], am[:n],
+                           t1[:n], en[:n], res, ws, 0, stream)
+            res_h.copy_(res, non_blocking=True)
+            stream.synchronize()
+            kv_b += 2 * (L + n) * H * d * 2
+            toks += n
+            hist[kix] += 1
+            accepted.append(int(res_h[0]))
+            L = int(res_h[2])
+        return L, kix, toks, kv_b, accepted, hist
+
+    L, kix, *_ = loop(0, args.warmup, L0, 0)
+    sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]
+                           if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
+    sampler.start()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    L_end, _, toks, kv_b, accepted, hist = loop(args.warmup, args.warmup + steps, L, kix)
+    el = time.perf_counter() - t0
+    clocks = sampler.stop()
+    bank.close()
+    if rank != 0:
+        return
+    peaks, peak_src = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    w_b = V * D * 2 * steps
+    line = {
+        "metric": "verify-steps/s", "value": round(steps / el, 3), "unit": "verify-steps/s", "n_gpus": world,
+        "steps": steps, "warmup": args.warmup, "ms_per_step": round(el / steps * 1e3, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded), AR(1) entropy trace",
+        "config": {"workload": sh.name, "bank_sizes": [len(t) for t in trees], "L_start": L, "L_end": L_end,
+                   "policy": "hysteretic step ladder: up below 1.5 nats, down above 2.5 nats",
+                   "host_read_per_step": True},
+        "tree_tokens_per_s": round(toks / el, 1),
+        "tau_mean_accept_len": round(float(np.mean(accepted)), 4),
+        "tree_histogram": hist,
+        "hbm_roofline": {"bytes": kv_b + w_b, "frac": round((kv_b + w_b) / el / 1e9 / hbm, 4), "peak_gbs": hbm,
+                         "peak_src": peak_src},
+        "gpu_launches": 3 * steps,
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+
+
 # ----------------------------------------------------------------------------- CPU oracle (reference arm)
 
 
@@ -515,7 +613,7 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c4", "c5"])
+    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c3", "c4", "c5"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
@@ -527,6 +625,8 @@ def main(argv=None):
         run_reference(args)
     elif args.config == "c5":
         run_gpu_batched(args)
+    elif args.config == "c3":
+        run_gpu_bank_loop(args)
     else:
         run_gpu(args)
 

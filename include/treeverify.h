@@ -211,6 +211,32 @@ TB_API tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, 
                       float *top1, float *entropy, tb_result *result, void *workspace,
                       size_t workspace_bytes, int flags, tb_stream stream);
 
+/* ------------------------------------------------------------------------
+ * Per-step tree selection (Sec. 4, "Policy"): which bank entry the next step
+ * verifies.  Pure host functions, O(1); switching is then the bank_id passed
+ * to the next verify_step (no GPU work).
+ * ---------------------------------------------------------------------- */
+
+/* Hysteretic step ladder over trees 0..n_trees-1 ordered from smallest to
+ * largest, driven by a feature that is LOW when the continuation is
+ * predictable (the entropy of the verifier's distribution, nats): move one
+ * tree up when feature < up_below, one tree down when feature > down_above,
+ * otherwise stay (up_below <= down_above gives a dead band against flapping).
+ * Returns the next index, clamped to [0, n_trees). */
+TB_API int tb_schedule_hysteretic_ladder(int current, int n_trees, double feature, double up_below,
+                                         double down_above);
+
+/* The paper's binary hysteretic rule on the path-value score s (HIGH when
+ * deep drafts are likely): switch to the aggressive tree when s > tau_on,
+ * back to the conservative tree when s <= tau_off, tau_off <= tau_on.
+ * `aggressive` is 1 when the current tree is the aggressive one; returns the
+ * new value. */
+TB_API int tb_schedule_binary(int aggressive, double s, double tau_on, double tau_off);
+
+/* threshold_ladder: the index of the interval of s among n_trees - 1
+ * ascending edges (s < edges[0] -> 0, ..., s >= edges[n_trees-2] -> n_trees-1). */
+TB_API int tb_schedule_threshold_ladder(double s, const double *edges, int n_trees);
+
 /* One sequence of a batched verification step. */
 typedef struct tb_seq {
     int32_t bank_id;              /* its draft-tree topology */

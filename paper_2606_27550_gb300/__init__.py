@@ -28,7 +28,8 @@ RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
-       "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error")
+       "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error",
+       "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder")
 
 
 class TreeVerifyError(RuntimeError):
@@ -83,6 +84,12 @@ def load(path: str = LIB_PATH):
     for name, args in sig.items():
         f = getattr(lib, name)
         f.argtypes = args
+        f.restype = ctypes.c_int
+    d = ctypes.c_double
+    lib.tb_schedule_hysteretic_ladder.argtypes = [i32, i32, d, d, d]
+    lib.tb_schedule_binary.argtypes = [i32, d, d, d]
+    lib.tb_schedule_threshold_ladder.argtypes = [d, P, i32]
+    for f in (lib.tb_schedule_hysteretic_ladder, lib.tb_schedule_binary, lib.tb_schedule_threshold_ladder):
         f.restype = ctypes.c_int
     lib.tb_workspace_size.restype = ctypes.c_size_t
     lib.tb_last_error.restype = ctypes.c_char_p
@@ -293,3 +300,20 @@ def verify_step_batched(bank: Bank, seqs, hidden, lm_head, argmax, top1, entropy
     _check(load().verify_step_batched(bank.handle, len(seqs), arr, seqs[0].q.shape[2], _ptr(hidden), _ptr(lm_head),
                                       hidden.shape[1], lm_head.shape[0], _ptr(argmax), _ptr(top1), _ptr(entropy),
                                       _ptr(ws), ws.numel(), flags, _stream(stream)), "verify_step_batched")
+
+
+# --------------------------------------------------------------------- per-step tree selection
+
+
+def tb_schedule_hysteretic_ladder(current: int, n_trees: int, feature: float, up_below: float,
+                                  down_above: float) -> int:
+    return int(load().tb_schedule_hysteretic_ladder(current, n_trees, feature, up_below, down_above))
+
+
+def tb_schedule_binary(aggressive: int, s: float, tau_on: float, tau_off: float) -> int:
+    return int(load().tb_schedule_binary(int(aggressive), s, tau_on, tau_off))
+
+
+def tb_schedule_threshold_ladder(s: float, edges) -> int:
+    e = np.ascontiguousarray(edges, dtype=np.float64)
+    return int(load().tb_schedule_threshold_ladder(s, _ptr(e), len(e) + 1))

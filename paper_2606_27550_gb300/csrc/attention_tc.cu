@@ -455,44 +455,43 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             tc_fence_after();
             const bool whole = (g.start == g.u_first && g.end == g.u_last);
             float *slot = p.part + ((size_t)c * 2 + (g.start == t0 ? 0 : 1)) * kSlot;
+            float o[kD];
             {
-                const float inv = 1.f / l;
-                uint4 *dst =
-                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
-                float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
-#pragma unroll 1
-                for (int c0 = 0; c0 < kD; c0 += 32) {
-                    uint32_t r[32];
-                    tmem_ld_32x32b_x32(lane_addr + kColO + c0, r);
-                    tmem_ld_wait();
-                    if (!g.valid)
-                        continue;
-                    if (whole) {
-#pragma unroll
-                        for (int ch = 0; ch < 4; ++ch) {
-                            uint4 v;
-                            v.x = pack_bf16x2(__uint_as_float(r[8 * ch + 0]) * inv, __uint_as_float(r[8 * ch + 1]) * inv);
-                            v.y = pack_bf16x2(__uint_as_float(r[8 * ch + 2]) * inv, __uint_as_float(r[8 * ch + 3]) * inv);
-                            v.z = pack_bf16x2(__uint_as_float(r[8 * ch + 4]) * inv, __uint_as_float(r[8 * ch + 5]) * inv);
-                            v.w = pack_bf16x2(__uint_as_float(r[8 * ch + 6]) * inv, __uint_as_float(r[8 * ch + 7]) * inv);
-                            dst[c0 / 8 + ch] = v;
-                        }
-                    } else {
-#pragma unroll
-                        for (int x = 0; x < 8; ++x)
-                            pdst[c0 / 4 + x] = make_float4(__uint_as_float(r[4 * x]), __uint_as_float(r[4 * x + 1]),
-                                                           __uint_as_float(r[4 * x + 2]), __uint_as_float(r[4 * x + 3]));
-                    }
-                }
+                uint32_t *r = reinterpret_cast<uint32_t *>(o);
+                tmem_ld_32x32b_x32(lane_addr + kColO, r);
+                tmem_ld_32x32b_x32(lane_addr + kColO + 32, r + 32);
+                tmem_ld_32x32b_x32(lane_addr + kColO + 64, r + 64);
+                tmem_ld_32x32b_x32(lane_addr + kColO + 96, r + 96);
+                tmem_ld_wait();
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&o_free);
+            auto store_out = [&](const float *x, float scale) {
+                uint4 *dst =
+                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
+#pragma unroll
+                for (int ch = 0; ch < kD / 8; ++ch) {
+                    uint4 v;
+                    v.x = pack_bf16x2(x[8 * ch + 0] * scale, x[8 * ch + 1] * scale);
+                    v.y = pack_bf16x2(x[8 * ch + 2] * scale, x[8 * ch + 3] * scale);
+                    v.z = pack_bf16x2(x[8 * ch + 4] * scale, x[8 * ch + 5] * scale);
+                    v.w = pack_bf16x2(x[8 * ch + 6] * scale, x[8 * ch + 7] * scale);
+                    dst[ch] = v;
+                }
+            };
 
-            if (!whole) {
-                // partial (O, m_ref, l) is in this CTA's slot; take the unit's arrival ticket
+            if (whole) {
+                if (g.valid)
+                    store_out(o, 1.f / l);
+            } else {
+                // partial (O, m_ref, l) -> this CTA's slot; then the unit's arrival ticket
                 if (g.valid) {
+                    float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
+#pragma unroll
+                    for (int x = 0; x < kD / 4; ++x)
+                        pdst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
                     slot[128 * kD + rloc] = m_ref;
                     slot[128 * kD + 128 + rloc] = l;
                 }
@@ -515,6 +514,8 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 if (last) {
                     __threadfence();
                     if (g.valid) {
+                        // log-sum-exp merge of every CTA's partial of this unit; each slot's
+                        // row is fetched with 32 independent 16-byte loads
                         float M = -INFINITY;
                         for (int cc = c_lo; cc <= c_hi; ++cc) {
                             const float *sl =
@@ -522,46 +523,29 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                             M = fmaxf(M, __ldcg(sl + 128 * kD + rloc));
                         }
                         float lsum = 0.f;
+#pragma unroll
+                        for (int x = 0; x < kD; ++x)
+                            o[x] = 0.f;
                         for (int cc = c_lo; cc <= c_hi; ++cc) {
                             const float *sl =
                                 p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
                             const float ms = __ldcg(sl + 128 * kD + rloc);
-                            lsum += (ms == -INFINITY) ? 0.f : ex2_approx(ms - M) * __ldcg(sl + 128 * kD + 128 + rloc);
-                        }
-                        const float inv = 1.f / lsum;
-                        uint4 *dst = reinterpret_cast<uint4 *>(
-                            g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
-#pragma unroll 1
-                        for (int c0 = 0; c0 < kD; c0 += 32) {
-                            float acc[32];
+                            const float w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
+                            lsum += w * __ldcg(sl + 128 * kD + 128 + rloc);
+                            const float4 *src = reinterpret_cast<const float4 *>(sl + rloc * kD);
+                            float4 vv[kD / 4];
 #pragma unroll
-                            for (int x = 0; x < 32; ++x)
-                                acc[x] = 0.f;
-                            for (int cc = c_lo; cc <= c_hi; ++cc) {
-                                const float *sl =
-                                    p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
-                                const float ms = __ldcg(sl + 128 * kD + rloc);
-                                const float w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M) * inv;
-                                const float4 *src = reinterpret_cast<const float4 *>(sl + rloc * kD + c0);
+                            for (int x = 0; x < kD / 4; ++x)
+                                vv[x] = __ldcg(src + x);
 #pragma unroll
-                                for (int x = 0; x < 8; ++x) {
-                                    const float4 v = __ldcg(src + x);
-                                    acc[4 * x] += w * v.x;
-                                    acc[4 * x + 1] += w * v.y;
-                                    acc[4 * x + 2] += w * v.z;
-                                    acc[4 * x + 3] += w * v.w;
-                                }
-                            }
-#pragma unroll
-                            for (int ch = 0; ch < 4; ++ch) {
-                                uint4 v;
-                                v.x = pack_bf16x2(acc[8 * ch + 0], acc[8 * ch + 1]);
-                                v.y = pack_bf16x2(acc[8 * ch + 2], acc[8 * ch + 3]);
-                                v.z = pack_bf16x2(acc[8 * ch + 4], acc[8 * ch + 5]);
-                                v.w = pack_bf16x2(acc[8 * ch + 6], acc[8 * ch + 7]);
-                                dst[c0 / 8 + ch] = v;
+                            for (int x = 0; x < kD / 4; ++x) {
+                                o[4 * x] += w * vv[x].x;
+                                o[4 * x + 1] += w * vv[x].y;
+                                o[4 * x + 2] += w * vv[x].z;
+                                o[4 * x + 3] += w * vv[x].w;
                             }
                         }
+                        store_out(o, 1.f / lsum);
                     }
                     if (warp == 2 && lane == 0)
                         p.counters[g.ucount] = 0;

@@ -814,3 +814,37 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
         return cuda_fail(e, fn);
     return ok();
 }
+
+// ------------------------------------------------------------------ per-step tree selection
+
+extern "C" int tb_schedule_hysteretic_ladder(int current, int n_trees, double feature, double up_below,
+                                             double down_above)
+{
+    if (n_trees < 1)
+        return 0;
+    int k = current < 0 ? 0 : (current >= n_trees ? n_trees - 1 : current);
+    if (feature < up_below)
+        k = k + 1 < n_trees ? k + 1 : n_trees - 1;
+    else if (feature > down_above)
+        k = k > 0 ? k - 1 : 0;
+    return k;
+}
+
+extern "C" int tb_schedule_binary(int aggressive, double s, double tau_on, double tau_off)
+{
+    if (s > tau_on)
+        return 1;
+    if (s <= tau_off)
+        return 0;
+    return aggressive ? 1 : 0;
+}
+
+extern "C" int tb_schedule_threshold_ladder(double s, const double *edges, int n_trees)
+{
+    if (!edges || n_trees <= 1)
+        return 0;
+    int k = 0;
+    while (k < n_trees - 1 && s >= edges[k])
+        ++k;
+    return k;
+}
