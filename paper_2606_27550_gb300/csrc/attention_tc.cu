@@ -3,8 +3,11 @@
 //
 // Same operation and work split as attention.cu (tree decoding, Sec. 3.2;
 // ancestor-bitset mask, Sec. 2.3; flattened (layer, kv head, row block) x
-// key-tile space split evenly over a persistent grid, ticketed log-sum-exp
-// merge of split units), with the contractions on tcgen05:
+// key-tile space split evenly over a persistent grid), with the contractions
+// on tcgen05.  A CTA that covers a whole unit writes its output; a unit split
+// between CTAs leaves one (O, m, l) partial per CTA, and a second small kernel
+// (k1_merge_split, one warp per query row) combines them by log-sum-exp after
+// the first one has finished:
 //
 //   S   = Q K^T   tcgen05.mma kind::f16, M = 128 query rows, N = 128 keys,
 //                 K = 128 = head_dim; Q (bf16) is the TMEM A operand, the K
@@ -73,12 +76,17 @@ struct TcParams {
 };
 
 // Sequence holding flattened tile t, searching forward from `b` (tiles are
-// visited in increasing order by every role).
+// visited in increasing order by every role).  kBatched = false: sequence 0.
+template <bool kBatched>
 __device__ __forceinline__ int seq_at(const TcParams &p, long long t, int b)
 {
-    while (b + 1 < p.n_seq && t >= p.seq[b + 1].tile_base)
-        ++b;
-    return b;
+    if constexpr (!kBatched) {
+        return 0;
+    } else {
+        while (b + 1 < p.n_seq && t >= p.seq[b + 1].tile_base)
+            ++b;
+        return b;
+    }
 }
 
 __device__ __forceinline__ long long tc_seg_begin(const TcParams &p, int c)
@@ -100,15 +108,15 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t l
 
 }  // namespace
 
+template <bool kBatched>
 __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
     __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
-    __shared__ __align__(8) uint64_t q_full, o_free, drain_bar, epi_written, epi_ticket;
+    __shared__ __align__(8) uint64_t q_full, o_free, drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
-    __shared__ int ticket;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sKV = smem;
@@ -132,11 +140,9 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         mbar_init(&q_full, 4);
         mbar_init(&o_free, 4);
         mbar_init(&drain_bar, 1);
-        mbar_init(&epi_written, 4);
-        mbar_init(&epi_ticket, 1);
         abort_flag = 0;
         fence_mbar_init();
-        for (int b = 0; b < p.n_seq; ++b) {
+        for (int b = 0; b < (kBatched ? p.n_seq : 1); ++b) {
             prefetch_tmap(&p.tmap[2 * b]);
             prefetch_tmap(&p.tmap[2 * b + 1]);
         }
@@ -161,7 +167,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
                     break;
                 const long long t = t0 + it;
-                sb = seq_at(p, t, sb);
+                sb = seq_at<kBatched>(p, t, sb);
                 const TcSeq &sq = p.seq[sb];
                 const long long tl = t - sq.tile_base;
                 const int u = (int)(tl / sq.T);
@@ -215,7 +221,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             int sb = 0;
             for (long long it = 0; it < n_tiles && ok; ++it) {
                 const long long t = t0 + it;
-                sb = seq_at(p, t, sb);
+                sb = seq_at<kBatched>(p, t, sb);
                 const bool first = (it == 0) || ((t - p.seq[sb].tile_base) % p.seq[sb].T == 0);
                 if (first)
                     ++sg;
@@ -276,7 +282,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         int sb = 0;
         auto describe = [&](long long t) {
             Seg g;
-            sb = seq_at(p, t, sb);
+            sb = seq_at<kBatched>(p, t, sb);
             const TcSeq &sq = p.seq[sb];
             g.b = sb;
             g.start = t;
@@ -325,7 +331,6 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                 mbar_arrive(&q_full);
         };
         long long it = 0;
-        int n_partial = 0;  // partial segments so far (phase of epi_written / epi_ticket)
         bool aborted = (n_tiles == 0);
         Seg g;
         if (!aborted) {
@@ -455,101 +460,45 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             tc_fence_after();
             const bool whole = (g.start == g.u_first && g.end == g.u_last);
             float *slot = p.part + ((size_t)c * 2 + (g.start == t0 ? 0 : 1)) * kSlot;
-            float o[kD];
             {
-                uint32_t *r = reinterpret_cast<uint32_t *>(o);
-                tmem_ld_32x32b_x32(lane_addr + kColO, r);
-                tmem_ld_32x32b_x32(lane_addr + kColO + 32, r + 32);
-                tmem_ld_32x32b_x32(lane_addr + kColO + 64, r + 64);
-                tmem_ld_32x32b_x32(lane_addr + kColO + 96, r + 96);
-                tmem_ld_wait();
+                const float inv = 1.f / l;
+                uint4 *dst =
+                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
+                float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
+#pragma unroll 1
+                for (int c0 = 0; c0 < kD; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32b_x32(lane_addr + kColO + c0, r);
+                    tmem_ld_wait();
+                    if (!g.valid)
+                        continue;
+                    if (whole) {
+#pragma unroll
+                        for (int ch = 0; ch < 4; ++ch) {
+                            uint4 v;
+                            v.x = pack_bf16x2(__uint_as_float(r[8 * ch + 0]) * inv, __uint_as_float(r[8 * ch + 1]) * inv);
+                            v.y = pack_bf16x2(__uint_as_float(r[8 * ch + 2]) * inv, __uint_as_float(r[8 * ch + 3]) * inv);
+                            v.z = pack_bf16x2(__uint_as_float(r[8 * ch + 4]) * inv, __uint_as_float(r[8 * ch + 5]) * inv);
+                            v.w = pack_bf16x2(__uint_as_float(r[8 * ch + 6]) * inv, __uint_as_float(r[8 * ch + 7]) * inv);
+                            dst[c0 / 8 + ch] = v;
+                        }
+                    } else {
+#pragma unroll
+                        for (int x = 0; x < 8; ++x)
+                            pdst[c0 / 4 + x] = make_float4(__uint_as_float(r[4 * x]), __uint_as_float(r[4 * x + 1]),
+                                                           __uint_as_float(r[4 * x + 2]), __uint_as_float(r[4 * x + 3]));
+                    }
+                }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
                 mbar_arrive(&o_free);
-            auto store_out = [&](const float *x, float scale) {
-                uint4 *dst =
-                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
-#pragma unroll
-                for (int ch = 0; ch < kD / 8; ++ch) {
-                    uint4 v;
-                    v.x = pack_bf16x2(x[8 * ch + 0] * scale, x[8 * ch + 1] * scale);
-                    v.y = pack_bf16x2(x[8 * ch + 2] * scale, x[8 * ch + 3] * scale);
-                    v.z = pack_bf16x2(x[8 * ch + 4] * scale, x[8 * ch + 5] * scale);
-                    v.w = pack_bf16x2(x[8 * ch + 6] * scale, x[8 * ch + 7] * scale);
-                    dst[ch] = v;
-                }
-            };
 
-            if (whole) {
-                if (g.valid)
-                    store_out(o, 1.f / l);
-            } else {
-                // partial (O, m_ref, l) -> this CTA's slot; then the unit's arrival ticket
-                if (g.valid) {
-                    float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
-#pragma unroll
-                    for (int x = 0; x < kD / 4; ++x)
-                        pdst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
-                    slot[128 * kD + rloc] = m_ref;
-                    slot[128 * kD + 128 + rloc] = l;
-                }
-                // all four warps' rows written -> one ticket for the CTA -> broadcast
-                __threadfence();
-                __syncwarp();
-                if (lane == 0)
-                    mbar_arrive(&epi_written);
-                const int c_lo = tc_cta_of(p, g.u_first), c_hi = tc_cta_of(p, g.u_last - 1);
-                const uint32_t eph = (uint32_t)n_partial & 1u;
-                ++n_partial;
-                if (warp == 2 && lane == 0) {
-                    if (mbar_wait_bounded(&epi_written, eph, &abort_flag, p.status))
-                        ticket = atomicAdd(&p.counters[g.ucount], 1);
-                    mbar_arrive(&epi_ticket);
-                }
-                if (!mbar_wait_bounded(&epi_ticket, eph, &abort_flag, p.status))
-                    break;
-                const bool last = (ticket == c_hi - c_lo);
-                if (last) {
-                    __threadfence();
-                    if (g.valid) {
-                        // log-sum-exp merge of every CTA's partial of this unit; each slot's
-                        // row is fetched with 32 independent 16-byte loads
-                        float M = -INFINITY;
-                        for (int cc = c_lo; cc <= c_hi; ++cc) {
-                            const float *sl =
-                                p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
-                            M = fmaxf(M, __ldcg(sl + 128 * kD + rloc));
-                        }
-                        float lsum = 0.f;
-#pragma unroll
-                        for (int x = 0; x < kD; ++x)
-                            o[x] = 0.f;
-                        for (int cc = c_lo; cc <= c_hi; ++cc) {
-                            const float *sl =
-                                p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= g.u_first ? 0 : 1)) * kSlot;
-                            const float ms = __ldcg(sl + 128 * kD + rloc);
-                            const float w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
-                            lsum += w * __ldcg(sl + 128 * kD + 128 + rloc);
-                            const float4 *src = reinterpret_cast<const float4 *>(sl + rloc * kD);
-                            float4 vv[kD / 4];
-#pragma unroll
-                            for (int x = 0; x < kD / 4; ++x)
-                                vv[x] = __ldcg(src + x);
-#pragma unroll
-                            for (int x = 0; x < kD / 4; ++x) {
-                                o[4 * x] += w * vv[x].x;
-                                o[4 * x + 1] += w * vv[x].y;
-                                o[4 * x + 2] += w * vv[x].z;
-                                o[4 * x + 3] += w * vv[x].w;
-                            }
-                        }
-                        store_out(o, 1.f / lsum);
-                    }
-                    if (warp == 2 && lane == 0)
-                        p.counters[g.ucount] = 0;
-                }
+            if (!whole && g.valid) {
+                // partial (O in the slot already, m_ref, l); k1_merge_split finishes the unit
+                slot[128 * kD + rloc] = m_ref;
+                slot[128 * kD + 128 + rloc] = l;
             }
             if (!has_next)
                 break;
@@ -566,6 +515,88 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         __syncwarp();
         tmem_dealloc(tmem, 512);
     }
+}
+
+// Log-sum-exp merge of the partials of every unit split between CTAs.  A unit
+// is split exactly when a CTA range starts inside it, so the grid runs over
+// the CTA boundaries c = 1 .. P-1 (x) and groups of 8 query rows (y); the
+// first boundary inside a unit handles it.  One warp per query row, each lane
+// 4 of the 128 output columns, the slots' loads issued together.
+template <bool kBatched>
+__global__ void __launch_bounds__(256) k1_merge_split(const __grid_constant__ TcParams p)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int cb = blockIdx.x + 1;  // CTA range starting at tile t_c
+    const long long tc = tc_seg_begin(p, cb);
+    int b = 0;
+    if constexpr (kBatched) {
+        while (b + 1 < p.n_seq && tc >= p.seq[b + 1].tile_base)
+            ++b;
+    }
+    const TcSeq &sq = p.seq[b];
+    const int u = (int)((tc - sq.tile_base) / sq.T);
+    const long long u_first = sq.tile_base + (long long)u * sq.T, u_last = u_first + sq.T;
+    if (tc == u_first)
+        return;  // the boundary is a unit boundary
+    const int c_lo = tc_cta_of(p, u_first), c_hi = tc_cta_of(p, u_last - 1);
+    if (cb != c_lo + 1)
+        return;  // an earlier boundary inside this unit handles it
+    const int nseg = c_hi - c_lo + 1;
+    const int rb = u % sq.row_blocks;
+    const int head = (u / sq.row_blocks) % p.Hkv;
+    const int layer_rel = u / (sq.row_blocks * p.Hkv);
+    const int rows_here = min(128, sq.rows - rb * 128);
+    const int r = blockIdx.y * 8 + warp;
+    if (r >= rows_here)
+        return;
+    auto slot_of = [&](int cc) {
+        return p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
+    };
+    // global max of the partial maxima
+    float M = -INFINITY;
+    for (int j = lane; j < nseg; j += 32)
+        M = fmaxf(M, __ldcg(slot_of(c_lo + j) + 128 * kD + r));
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1)
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, m));
+    float lsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j0 = 0; j0 < nseg; j0 += 32) {
+        // lane j holds the weight of slot j0 + j
+        float w = 0.f;
+        if (j0 + lane < nseg) {
+            const float *sl = slot_of(c_lo + j0 + lane);
+            const float ms = __ldcg(sl + 128 * kD + r);
+            w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
+            lsum += w * __ldcg(sl + 128 * kD + 128 + r);
+        }
+        const int cnt = min(32, nseg - j0);
+        for (int j1 = 0; j1 < cnt; j1 += 8) {
+            float4 v[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                v[k] = (j1 + k < cnt)
+                           ? __ldcg(reinterpret_cast<const float4 *>(slot_of(c_lo + j0 + j1 + k) + r * kD) + lane)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const float wk = __shfl_sync(0xffffffffu, w, (j1 + k) & 31);
+                acc.x += wk * v[k].x;
+                acc.y += wk * v[k].y;
+                acc.z += wk * v[k].z;
+                acc.w += wk * v[k].w;
+            }
+        }
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1)
+        lsum += __shfl_xor_sync(0xffffffffu, lsum, m);
+    const float inv = 1.f / lsum;
+    const int grow = rb * 128 + r;
+    const int node = grow / p.group;
+    const int qh = head * p.group + grow % p.group;
+    uint2 *dst = reinterpret_cast<uint2 *>(sq.out + (((size_t)layer_rel * sq.N + node) * p.Hq + qh) * kD) + lane;
+    *dst = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
 }
 
 // ----------------------------------------------------------------------------
@@ -620,7 +651,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     }
     TcParams p{};
     long long tiles = 0;
-    int units = 0;
+    int units = 0, max_rows = 0;
     const int Hkv = seqs[0].kv->n_kv_heads;
     for (int b = 0; b < n_seq; ++b) {
         const tb_kv *kv = seqs[b].kv;
@@ -643,6 +674,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
         sq.unit_base = units;
         tiles += pl.total;
         units += pl.n_units;
+        max_rows = pl.rows < 128 ? (pl.rows > max_rows ? pl.rows : max_rows) : 128;
     }
     p.n_seq = n_seq;
     p.Hq = Hq;
@@ -655,10 +687,24 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     p.part = part;
     p.counters = counters;
     p.status = status;
-    cudaError_t e = allow_max_smem((const void *)k1_tree_attention_tc);
-    if (e != cudaSuccess)
-        return e;
-    k1_tree_attention_tc<<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+    cudaError_t e;
+    if (n_seq == 1) {
+        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
+            return e;
+        k1_tree_attention_tc<false><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+        if ((e = cudaGetLastError()) != cudaSuccess)
+            return e;
+        if (p.P > 1)
+            k1_merge_split<false><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
+    } else {
+        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<true>)) != cudaSuccess)
+            return e;
+        k1_tree_attention_tc<true><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+        if ((e = cudaGetLastError()) != cudaSuccess)
+            return e;
+        if (p.P > 1)
+            k1_merge_split<true><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
+    }
     return cudaGetLastError();
 }
 

@@ -213,6 +213,13 @@ struct tb_bank {
     TreeDesc *d_desc;
     std::vector<TreeDesc> h_desc;
     std::vector<int32_t> h_parent;  // canonical parents, capacity x 64
+    // A verification step forks the LM head onto `aux` so that it runs in the
+    // tail of the attention kernel (whose CTAs each hold a whole SM), then
+    // joins back before acceptance.  The mutex keeps one step's fork/join
+    // enqueue sequence contiguous when several host threads share the bank.
+    cudaStream_t aux;
+    cudaEvent_t ev_fork, ev_join;
+    std::mutex fork_mu;
 };
 
 extern "C" tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
@@ -303,6 +310,18 @@ extern "C" tb_status tb_create(tb_bank **out, int max_topologies, int device)
     }
     b->h_desc.resize(max_topologies);
     b->h_parent.assign((size_t)max_topologies * TB_MAX_NODES, -1);
+    b->aux = nullptr;
+    b->ev_fork = b->ev_join = nullptr;
+    if ((e = cudaSetDevice(device)) == cudaSuccess &&
+        (e = cudaStreamCreateWithFlags(&b->aux, cudaStreamNonBlocking)) == cudaSuccess &&
+        (e = cudaEventCreateWithFlags(&b->ev_fork, cudaEventDisableTiming)) == cudaSuccess)
+        e = cudaEventCreateWithFlags(&b->ev_join, cudaEventDisableTiming);
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        tb_destroy(b);
+        return cuda_fail(e, "tb_create: helper stream / events");
+    }
     *out = b;
     return ok();
 }
@@ -378,6 +397,12 @@ extern "C" tb_status tb_destroy(tb_bank *bank)
     cudaError_t e = cudaSetDevice(bank->device);
     if (e == cudaSuccess && bank->d_desc)
         e = cudaFree(bank->d_desc);
+    if (bank->ev_fork)
+        cudaEventDestroy(bank->ev_fork);
+    if (bank->ev_join)
+        cudaEventDestroy(bank->ev_join);
+    if (bank->aux)
+        cudaStreamDestroy(bank->aux);
     if (prev >= 0)
         cudaSetDevice(prev);
     delete bank;
@@ -694,11 +719,26 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
         return st;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = (cudaStream_t)stream;
-    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s,
-                         fn)) != TB_OK)
-        return st;
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
-        return st;
+    {
+        // attention on the caller's stream; the LM head forked onto the bank's
+        // helper stream fills the SMs that attention CTAs release; join before acceptance
+        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
+        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step: fork");
+        if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+            return st;
+        if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                             bank->aux, fn)) != TB_OK)
+            return st;
+        e = cudaEventRecord(bank->ev_join, bank->aux);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step: join");
+    }
     AcceptParams p =
         accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
     if (!(flags & TB_NO_COMPACT))
@@ -767,24 +807,23 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = (cudaStream_t)stream;
 
-    // LM head over every row of the batch, in chunks of up to 256 rows
-    const uint8_t *h8 = static_cast<const uint8_t *>(hidden);
-    for (int r0 = 0; r0 < rows_total; r0 += 256) {
-        const int rc = rows_total - r0 < 256 ? rows_total - r0 : 256;
-        if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
-                             entropy + r0, ws, kPartBase + attn_bytes, s, fn)) != TB_OK)
-            return st;
-    }
+    // attention on the caller's stream, the LM head forked onto the helper
+    // stream (it fills the SMs the attention CTAs release), joined before acceptance
+    std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
+    cudaError_t e = cudaEventRecord(bank->ev_fork, s);
+    if (e == cudaSuccess)
+        e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "verify_step_batched: fork");
     // tree attention of every sequence
     if (tc) {
         AttnSeq as[TB_MAX_BATCH];
         for (int b = 0; b < batch; ++b)
             as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
         const char *err = "";
-        cudaError_t e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads,
-                                             reinterpret_cast<float *>(ws + kPartBase),
-                                             reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws),
-                                             nsm, s, &err);
+        e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
+                                 reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
+                                 &err);
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
@@ -799,6 +838,19 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
                 return st;
         }
     }
+    // LM head over every row of the batch, in chunks of up to 256 rows
+    const uint8_t *h8 = static_cast<const uint8_t *>(hidden);
+    for (int r0 = 0; r0 < rows_total; r0 += 256) {
+        const int rc = rows_total - r0 < 256 ? rows_total - r0 : 256;
+        if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
+                             entropy + r0, ws, kPartBase + attn_bytes, bank->aux, fn)) != TB_OK)
+            return st;
+    }
+    e = cudaEventRecord(bank->ev_join, bank->aux);
+    if (e == cudaSuccess)
+        e = cudaStreamWaitEvent(s, bank->ev_join, 0);
+    if (e != cudaSuccess)
+        return cuda_fail(e, "verify_step_batched: join");
     // acceptance + compaction, one launch
     AcceptParams ps[TB_MAX_BATCH];
     int r0 = 0;
@@ -809,7 +861,7 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
             add_compaction(ps[b], &seqs[b].kv);
         r0 += Ns[b];
     }
-    cudaError_t e = accept_launch_batch(ps, batch, nsm, s);
+    e = accept_launch_batch(ps, batch, nsm, s);
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
