@@ -198,6 +198,13 @@ TB_API tb_status greedy_accept(const tb_bank *bank, int bank_id, const int32_t *
 TB_API tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream);
 
 #define TB_NO_COMPACT 1 /* verify_step flag: skip the KV-cache update */
+/* verify_step test hook for failure detection: the LM-head kernel waits on a
+ * barrier that nothing arrives on, so its bounded wait (about one second)
+ * expires; the kernel then stops cleanly (in-flight copies land, issued MMAs
+ * retire, TMEM is freed), the step reports TB_ETIMEOUT in tb_result.status
+ * and in the workspace status word, and argmax/top1/entropy are not written.
+ * The workspace must be re-initialised (tb_workspace_init) afterwards. */
+#define TB_DEBUG_EXPIRE_WAIT (1 << 30)
 
 /* One full verification step of topology bank_id: tree_attention over all
  * kv->n_layers layers, lm_head_stats over the N node rows, greedy_accept, and

@@ -24,6 +24,7 @@ TB_OK, TB_EINVAL, TB_ENOMEM, TB_ECUDA, TB_ENOTFOUND, TB_ECAPACITY, TB_ETIMEOUT, 
     0, -1, -2, -3, -4, -5, -6, -7)
 TB_MAX_NODES = 64
 TB_NO_COMPACT = 1
+TB_DEBUG_EXPIRE_WAIT = 1 << 30
 RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",

@@ -14,7 +14,7 @@ struct LmPlan {
 LmPlan lm_plan(int R, int D, int V);
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
-                           const char **err);
+                           const char **err, int expire_wait = 0);
 
 // tree attention (attention.cu)
 struct AttnPlan {

@@ -35,6 +35,7 @@ struct LmParams {
     float4 *part_group;  // [n_groups][R_pad]
     int *counters;       // [n_groups + 1], zero between launches
     int *status;
+    int expire_wait;     // test hook: the epilogue waits on a barrier nothing arrives on
     int32_t *argmax;
     float *top1;
     float *entropy;
@@ -166,6 +167,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     __shared__ __align__(8) uint64_t full_bar[8];
     __shared__ __align__(8) uint64_t empty_bar[8];
     __shared__ __align__(8) uint64_t acc_bar;
+    __shared__ __align__(8) uint64_t never_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
     __shared__ int ticket;
@@ -189,6 +191,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             mbar_init(&empty_bar[s], 1);
         }
         mbar_init(&acc_bar, 1);
+        mbar_init(&never_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&p.tmap_w);
@@ -257,7 +260,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     __syncwarp();
 
     // ---------------- epilogue: TMEM -> shared (transposed) -> per-row stats
-    mbar_wait_bounded(&acc_bar, 0, &abort_flag, p.status);
+    mbar_wait_bounded(p.expire_wait ? &never_bar : &acc_bar, 0, &abort_flag, p.status);
     tc_fence_after();
     __syncthreads();
     const bool ok = (abort_flag == 0);
@@ -398,7 +401,7 @@ LmPlan lm_plan(int R, int D, int V)
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
-                           const char **err)
+                           const char **err, int expire_wait)
 {
     const LmPlan pl = lm_plan(R, D, V);
     LmParams p{};
@@ -424,6 +427,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.argmax = argmax;
     p.top1 = top1;
     p.entropy = entropy;
+    p.expire_wait = expire_wait;
     cudaError_t e = allow_max_smem((const void *)k2_lm_head);
     if (e != cudaSuccess)
         return e;

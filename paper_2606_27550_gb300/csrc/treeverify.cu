@@ -582,12 +582,12 @@ static tb_status lm_validate(const void *hidden, int R, const void *W, int D, in
 }
 
 static tb_status lm_enqueue(const void *hidden, int R, const void *W, int D, int V, int32_t *am, float *t1, float *en,
-                            uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn)
+                            uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn, int expire_wait = 0)
 {
     const char *err = "";
     cudaError_t e = lm_head_launch(hidden, R, W, D, V, am, t1, en, ws + part_off,
                                    reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws), stream,
-                                   &err);
+                                   &err, expire_wait);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -731,7 +731,7 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
         if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
             return st;
         if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                             bank->aux, fn)) != TB_OK)
+                             bank->aux, fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0)) != TB_OK)
             return st;
         e = cudaEventRecord(bank->ev_join, bank->aux);
         if (e == cudaSuccess)
