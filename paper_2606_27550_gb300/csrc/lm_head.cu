@@ -372,7 +372,11 @@ LmPlan lm_plan(int R, int D, int V)
     pl.bps = lm_boxes_per_stage(pl.R_pad);
     pl.n_kblocks = ceil_div(D, 64 * pl.bps);
     const int stage_bytes = (16384 + pl.R_pad * 128) * pl.bps;
-    pl.stages = (110 * 1024) / stage_bytes;
+    // Up to 64 rows two CTAs share an SM (110 KB each); wider rows need a
+    // transpose buffer that leaves one CTA per SM, so its ring takes ~200 KB.
+    const size_t transpose_bytes = (size_t)pl.R_pad * (128 + 8) * 4;
+    const int budget = (transpose_bytes + 1024 <= 110 * 1024) ? 110 * 1024 : 200 * 1024;
+    pl.stages = budget / stage_bytes;
     if (pl.stages > 8)
         pl.stages = 8;
     if (pl.stages < 2)
