@@ -61,11 +61,7 @@ def workload(cfg: str, layers: int | None = None):
     return sh, kv_bytes, w_bytes, flops
 
 
-def dist_info():
-    ws = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return ws, rank, local
+from paper_2606_27550_gb300.replicas import dist_info, job_throughput, max_over_ranks  # noqa: E402
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -208,9 +204,7 @@ def run_gpu(args):
     elapsed_ms = e0.elapsed_time(e1)
     if world > 1:
         dist.barrier()
-        t = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, dev)
     r = tv.parse_result(res)
 
     # per-kernel durations: the same work through the stage entry points, events between stages
@@ -257,11 +251,7 @@ def run_gpu(args):
         stats_h[2].copy_(en, non_blocking=True)
         stream.synchronize()
         _ = int(res_h[0])  # the per-step host read of the accepted length
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
     clocks = sampler.stop()
 
     if world > 1:
@@ -274,7 +264,7 @@ def run_gpu(args):
     peaks, peak_src = load_peaks()
     hbm = float(peaks["hbm_gbs"])
     ms = elapsed_ms / args.steps
-    value = world * args.steps / (elapsed_ms / 1e3)
+    value = job_throughput(args.steps, elapsed_ms / 1e3, world)
     at_gbs = kv_bytes / (t_at * 1e-3) / 1e9
     line = {
         "metric": "verify-steps/s",
@@ -304,7 +294,7 @@ def run_gpu(args):
                        "k3_accept_compact": round(t_ac, 4)},
         "lm_head_gbs": round(w_bytes / (t_lm * 1e-3) / 1e9, 1),
         "accept_len_last": r["accept_len"],
-        "e2e": {"value": round(world * n_e2e / e2e_s, 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": 3 * args.steps,
         "clocks": clocks,
@@ -385,11 +375,7 @@ def run_gpu_batched(args):
         step()
         ev[i][1].record(stream)
     torch.cuda.synchronize()
-    elapsed_ms = sum(a.elapsed_time(b) for a, b in ev)
-    if world > 1:
-        t = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in ev), dev)
     clocks = sampler.stop()
     if world > 1:
         dist.destroy_process_group()
@@ -400,7 +386,7 @@ def run_gpu_batched(args):
     hbm = float(peaks["hbm_gbs"])
     tflops = float(peaks.get("bf16_tflops_sustained", 1700.0))
     ms = elapsed_ms / args.steps
-    value = world * args.steps / (elapsed_ms / 1e3)
+    value = job_throughput(args.steps, elapsed_ms / 1e3, world)
     t_mem = (kv_bytes + w_bytes) / (hbm * 1e9) * 1e3
     t_comp = flops / (tflops * 1e12) * 1e3
     line = {
