@@ -296,7 +296,8 @@ def run_gpu(args):
         "accept_len_last": r["accept_len"],
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": 3 * args.steps,
+        # per step: LM head, attention, split-unit merge (head_dim 128), acceptance + compaction
+        "gpu_launches": (4 if d == 128 else 3) * args.steps,
         "clocks": clocks,
     }
     if args.layers:
@@ -400,7 +401,7 @@ def run_gpu_batched(args):
         "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
                      "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
                      "flops_per_step": flops, "peak_gbs": hbm, "peak_tflops_sustained": tflops, "peak_src": peak_src},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": 4 * args.steps,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -498,7 +499,7 @@ def run_gpu_bank_loop(args):
         "tree_histogram": hist,
         "hbm_roofline": {"bytes": kv_b + w_b, "frac": round((kv_b + w_b) / el / 1e9 / hbm, 4), "peak_gbs": hbm,
                          "peak_src": peak_src},
-        "gpu_launches": 3 * steps,
+        "gpu_launches": 4 * steps,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)

@@ -521,9 +521,10 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 // is split exactly when a CTA range starts inside it, so the grid runs over
 // the CTA boundaries c = 1 .. P-1 (x) and groups of 8 query rows (y); the
 // first boundary inside a unit handles it.  One warp per query row, each lane
-// 4 of the 128 output columns, the slots' loads issued together.
+// 4 of the 128 output columns, four slots' loads issued together; 32 registers
+// per thread keep every row's warp resident at once.
 template <bool kBatched>
-__global__ void __launch_bounds__(256) k1_merge_split(const __grid_constant__ TcParams p)
+__global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__ TcParams p)
 {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int cb = blockIdx.x + 1;  // CTA range starting at tile t_c
@@ -549,42 +550,49 @@ __global__ void __launch_bounds__(256) k1_merge_split(const __grid_constant__ Tc
     const int r = blockIdx.y * 8 + warp;
     if (r >= rows_here)
         return;
-    auto slot_of = [&](int cc) {
-        return p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
-    };
-    // global max of the partial maxima
+    // lane j of each 32-slot block owns slot c_lo + j0 + j: its row pointer, max and weight
     float M = -INFINITY;
-    for (int j = lane; j < nseg; j += 32)
-        M = fmaxf(M, __ldcg(slot_of(c_lo + j) + 128 * kD + r));
+    for (int j0 = 0; j0 < nseg; j0 += 32) {
+        const int cc = c_lo + j0 + lane;
+        if (j0 + lane < nseg) {
+            const float *sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
+            M = fmaxf(M, __ldcg(sl + 128 * kD + r));
+        }
+    }
 #pragma unroll
     for (int m = 16; m >= 1; m >>= 1)
         M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, m));
     float lsum = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int j0 = 0; j0 < nseg; j0 += 32) {
-        // lane j holds the weight of slot j0 + j
+        const int cc = c_lo + j0 + lane;
+        const float *sl = p.part;
         float w = 0.f;
         if (j0 + lane < nseg) {
-            const float *sl = slot_of(c_lo + j0 + lane);
+            sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
             const float ms = __ldcg(sl + 128 * kD + r);
             w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             lsum += w * __ldcg(sl + 128 * kD + 128 + r);
         }
+        const unsigned long long row_ptr = reinterpret_cast<unsigned long long>(sl + r * kD) + 16ull * lane;
         const int cnt = min(32, nseg - j0);
-        for (int j1 = 0; j1 < cnt; j1 += 8) {
-            float4 v[8];
+        for (int j1 = 0; j1 < cnt; j1 += 4) {
+            float4 v[4];
+            float wk[4];
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-                v[k] = (j1 + k < cnt)
-                           ? __ldcg(reinterpret_cast<const float4 *>(slot_of(c_lo + j0 + j1 + k) + r * kD) + lane)
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int k = 0; k < 4; ++k) {
+                const int src = (j1 + k) & 31;
+                // lane's 16-byte column block of slot j0 + j1 + k
+                const unsigned long long base = __shfl_sync(0xffffffffu, row_ptr - 16ull * lane, src) + 16ull * lane;
+                wk[k] = __shfl_sync(0xffffffffu, w, src);
+                v[k] = (j1 + k < cnt) ? __ldcg(reinterpret_cast<const float4 *>(base)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const float wk = __shfl_sync(0xffffffffu, w, (j1 + k) & 31);
-                acc.x += wk * v[k].x;
-                acc.y += wk * v[k].y;
-                acc.z += wk * v[k].z;
-                acc.w += wk * v[k].w;
+            for (int k = 0; k < 4; ++k) {
+                acc.x += wk[k] * v[k].x;
+                acc.y += wk[k] * v[k].y;
+                acc.z += wk[k] * v[k].z;
+                acc.w += wk[k] * v[k].w;
             }
         }
     }
