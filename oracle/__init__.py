@@ -3,8 +3,8 @@
 Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's CPU baseline
 leg import this package.  The product library never does.
 
-``oracle.c`` holds the arithmetic (tree sets, attention, LM head, greedy
-acceptance); this module compiles it with gcc, loads it with ctypes and adds
+``oracle.c`` holds the arithmetic (tree sets, attention, LM head, greedy and
+typical acceptance); this module compiles it with gcc, loads it with ctypes and adds
 the KV compaction, which is a plain gather written out below.
 """
 from __future__ import annotations
@@ -46,6 +46,9 @@ def _load():
             lib.oracle_lm_head.argtypes = [P, P, i32, i32, i32, P, P, P, P, P]
             lib.oracle_accept.argtypes = [P, i32, P, P, P, P, P]
             lib.oracle_num_threads.argtypes = []
+            d = ctypes.c_double
+            lib.oracle_typical_accept.argtypes = [P, i32, P, P, i32, d, d, d, P, P, P, P, P, P]
+            lib.oracle_typical_accept.restype = ctypes.c_int
             for f in (lib.oracle_tree, lib.oracle_tree_attention, lib.oracle_lm_head,
                       lib.oracle_accept, lib.oracle_num_threads):
                 f.restype = ctypes.c_int
@@ -139,3 +142,32 @@ def kv_compact(cache, L: int, path):
     for j, src in enumerate(path):
         new[..., L + j, :] = old[..., L + src, :]
     return new
+
+
+def typical_accept(parent, draft, logits, temperature: float, eps: float, alpha: float, detail: bool = False):
+    """Typical acceptance: (accept_len, path list, bonus token[, detail dict]).
+
+    logits: float64 [N][V], the target logits after every node.  detail adds
+    per-edge margins (p - threshold) / threshold, per-node path
+    log-likelihoods and per-node accepted flags."""
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    draft = np.ascontiguousarray(draft, dtype=np.int32)
+    logits = np.ascontiguousarray(logits, dtype=np.float64)
+    n, V = logits.shape
+    if n != len(parent) or len(draft) < n:
+        raise ValueError("one logit row and one draft token per node")
+    path = np.zeros(max(n, 1), dtype=np.int32)
+    alen = np.zeros(1, dtype=np.int32)
+    bonus = np.zeros(1, dtype=np.int32)
+    margin = np.zeros(n)
+    loglik = np.zeros(n)
+    acc = np.zeros(n, dtype=np.int32)
+    if _load().oracle_typical_accept(_ptr(parent), n, _ptr(draft), _ptr(logits), V, temperature, eps, alpha,
+                                     _ptr(alen), _ptr(path), _ptr(bonus), _ptr(margin), _ptr(loglik),
+                                     _ptr(acc)) != 0:
+        raise ValueError("bad tree, vocab or temperature")
+    k = int(alen[0])
+    out = (k, [int(x) for x in path[:k]], int(bonus[0]))
+    if detail:
+        return out + ({"margin": margin, "loglik": loglik, "accepted": acc.astype(bool)},)
+    return out

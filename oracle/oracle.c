@@ -25,6 +25,10 @@
  *                  index among equally deep ones); accept_len = depth + 1 counts
  *                  the accepted drafts plus the bonus token argmax[j*]
  *                  (greedy form of the verification step, Sec. 3.2 / 5.1 tau).
+ *   typical        the Medusa/Hydra typical-acceptance rule (Sec. 5.1, 5.2:
+ *                  T = 0.7, eps = 0.09, alpha = 0.3): an edge is accepted when
+ *                  the tempered target probability of its draft token exceeds
+ *                  min(eps, alpha exp(-H)); see oracle_typical_accept.
  *
  * Pinned by tests/test_oracle_pins.py against independent references
  * (torch float64 attention, brute-force path enumeration, closed forms).
@@ -249,5 +253,104 @@ int oracle_accept(const int32_t *parent, int N, const int32_t *draft,
     }
     *accept_len = len;
     *bonus = argmax[best];
+    return 0;
+}
+
+/*
+ * Typical acceptance: the verification rule of Medusa/Hydra decoding that the
+ * paper keeps unchanged and runs with T = 0.7, eps = 0.09, alpha = 0.3
+ * (Sec. 5.1, 5.2).  The rule itself is the published Medusa one: the target
+ * distribution after node u is p_u = softmax(z_u / T) with entropy
+ * H_u = -sum_v p_u(v) ln p_u(v) (nats); the edge into non-root node j is
+ * accepted when
+ *     p_{parent(j)}(draft[j]) > min(eps, alpha * exp(-H_{parent(j)})),
+ * and node i is accepted when every edge on its root path is.  Among the
+ * deepest accepted nodes the one whose path has the largest log-likelihood
+ * sum_{j on the path, j != root} ln p_{parent(j)}(draft[j]) wins (smallest
+ * index on exact ties).  accept_len = depth + 1; the bonus token is the
+ * greedy token after the last accepted node, argmax z_{j*} (lowest index on
+ * ties): the first token of every step is taken greedily.
+ *   logits [N][V]       z_u for every node u (double)
+ *   margin[j]  (NULL ok) (p - threshold) / threshold of the edge into j; 0 for the root
+ *   loglik[i]  (NULL ok) path log-likelihood of node i; 0 for the root
+ *   accepted[i](NULL ok) 1 when node i is accepted
+ * A draft token outside [0, V) has probability 0 and is never accepted.
+ */
+int oracle_typical_accept(const int32_t *parent, int N, const int32_t *draft, const double *logits, int V,
+                          double temperature, double eps, double alpha, int32_t *accept_len, int32_t *path,
+                          int32_t *bonus, double *margin, double *loglik, int32_t *accepted)
+{
+    uint8_t in_anc[ORACLE_MAX_NODES * ORACLE_MAX_NODES];
+    int32_t depth[ORACLE_MAX_NODES];
+    if (oracle_tree(parent, N, depth, in_anc) != 0 || V < 1 || !(temperature > 0.0))
+        return -1;
+    double p_edge[ORACLE_MAX_NODES], thr[ORACLE_MAX_NODES];
+    int32_t amax[ORACLE_MAX_NODES];
+    for (int u = 0; u < N; ++u) {
+        const double *z = logits + (size_t)u * V;
+        int best = 0;
+        for (int v = 1; v < V; ++v)
+            if (z[v] > z[best])
+                best = v;
+        amax[u] = best;
+    }
+    /* per edge: the target probability of the drafted token and the threshold */
+    for (int j = 0; j < N; ++j) {
+        p_edge[j] = 1.0;
+        thr[j] = 0.0;
+        if (j == 0)
+            continue;
+        const int u = parent[j];
+        const double *z = logits + (size_t)u * V;
+        const double m = z[amax[u]];
+        double denom = 0.0;
+        for (int v = 0; v < V; ++v)
+            denom += exp((z[v] - m) / temperature);
+        double ent = 0.0;
+        for (int v = 0; v < V; ++v) {
+            const double p = exp((z[v] - m) / temperature) / denom;
+            if (p > 0.0)
+                ent -= p * log(p);
+        }
+        const int tok = draft[j];
+        p_edge[j] = (tok >= 0 && tok < V) ? exp((z[tok] - m) / temperature) / denom : 0.0;
+        const double a = alpha * exp(-ent);
+        thr[j] = eps < a ? eps : a;
+    }
+    /* per node: accepted when every edge of its root path is; path log-likelihood */
+    int32_t ok[ORACLE_MAX_NODES];
+    double ll[ORACLE_MAX_NODES];
+    for (int i = 0; i < N; ++i) {
+        ok[i] = 1;
+        ll[i] = 0.0;
+        for (int j = 0; j < N; ++j)
+            if (j != 0 && in_anc[(size_t)i * N + j]) {
+                if (!(p_edge[j] > thr[j]))
+                    ok[i] = 0;
+                ll[i] += p_edge[j] > 0.0 ? log(p_edge[j]) : -INFINITY;
+            }
+    }
+    int best = 0;
+    for (int i = 1; i < N; ++i) {
+        if (!ok[i])
+            continue;
+        if (depth[i] > depth[best] || (depth[i] == depth[best] && ll[i] > ll[best]))
+            best = i;
+    }
+    const int len = depth[best] + 1;
+    for (int j = best, pos = len - 1; pos >= 0; --pos) {
+        path[pos] = j;
+        j = (j == 0) ? -1 : parent[j];
+    }
+    *accept_len = len;
+    *bonus = amax[best];
+    for (int j = 0; j < N; ++j) {
+        if (margin)
+            margin[j] = (j == 0 || thr[j] == 0.0) ? 0.0 : (p_edge[j] - thr[j]) / thr[j];
+        if (loglik)
+            loglik[j] = ll[j];
+        if (accepted)
+            accepted[j] = ok[j];
+    }
     return 0;
 }
