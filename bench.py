@@ -142,6 +142,12 @@ def kernel_source_hash(files: str) -> str:
     return h.hexdigest()[:16]
 
 
+def acceptance_label(args) -> str:
+    if getattr(args, "accept", "greedy") == "typical":
+        return "typical (T=0.7, eps=0.09, alpha=0.3)"
+    return "greedy"
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -183,8 +189,15 @@ def run_gpu(args):
     torch.cuda.synchronize()
     drafts = torch.from_numpy(synth.gen_drafts(seed, sh.parent, am.cpu().numpy(), V, sh.p_match)).to(dev)
 
+    typical = args.accept == "typical"
+    lz, et, dl = (torch.empty(N, dtype=torch.float32, device=dev) for _ in range(3))
+
     def step():
-        tv.verify_step(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, 0, stream)
+        if typical:
+            tv.verify_step_typical(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, *tv.PAPER_TYPICAL,
+                                   0, stream)
+        else:
+            tv.verify_step(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, 0, stream)
 
     visible = os.environ.get("CUDA_VISIBLE_DEVICES")
     sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
@@ -215,11 +228,18 @@ def run_gpu(args):
     torch.cuda._sleep(200_000_000)
     for i in range(n_k):
         ev[i][0].record(stream)
-        tv.lm_head_stats(hidden, W, am, t1, en, ws, stream)
+        if typical:
+            tv.lm_head_stats_typical(bank, bid, hidden, W, tv.PAPER_TYPICAL[0], drafts, am, t1, en, lz, et, dl, ws,
+                                     stream)
+        else:
+            tv.lm_head_stats(hidden, W, am, t1, en, ws, stream)
         ev[i][1].record(stream)
         tv.tree_attention(bank, bid, kv, q, out, ws, 0, nl, stream)
         ev[i][2].record(stream)
-        tv.greedy_accept(bank, bid, drafts, am, V, L, res, stream)
+        if typical:
+            tv.typical_accept(bank, bid, drafts, am, lz, et, dl, V, L, res, *tv.PAPER_TYPICAL, stream=stream)
+        else:
+            tv.greedy_accept(bank, bid, drafts, am, V, L, res, stream)
         tv.kv_compact(kv, res, stream)
         ev[i][3].record(stream)
     torch.cuda.synchronize()
@@ -282,7 +302,8 @@ def run_gpu(args):
                 "drafts = parent greedy token with p, else uniform",
         "config": {"workload": sh.name, "layers": nl, "q_heads": H, "kv_heads": Hkv, "head_dim": d, "L": L,
                    "tree_nodes": N, "tree_depth": int(synth.depth_of(sh.parent).max()), "d_model": D, "vocab": V,
-                   "batch": 1, "l2": f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)"},
+                   "batch": 1, "l2": f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)",
+                   "acceptance": acceptance_label(args)},
         "tree_tokens_per_s": round(value * N, 1),
         "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
                          "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
@@ -358,7 +379,11 @@ def run_gpu_batched(args):
     stream = torch.cuda.current_stream()
 
     def step():
-        tv.verify_step_batched(bank, seqs, hidden, W, am, t1, en, ws, tv.TB_NO_COMPACT, stream)
+        if args.accept == "typical":
+            tv.verify_step_batched_typical(bank, seqs, hidden, W, am, t1, en, ws, *tv.PAPER_TYPICAL,
+                                           tv.TB_NO_COMPACT, stream)
+        else:
+            tv.verify_step_batched(bank, seqs, hidden, W, am, t1, en, ws, tv.TB_NO_COMPACT, stream)
 
     sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]
                            if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
@@ -396,7 +421,8 @@ def run_gpu_batched(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded)",
         "config": {"workload": sh.name, "batch": len(sh.parents), "tree_nodes": sh.Ns, "L": sh.Ls, "q_heads": Hq,
                    "kv_heads": Hkv, "head_dim": d, "d_model": D, "vocab": V,
-                   "l2": "256 MB flush before every step (the batch's KV fits in L2)"},
+                   "l2": "256 MB flush before every step (the batch's KV fits in L2)",
+                   "acceptance": acceptance_label(args)},
         "tree_tokens_per_s": round(value * R, 1),
         "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
                      "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
@@ -605,7 +631,11 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
+                    help="verification rule: greedy (default) or typical acceptance at T=0.7, eps=0.09, alpha=0.3")
     args = ap.parse_args(argv)
+    if args.accept == "typical" and (args.impl == "reference" or args.config == "c3"):
+        ap.error("--accept typical applies to the GPU arm of c1, c2, c4 and c5")
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":

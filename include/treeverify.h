@@ -290,6 +290,64 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
 TB_API tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
                                        int32_t *argmax, float *top1, float *entropy, tb_stream stream);
 
+/* ------------------------------------------------------------------------
+ * Typical acceptance: the Medusa/Hydra verification rule that the paper keeps
+ * unchanged and runs with T = 0.7, eps = 0.09, alpha = 0.3 (Sec. 5.1, 5.2).
+ * ---------------------------------------------------------------------- */
+
+/* Parameters of the rule (host struct, read at call time). */
+typedef struct tb_typical {
+    float temperature; /* T > 0: the target distribution is softmax(z / T) */
+    float eps;         /* posterior threshold epsilon >= 0 */
+    float alpha;       /* mixing coefficient alpha >= 0 */
+    int32_t reserved;  /* 0 */
+} tb_typical;
+
+/* lm_head_stats over the N node rows of topology bank_id (canonical order)
+ * plus, from the same pass over W, what typical acceptance consumes:
+ *   logz_t[r]      = ln sum_v e^(z_r[v] / T)              (log-partition at T)
+ *   entropy_t[r]   = -sum_v p ln p with p = softmax(z_r / T) (nats)
+ *   draft_logit[j] = z_{parent(j)}[draft_tokens[j]] for every non-root node j
+ *                    whose draft token lies in [0, vocab); other entries are
+ *                    left unwritten.
+ *   hidden bf16 [N][d_model]; draft_tokens device int32 [N];
+ *   argmax int32, top1 / entropy / logz_t / entropy_t / draft_logit float,
+ *   all device [N].  top1 and entropy stay at temperature 1. */
+TB_API tb_status lm_head_stats_typical(const tb_bank *bank, int bank_id, const void *hidden, const void *lm_head,
+                                       int d_model, int vocab, float temperature, const int32_t *draft_tokens,
+                                       int32_t *argmax, float *top1, float *entropy, float *logz_t, float *entropy_t,
+                                       float *draft_logit, void *workspace, size_t workspace_bytes, tb_stream stream);
+
+/* Typical acceptance over topology bank_id: the edge into non-root node j
+ * passes when
+ *   p_j = e^(draft_logit[j] / T - logz_t[parent(j)]) > min(eps, alpha e^(-entropy_t[parent(j)])),
+ * node i is accepted when every edge of its root path passes, and j* is the
+ * deepest accepted node with the largest path log-likelihood sum ln p_j over
+ * its edges (smallest canonical id on exact ties).  Writes *result as
+ * greedy_accept does, bonus_token = argmax[j*]; a draft token outside
+ * [0, vocab) never passes and sets status TB_EINVAL.  All arrays are device
+ * [N] in canonical node order (the outputs of lm_head_stats_typical). */
+TB_API tb_status typical_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens,
+                                const int32_t *argmax, const float *logz_t, const float *entropy_t,
+                                const float *draft_logit, int vocab, int L, const tb_typical *params,
+                                tb_result *result, tb_stream stream);
+
+/* verify_step with typical acceptance: the LM-head pass also produces the
+ * tempered statistics and draft logits (kept in the workspace) and the
+ * acceptance follows typical_accept.  Arguments as for verify_step. */
+TB_API tb_status verify_step_typical(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q,
+                                     int n_q_heads, const void *hidden, const void *lm_head, int d_model, int vocab,
+                                     const int32_t *draft_tokens, void *attn_out, int32_t *argmax, float *top1,
+                                     float *entropy, const tb_typical *params, tb_result *result, void *workspace,
+                                     size_t workspace_bytes, int flags, tb_stream stream);
+
+/* verify_step_batched with typical acceptance (same parameters for every
+ * sequence).  Arguments as for verify_step_batched. */
+TB_API tb_status verify_step_batched_typical(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                             const void *hidden, const void *lm_head, int d_model, int vocab,
+                                             int32_t *argmax, float *top1, float *entropy, const tb_typical *params,
+                                             void *workspace, size_t workspace_bytes, int flags, tb_stream stream);
+
 /* Message for the last failing call on this thread ("" if none). */
 TB_API const char *tb_last_error(void);
 

@@ -49,6 +49,8 @@ def _load():
             d = ctypes.c_double
             lib.oracle_typical_accept.argtypes = [P, i32, P, P, i32, d, d, d, P, P, P, P, P, P]
             lib.oracle_typical_accept.restype = ctypes.c_int
+            lib.oracle_tempered_stats.argtypes = [P, i32, i32, d, P, P]
+            lib.oracle_tempered_stats.restype = ctypes.c_int
             for f in (lib.oracle_tree, lib.oracle_tree_attention, lib.oracle_lm_head,
                       lib.oracle_accept, lib.oracle_num_threads):
                 f.restype = ctypes.c_int
@@ -171,3 +173,14 @@ def typical_accept(parent, draft, logits, temperature: float, eps: float, alpha:
     if detail:
         return out + ({"margin": margin, "loglik": loglik, "accepted": acc.astype(bool)},)
     return out
+
+
+def tempered_stats(logits, temperature: float):
+    """(logz float64[R], entropy float64[R]) of softmax(logits / T) per row."""
+    logits = np.ascontiguousarray(logits, dtype=np.float64)
+    R, V = logits.shape
+    logz = np.zeros(R)
+    ent = np.zeros(R)
+    if _load().oracle_tempered_stats(_ptr(logits), R, V, temperature, _ptr(logz), _ptr(ent)) != 0:
+        raise ValueError("bad shape or temperature")
+    return logz, ent

@@ -354,3 +354,35 @@ int oracle_typical_accept(const int32_t *parent, int N, const int32_t *draft, co
     }
     return 0;
 }
+
+/*
+ * Statistics of the tempered target distribution p = softmax(z / T) of each
+ * row (the quantities typical acceptance reads, Sec. 5.1/5.2 settings):
+ *   logz[r] = ln sum_v e^(z_r[v] / T)       (log-partition)
+ *   ent[r]  = -sum_v p_r(v) ln p_r(v)       (entropy, nats)
+ * logits [R][V] (double).
+ */
+int oracle_tempered_stats(const double *logits, int R, int V, double temperature, double *logz, double *ent)
+{
+    if (R < 0 || V < 1 || !(temperature > 0.0))
+        return -1;
+    for (int r = 0; r < R; ++r) {
+        const double *z = logits + (size_t)r * V;
+        double m = z[0];
+        for (int v = 1; v < V; ++v)
+            if (z[v] > m)
+                m = z[v];
+        double denom = 0.0;
+        for (int v = 0; v < V; ++v)
+            denom += exp((z[v] - m) / temperature);
+        double h = 0.0;
+        for (int v = 0; v < V; ++v) {
+            const double p = exp((z[v] - m) / temperature) / denom;
+            if (p > 0.0)
+                h -= p * log(p);
+        }
+        logz[r] = m / temperature + log(denom);
+        ent[r] = h;
+    }
+    return 0;
+}

@@ -30,7 +30,8 @@ RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
        "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error",
-       "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder")
+       "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
+       "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical")
 
 
 class TreeVerifyError(RuntimeError):
@@ -49,6 +50,14 @@ class TbSeq(ctypes.Structure):
     _fields_ = [("bank_id", ctypes.c_int32), ("reserved", ctypes.c_int32), ("kv", TbKv), ("q", ctypes.c_void_p),
                 ("draft_tokens", ctypes.c_void_p), ("attn_out", ctypes.c_void_p), ("result", ctypes.c_void_p)]
 
+
+class TbTypical(ctypes.Structure):
+    _fields_ = [("temperature", ctypes.c_float), ("eps", ctypes.c_float), ("alpha", ctypes.c_float),
+                ("reserved", ctypes.c_int32)]
+
+
+# the paper's verification settings (temperature, posterior threshold, mixing coefficient)
+PAPER_TYPICAL = (0.7, 0.09, 0.3)
 
 TB_MAX_BATCH = 16
 
@@ -81,6 +90,10 @@ def load(path: str = LIB_PATH):
         "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, P],
         "verify_step_batched": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, sz, i32, P],
         "tb_last_error": [],
+        "lm_head_stats_typical": [P, i32, P, P, i32, i32, ctypes.c_float, P, P, P, P, P, P, P, P, sz, P],
+        "typical_accept": [P, i32, P, P, P, P, P, i32, i32, P, P, P],
+        "verify_step_typical": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, P, sz, i32, P],
+        "verify_step_batched_typical": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, P, sz, i32, P],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -301,6 +314,51 @@ def verify_step_batched(bank: Bank, seqs, hidden, lm_head, argmax, top1, entropy
     _check(load().verify_step_batched(bank.handle, len(seqs), arr, seqs[0].q.shape[2], _ptr(hidden), _ptr(lm_head),
                                       hidden.shape[1], lm_head.shape[0], _ptr(argmax), _ptr(top1), _ptr(entropy),
                                       _ptr(ws), ws.numel(), flags, _stream(stream)), "verify_step_batched")
+
+
+# --------------------------------------------------------------------- typical acceptance
+
+
+def _typical(temperature: float, eps: float, alpha: float) -> TbTypical:
+    return TbTypical(float(temperature), float(eps), float(alpha), 0)
+
+
+def lm_head_stats_typical(bank: Bank, bank_id: int, hidden, lm_head, temperature: float, draft, argmax, top1, entropy,
+                          logz_t, entropy_t, draft_logit, ws, stream=None):
+    """hidden bf16 [N][d_model] (the tree's rows); every output [N]."""
+    _check(load().lm_head_stats_typical(bank.handle, bank_id, _ptr(hidden), _ptr(lm_head), hidden.shape[1],
+                                        lm_head.shape[0], float(temperature), _ptr(draft), _ptr(argmax), _ptr(top1),
+                                        _ptr(entropy), _ptr(logz_t), _ptr(entropy_t), _ptr(draft_logit), _ptr(ws),
+                                        ws.numel(), _stream(stream)), "lm_head_stats_typical")
+
+
+def typical_accept(bank: Bank, bank_id: int, draft, argmax, logz_t, entropy_t, draft_logit, vocab: int, L: int,
+                   result, temperature: float, eps: float, alpha: float, stream=None):
+    t = _typical(temperature, eps, alpha)
+    _check(load().typical_accept(bank.handle, bank_id, _ptr(draft), _ptr(argmax), _ptr(logz_t), _ptr(entropy_t),
+                                 _ptr(draft_logit), vocab, L, ctypes.byref(t), _ptr(result), _stream(stream)),
+           "typical_accept")
+
+
+def verify_step_typical(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft, attn_out, argmax, top1,
+                        entropy, result, ws, temperature: float, eps: float, alpha: float, flags: int = 0,
+                        stream=None):
+    c = kv.as_c()
+    t = _typical(temperature, eps, alpha)
+    _check(load().verify_step_typical(bank.handle, bank_id, ctypes.byref(c), _ptr(q), q.shape[2], _ptr(hidden),
+                                      _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(draft), _ptr(attn_out),
+                                      _ptr(argmax), _ptr(top1), _ptr(entropy), ctypes.byref(t), _ptr(result),
+                                      _ptr(ws), ws.numel(), flags, _stream(stream)), "verify_step_typical")
+
+
+def verify_step_batched_typical(bank: Bank, seqs, hidden, lm_head, argmax, top1, entropy, ws, temperature: float,
+                                eps: float, alpha: float, flags: int = 0, stream=None):
+    arr = (TbSeq * len(seqs))(*[s.as_c() for s in seqs])
+    t = _typical(temperature, eps, alpha)
+    _check(load().verify_step_batched_typical(bank.handle, len(seqs), arr, seqs[0].q.shape[2], _ptr(hidden),
+                                              _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(argmax),
+                                              _ptr(top1), _ptr(entropy), ctypes.byref(t), _ptr(ws), ws.numel(),
+                                              flags, _stream(stream)), "verify_step_batched_typical")
 
 
 # --------------------------------------------------------------------- per-step tree selection

@@ -17,6 +17,13 @@
 // earlier copy overwrote; one warp copies one (layer, head, K|V) row set in
 // that order, with a warp barrier between rows.
 //
+// Typical acceptance (the Medusa/Hydra rule the paper keeps, Sec. 5.1/5.2):
+// edge j passes when p_T(draft[j] | parent) > min(eps, alpha e^(-H_T(parent))),
+// with p_T = e^(z / T - logZ_T) from the LM head's tempered statistics and
+// gathered draft logit.  Accepted nodes follow from the same bitset test;
+// among the deepest the largest path log-likelihood sum ln p_T wins (smallest
+// id on exact ties), and the bonus token is still argmax[j*].
+//
 // Every CTA recomputes the (tiny) acceptance itself, so acceptance and
 // compaction run as one launch without a grid-wide barrier.
 #include "kernels.cuh"
@@ -46,6 +53,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
 {
     const AcceptParams &p = pb.seq[blockIdx.y];
     __shared__ int s_path[kMaxNodes];
+    __shared__ float s_lp[kMaxNodes];
     __shared__ int s_len;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -67,30 +75,91 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                 bool m = false;
                 if (i >= 1 && i < n) {
                     const int tok = p.draft[i];
-                    bad |= (tok < 0 || tok >= p.vocab);
-                    m = (tok == p.argmax[t->parent[i]]);
+                    const bool bad_tok = (tok < 0 || tok >= p.vocab);
+                    bad |= bad_tok;
+                    if (!p.typical) {
+                        m = (tok == p.argmax[t->parent[i]]);
+                    } else {
+                        const int u = t->parent[i];
+                        float lp = -INFINITY;
+                        if (!bad_tok) {
+                            lp = p.draft_logit[i] * p.inv_t - p.logz_t[u];
+                            const float thr = fminf(p.eps, p.alpha * expf(-p.ent_t[u]));
+                            m = expf(lp) > thr;
+                        }
+                        s_lp[i] = lp;
+                    }
                 }
                 const uint32_t bits = __ballot_sync(0xffffffffu, m);
                 match |= (uint64_t)bits << (32 * h);
             }
             const bool any_bad = __any_sync(0xffffffffu, bad);
-            // key = depth * 128 + (127 - id): the max is the deepest, smallest-id accepted node
-            int best = 127;  // the root (depth 0, id 0) is always accepted
+            int jstar;
+            if (!p.typical) {
+                // key = depth * 128 + (127 - id): the max is the deepest, smallest-id accepted node
+                int best = 127;  // the root (depth 0, id 0) is always accepted
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int i = lane + 32 * h;
-                if (i < n) {
-                    const uint64_t a = t->anc[i];
-                    if ((a & ~match & ~1ull) == 0ull) {
-                        const int key = t->depth[i] * 128 + (127 - i);
-                        best = max(best, key);
+                for (int h = 0; h < 2; ++h) {
+                    const int i = lane + 32 * h;
+                    if (i < n) {
+                        const uint64_t a = t->anc[i];
+                        if ((a & ~match & ~1ull) == 0ull) {
+                            const int key = t->depth[i] * 128 + (127 - i);
+                            best = max(best, key);
+                        }
                     }
                 }
-            }
 #pragma unroll
-            for (int m = 16; m >= 1; m >>= 1)
-                best = max(best, __shfl_xor_sync(0xffffffffu, best, m));
-            const int jstar = 127 - (best & 127);
+                for (int m = 16; m >= 1; m >>= 1)
+                    best = max(best, __shfl_xor_sync(0xffffffffu, best, m));
+                jstar = 127 - (best & 127);
+            } else {
+                __syncwarp();
+                // accepted nodes, their depth and path log-likelihood (edges in increasing id)
+                int dep[2];
+                float ll[2];
+                int bdep = 0;  // the root is always accepted
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int i = lane + 32 * h;
+                    dep[h] = -1;
+                    ll[h] = -INFINITY;
+                    if (i < n) {
+                        uint64_t a = t->anc[i];
+                        if ((a & ~match & ~1ull) == 0ull) {
+                            float acc = 0.f;
+                            a &= ~1ull;
+                            while (a) {
+                                acc += s_lp[__ffsll((long long)a) - 1];
+                                a &= a - 1;
+                            }
+                            dep[h] = t->depth[i];
+                            ll[h] = acc;
+                            bdep = max(bdep, dep[h]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int m = 16; m >= 1; m >>= 1)
+                    bdep = max(bdep, __shfl_xor_sync(0xffffffffu, bdep, m));
+                float bll = -INFINITY;
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    if (dep[h] == bdep)
+                        bll = fmaxf(bll, ll[h]);
+#pragma unroll
+                for (int m = 16; m >= 1; m >>= 1)
+                    bll = fmaxf(bll, __shfl_xor_sync(0xffffffffu, bll, m));
+                int bid = kMaxNodes;
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    if (dep[h] == bdep && ll[h] == bll)
+                        bid = min(bid, lane + 32 * h);
+#pragma unroll
+                for (int m = 16; m >= 1; m >>= 1)
+                    bid = min(bid, __shfl_xor_sync(0xffffffffu, bid, m));
+                jstar = bid < n ? bid : 0;
+            }
             const uint64_t pa = t->anc[jstar];
             const int len = __popcll(pa);
 #pragma unroll

@@ -12,9 +12,28 @@ struct LmPlan {
     size_t ws_bytes;  // partials (tile + group), 256-byte aligned
 };
 LmPlan lm_plan(int R, int D, int V);
+// typical-acceptance inputs produced by the same pass: per-row statistics at
+// temperature T and the draft-token logit of every tree edge j, written to
+// seq[b].out[j] for edges whose parent row row_base + parent[j] is in [0, R)
+struct LmGatherSeq {
+    const TreeDesc *tree;
+    const int32_t *draft;
+    float *out;
+    int row_base, n;
+};
+struct LmGather {
+    LmGatherSeq seq[TB_MAX_BATCH];
+    int n_seq;
+};
+struct LmTypical {
+    float temperature;
+    float *logz_t;
+    float *ent_t;
+    LmGather gather;
+};
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
-                           const char **err, int expire_wait = 0);
+                           const char **err, int expire_wait = 0, const LmTypical *typ = nullptr);
 
 // tree attention (attention.cu)
 struct AttnPlan {
@@ -53,6 +72,11 @@ struct AcceptParams {
     const int32_t *draft;
     const int32_t *argmax;
     int vocab, L;
+    // typical acceptance (typical != 0): per-row tempered log-partition and
+    // entropy (indexed by node) and per-edge draft-token logits
+    int typical;
+    float inv_t, eps, alpha;
+    const float *logz_t, *ent_t, *draft_logit;
     tb_result *result;
     const int *ws_status;  // may be null
     // compaction (n_layers == 0: acceptance only)

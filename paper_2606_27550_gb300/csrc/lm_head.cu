@@ -17,6 +17,14 @@
 // and reduce each row.  Per-tile statistics are merged in two levels by
 // atomic arrival tickets (the last CTA of a group merges the group; the last
 // group merges everything); no CTA ever waits for another.
+//
+// Typical-acceptance mode (kTyp): the same pass also yields, per row, the
+// statistics of the tempered distribution softmax(z / T) -- its log-partition
+// logZ_T = m / T + ln sum e^((z-m)/T) and entropy H_T -- and gathers the logit
+// z_{parent(j)}[draft[j]] of every tree edge j straight from the tile's logits
+// in shared memory (the Medusa/Hydra typical-acceptance inputs, Sec. 5.1/5.2).
+// Warps 2-3, idle during the k-loop, find the edges whose token falls in this
+// CTA's vocab tile meanwhile.
 #include <math.h>
 #include <stdlib.h>
 
@@ -39,24 +47,34 @@ struct LmParams {
     int32_t *argmax;
     float *top1;
     float *entropy;
+    // typical-acceptance mode
+    float inv_t;          // 1 / T
+    float2 *part_tile_t;  // [n_tiles][R_pad]  (sT, tT)
+    float2 *part_group_t; // [n_groups][R_pad]
+    float *logz_t;        // [R] m / T + ln sT
+    float *ent_t;         // [R] ln sT - tT / sT
+    LmGather gather;
 };
 
 struct RowStat {
-    float m;  // running max logit
-    int idx;  // its vocab index (lowest on ties)
-    float s;  // sum e^(z - m)
-    float t;  // sum e^(z - m) (z - m)
+    float m;   // running max logit
+    int idx;   // its vocab index (lowest on ties)
+    float s;   // sum e^(z - m)
+    float t;   // sum e^(z - m) (z - m)
+    float sT;  // sum e^((z - m) / T)          (typical mode)
+    float tT;  // sum e^((z - m) / T) (z - m) / T
 };
 
 constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ RowStat stat_empty()
 {
-    return RowStat{-INFINITY, 0x7fffffff, 0.f, 0.f};
+    return RowStat{-INFINITY, 0x7fffffff, 0.f, 0.f, 0.f, 0.f};
 }
 
 // Combines the statistics of two disjoint vocab subsets.
-__device__ __forceinline__ RowStat stat_merge(RowStat a, RowStat b)
+template <bool kTyp>
+__device__ __forceinline__ RowStat stat_merge(RowStat a, RowStat b, float inv_t)
 {
     if (b.m > a.m || (b.m == a.m && b.idx < a.idx)) {
         RowStat x = a;
@@ -69,9 +87,16 @@ __device__ __forceinline__ RowStat stat_merge(RowStat a, RowStat b)
     const float e = ex2_approx(delta * kLog2e);
     a.s += b.s * e;
     a.t += (b.t + delta * b.s) * e;
+    if constexpr (kTyp) {
+        const float dT = delta * inv_t;
+        const float eT = ex2_approx(dT * kLog2e);
+        a.sT += b.sT * eT;
+        a.tT += (b.tT + dT * b.sT) * eT;
+    }
     return a;
 }
 
+template <bool kTyp>
 __device__ __forceinline__ RowStat stat_shfl_xor(RowStat a, int mask)
 {
     RowStat b;
@@ -79,6 +104,10 @@ __device__ __forceinline__ RowStat stat_shfl_xor(RowStat a, int mask)
     b.idx = __shfl_xor_sync(0xffffffffu, a.idx, mask);
     b.s = __shfl_xor_sync(0xffffffffu, a.s, mask);
     b.t = __shfl_xor_sync(0xffffffffu, a.t, mask);
+    if constexpr (kTyp) {
+        b.sT = __shfl_xor_sync(0xffffffffu, a.sT, mask);
+        b.tT = __shfl_xor_sync(0xffffffffu, a.tT, mask);
+    }
     return b;
 }
 
@@ -89,7 +118,7 @@ __device__ __forceinline__ float4 stat_pack(RowStat a)
 
 __device__ __forceinline__ RowStat stat_unpack(float4 v)
 {
-    return RowStat{v.x, __float_as_int(v.y), v.z, v.w};
+    return RowStat{v.x, __float_as_int(v.y), v.z, v.w, 0.f, 0.f};
 }
 
 // Threads per row for per-row scans by the 128 threads of a CTA: the largest
@@ -103,11 +132,25 @@ __device__ __forceinline__ int threads_per_row(int R_pad)
 }
 
 // Combines the statistics held by the tpr consecutive lanes of each row group.
-__device__ __forceinline__ RowStat group_merge(RowStat st, int tpr)
+template <bool kTyp>
+__device__ __forceinline__ RowStat group_merge(RowStat st, int tpr, float inv_t)
 {
     for (int m = 1; m < tpr; m <<= 1)
-        st = stat_merge(st, stat_shfl_xor(st, m));
+        st = stat_merge<kTyp>(st, stat_shfl_xor<kTyp>(st, m), inv_t);
     return st;
+}
+
+// Writes the draft-token logit of tree edge (sequence b, node j) when its
+// parent row lies in this launch and its token in this CTA's vocab tile.
+__device__ __forceinline__ bool gather_hit(const LmGather &g, int b, int j, int R, int v0, int nvalid, int *row,
+                                           int *col)
+{
+    const LmGatherSeq &sq = g.seq[b];
+    const int r = sq.row_base + sq.tree->parent[j];
+    const int c = sq.draft[j] - v0;
+    *row = r;
+    *col = c;
+    return r >= 0 && r < R && c >= 0 && c < nvalid;
 }
 
 // Merges count x R_pad partials (global, written by other CTAs): they are
@@ -115,7 +158,9 @@ __device__ __forceinline__ RowStat group_merge(RowStat st, int tpr)
 // independent passes (max / first argmax, then the rescaled sums), so there is
 // no serial dependency chain per row.  Writes the merged partial (dst) or the
 // final per-row outputs.
-__device__ void merge_partials(const LmParams &p, const float4 *src, int count, float4 *sbuf, float4 *dst)
+template <bool kTyp>
+__device__ void merge_partials(const LmParams &p, const float4 *src, const float2 *src_t, int count, float4 *sbuf,
+                               float4 *dst, float2 *dst_t)
 {
     const int n = count * p.R_pad;
     for (int i = threadIdx.x; i < n; i += blockDim.x)
@@ -143,24 +188,40 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, int count, 
                         const float e = ex2_approx(delta * kLog2e);
                         st.s += v.z * e;
                         st.t += (v.w + delta * v.z) * e;
+                        if constexpr (kTyp) {
+                            // the tempered sums are read once, straight from L2
+                            const float2 w = __ldcg(src_t + (size_t)k * p.R_pad + r);
+                            const float dT = delta * p.inv_t;
+                            const float eT = ex2_approx(dT * kLog2e);
+                            st.sT += w.x * eT;
+                            st.tT += (w.y + dT * w.x) * eT;
+                        }
                     }
                 }
             }
         }
-        st = group_merge(st, tpr);
+        st = group_merge<kTyp>(st, tpr, p.inv_t);
         if (sub == 0 && r < p.R) {
             if (dst) {
                 dst[r] = stat_pack(st);
+                if constexpr (kTyp)
+                    dst_t[r] = make_float2(st.sT, st.tT);
             } else {
                 p.argmax[r] = st.idx;
                 p.top1[r] = 1.0f / st.s;
                 p.entropy[r] = logf(st.s) - st.t / st.s;
+                if constexpr (kTyp) {
+                    const float ls = logf(st.sT);
+                    p.logz_t[r] = st.m * p.inv_t + ls;
+                    p.ent_t[r] = ls - st.tT / st.sT;
+                }
             }
         }
     }
     __syncthreads();
 }
 
+template <bool kTyp>
 __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -171,6 +232,11 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
     __shared__ int ticket;
+    // typical mode: edges whose draft token lies in this tile, packed as
+    // (seq << 24) | (node << 16) | (row << 7) | col; overflow -> rescan in the epilogue
+    constexpr int kHitCap = 64;
+    __shared__ int s_hit[kTyp ? kHitCap : 1];
+    __shared__ int s_nhit;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = p.stages;
@@ -193,6 +259,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
         mbar_init(&acc_bar, 1);
         mbar_init(&never_bar, 1);
         abort_flag = 0;
+        s_nhit = 0;
         fence_mbar_init();
         prefetch_tmap(&p.tmap_w);
         prefetch_tmap(&p.tmap_h);
@@ -256,6 +323,19 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             tc_commit(&empty_bar[s]);
         }
         tc_commit(&acc_bar);
+    } else if (kTyp && warp >= 2) {
+        // ---------------- edges to gather (warps 2-3 are otherwise idle here)
+        const int nvalid = min(128, p.V - v0);
+        for (int b = 0; b < p.gather.n_seq; ++b) {
+            for (int j = 1 + (threadIdx.x - 64); j < p.gather.seq[b].n; j += 64) {
+                int row, col;
+                if (gather_hit(p.gather, b, j, p.R, v0, nvalid, &row, &col)) {
+                    const int slot = atomicAdd(&s_nhit, 1);
+                    if (slot < kHitCap)
+                        s_hit[slot] = (b << 24) | (j << 16) | (row << 7) | col;
+                }
+            }
+        }
     }
     __syncwarp();
 
@@ -310,11 +390,37 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
                     const float e = ex2_approx(dz * kLog2e);
                     st.s += e;
                     st.t += e * dz;
+                    if constexpr (kTyp) {
+                        const float dT = dz * p.inv_t;
+                        const float eT = ex2_approx(dT * kLog2e);
+                        st.sT += eT;
+                        st.tT += eT * dT;
+                    }
                 }
             }
-            st = group_merge(st, tpr);
-            if (sub == 0 && r < p.R)
+            st = group_merge<kTyp>(st, tpr, p.inv_t);
+            if (sub == 0 && r < p.R) {
                 p.part_tile[(size_t)tile * p.R_pad + r] = stat_pack(st);
+                if constexpr (kTyp)
+                    p.part_tile_t[(size_t)tile * p.R_pad + r] = make_float2(st.sT, st.tT);
+            }
+        }
+        if constexpr (kTyp) {
+            const int nhit = s_nhit;
+            if (nhit <= kHitCap) {
+                for (int i = threadIdx.x; i < nhit; i += blockDim.x) {
+                    const int w = s_hit[i];
+                    const int b = w >> 24, j = (w >> 16) & 0xff, row = (w >> 7) & 0x1ff, col = w & 0x7f;
+                    p.gather.seq[b].out[j] = logits[row * ld + col];
+                }
+            } else {
+                for (int b = 0; b < p.gather.n_seq; ++b)
+                    for (int j = 1 + threadIdx.x; j < p.gather.seq[b].n; j += blockDim.x) {
+                        int row, col;
+                        if (gather_hit(p.gather, b, j, p.R, v0, nvalid, &row, &col))
+                            p.gather.seq[b].out[j] = logits[row * ld + col];
+                    }
+            }
         }
     }
 
@@ -331,7 +437,8 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
         return;
     __threadfence();
     float4 *sbuf = reinterpret_cast<float4 *>(smem);
-    merge_partials(p, p.part_tile + (size_t)g_first * p.R_pad, g_count, sbuf, p.part_group + (size_t)g * p.R_pad);
+    merge_partials<kTyp>(p, p.part_tile + (size_t)g_first * p.R_pad, p.part_tile_t + (size_t)g_first * p.R_pad,
+                         g_count, sbuf, p.part_group + (size_t)g * p.R_pad, p.part_group_t + (size_t)g * p.R_pad);
     if (threadIdx.x == 0)
         p.counters[g] = 0;
     __threadfence();
@@ -342,7 +449,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     if (ticket != p.n_groups - 1)
         return;
     __threadfence();
-    merge_partials(p, p.part_group, p.n_groups, sbuf, nullptr);
+    merge_partials<kTyp>(p, p.part_group, p.part_group_t, p.n_groups, sbuf, nullptr, nullptr);
     if (threadIdx.x == 0)
         p.counters[p.n_groups] = 0;
 }
@@ -399,13 +506,14 @@ LmPlan lm_plan(int R, int D, int V)
     if (mg > sm)
         sm = mg;
     pl.smem_bytes = sm + 1024;
-    pl.ws_bytes = ((size_t)pl.n_tiles * pl.R_pad * 16 + (size_t)pl.n_groups * pl.R_pad * 16 + 255) / 256 * 256;
+    // (max, argmax, s, t) partials, then the tempered (sT, tT) partials of typical mode
+    pl.ws_bytes = ((size_t)(pl.n_tiles + pl.n_groups) * pl.R_pad * (16 + 8) + 255) / 256 * 256;
     return pl;
 }
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
-                           const char **err, int expire_wait)
+                           const char **err, int expire_wait, const LmTypical *typ)
 {
     const LmPlan pl = lm_plan(R, D, V);
     LmParams p{};
@@ -432,10 +540,24 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.top1 = top1;
     p.entropy = entropy;
     p.expire_wait = expire_wait;
-    cudaError_t e = allow_max_smem((const void *)k2_lm_head);
-    if (e != cudaSuccess)
-        return e;
-    k2_lm_head<<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+    p.part_tile_t = reinterpret_cast<float2 *>(p.part_group + (size_t)pl.n_groups * pl.R_pad);
+    p.part_group_t = p.part_tile_t + (size_t)pl.n_tiles * pl.R_pad;
+    if (typ) {
+        p.inv_t = 1.0f / typ->temperature;
+        p.logz_t = typ->logz_t;
+        p.ent_t = typ->ent_t;
+        p.gather = typ->gather;
+        cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
+        if (e != cudaSuccess)
+            return e;
+        k2_lm_head<true><<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+    } else {
+        p.inv_t = 1.0f;
+        cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
+        if (e != cudaSuccess)
+            return e;
+        k2_lm_head<false><<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+    }
     return cudaGetLastError();
 }
 

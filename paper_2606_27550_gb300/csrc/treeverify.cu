@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -139,6 +140,7 @@ bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_h
 //   [0, 256)                    status word
 //   [256, 256 + 64 KiB)         attention unit counters (16384 int32)
 //   [.., + 4 KiB)               LM-head group counters (1024 int32)
+//   [.., + 12 KiB)              typical acceptance: logZ_T, H_T, draft logits (3 x 1024 float)
 //   [kPartBase, ..)             attention partials, then LM-head partials
 // Counters sit at fixed offsets so that calls of different shapes sharing one
 // workspace always find them zero; partials are written before they are read.
@@ -147,7 +149,9 @@ constexpr size_t kAttnCounterOff = 256;
 constexpr int kMaxAttnUnits = 16384;
 constexpr size_t kLmCounterOff = kAttnCounterOff + (size_t)kMaxAttnUnits * 4;
 constexpr int kMaxLmCounters = 1024;
-constexpr size_t kPartBase = kLmCounterOff + (size_t)kMaxLmCounters * 4;
+constexpr int kMaxTypRows = 1024;
+constexpr size_t kTypOff = kLmCounterOff + (size_t)kMaxLmCounters * 4;
+constexpr size_t kPartBase = kTypOff + (size_t)3 * kMaxTypRows * 4;
 
 static size_t align256(size_t x)
 {
@@ -582,12 +586,13 @@ static tb_status lm_validate(const void *hidden, int R, const void *W, int D, in
 }
 
 static tb_status lm_enqueue(const void *hidden, int R, const void *W, int D, int V, int32_t *am, float *t1, float *en,
-                            uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn, int expire_wait = 0)
+                            uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn, int expire_wait = 0,
+                            const LmTypical *typ = nullptr)
 {
     const char *err = "";
     cudaError_t e = lm_head_launch(hidden, R, W, D, V, am, t1, en, ws + part_off,
                                    reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws), stream,
-                                   &err, expire_wait);
+                                   &err, expire_wait, typ);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -607,6 +612,39 @@ static AcceptParams accept_params(const tb_bank *bank, int id, const int32_t *dr
     p.result = result;
     p.ws_status = ws_status;
     return p;
+}
+
+static tb_status check_typical(const tb_typical *t, const char *fn)
+{
+    if (!t)
+        return fail(TB_EINVAL, "%s: typical-acceptance parameters are NULL", fn);
+    if (!(t->temperature > 0.f) || !std::isfinite(t->temperature) || !(t->eps >= 0.f) || !(t->alpha >= 0.f) ||
+        !std::isfinite(t->eps) || !std::isfinite(t->alpha))
+        return fail(TB_EINVAL, "%s: need T > 0 and finite eps, alpha >= 0 (T=%g eps=%g alpha=%g)", fn,
+                    (double)t->temperature, (double)t->eps, (double)t->alpha);
+    return TB_OK;
+}
+
+static void add_typical(AcceptParams &p, const tb_typical *t, const float *logz_t, const float *ent_t,
+                        const float *draft_logit)
+{
+    p.typical = 1;
+    p.inv_t = 1.0f / t->temperature;
+    p.eps = t->eps;
+    p.alpha = t->alpha;
+    p.logz_t = logz_t;
+    p.ent_t = ent_t;
+    p.draft_logit = draft_logit;
+}
+
+// Workspace arrays of typical mode, indexed by the batch-wide row.
+struct TypRows {
+    float *logz_t, *ent_t, *draft_logit;
+};
+static TypRows typ_rows(uint8_t *ws)
+{
+    float *f = reinterpret_cast<float *>(ws + kTypOff);
+    return TypRows{f, f + kMaxTypRows, f + 2 * kMaxTypRows};
 }
 
 static void add_compaction(AcceptParams &p, const tb_kv *kv)
@@ -677,6 +715,62 @@ extern "C" tb_status greedy_accept(const tb_bank *bank, int bank_id, const int32
     return ok();
 }
 
+extern "C" tb_status lm_head_stats_typical(const tb_bank *bank, int bank_id, const void *hidden, const void *lm_head,
+                                           int d_model, int vocab, float temperature, const int32_t *draft_tokens,
+                                           int32_t *argmax, float *top1, float *entropy, float *logz_t,
+                                           float *entropy_t, float *draft_logit, void *workspace,
+                                           size_t workspace_bytes, tb_stream stream)
+{
+    const char *fn = "lm_head_stats_typical";
+    tb_status st = check_bank(bank, bank_id, fn);
+    if (st != TB_OK)
+        return st;
+    const int N = bank->h_desc[bank_id].n;
+    LmPlan plan;
+    if ((st = lm_validate(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, fn, &plan)) != TB_OK)
+        return st;
+    if (!draft_tokens || !logz_t || !entropy_t || !draft_logit)
+        return fail(TB_EINVAL, "%s: NULL draft_tokens / logz_t / entropy_t / draft_logit", fn);
+    const tb_typical t{temperature, 0.f, 0.f, 0};
+    if ((st = check_typical(&t, fn)) != TB_OK)
+        return st;
+    if ((st = check_ws(workspace, workspace_bytes, kPartBase + plan.ws_bytes, fn)) != TB_OK)
+        return st;
+    LmTypical lt{};
+    lt.temperature = temperature;
+    lt.logz_t = logz_t;
+    lt.ent_t = entropy_t;
+    lt.gather.n_seq = 1;
+    lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, draft_logit, 0, N};
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, static_cast<uint8_t *>(workspace),
+                         kPartBase, (cudaStream_t)stream, fn, 0, &lt)) != TB_OK)
+        return st;
+    return ok();
+}
+
+extern "C" tb_status typical_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens,
+                                    const int32_t *argmax, const float *logz_t, const float *entropy_t,
+                                    const float *draft_logit, int vocab, int L, const tb_typical *params,
+                                    tb_result *result, tb_stream stream)
+{
+    const char *fn = "typical_accept";
+    tb_status st = check_bank(bank, bank_id, fn);
+    if (st != TB_OK)
+        return st;
+    if (!draft_tokens || !argmax || !logz_t || !entropy_t || !draft_logit || !result)
+        return fail(TB_EINVAL, "%s: NULL argument", fn);
+    if ((st = check_typical(params, fn)) != TB_OK)
+        return st;
+    if (vocab < 1 || L < 0)
+        return fail(TB_EINVAL, "%s: vocab=%d L=%d", fn, vocab, L);
+    AcceptParams p = accept_params(bank, bank_id, draft_tokens, argmax, vocab, L, result, nullptr);
+    add_typical(p, params, logz_t, entropy_t, draft_logit);
+    cudaError_t e = accept_launch(p, sm_count(bank->device), (cudaStream_t)stream);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
+}
+
 extern "C" tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream)
 {
     const char *fn = "kv_compact";
@@ -695,13 +789,12 @@ extern "C" tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_str
     return ok();
 }
 
-extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q, int n_q_heads,
-                                 const void *hidden, const void *lm_head, int d_model, int vocab,
-                                 const int32_t *draft_tokens, void *attn_out, int32_t *argmax, float *top1,
-                                 float *entropy, tb_result *result, void *workspace, size_t workspace_bytes, int flags,
-                                 tb_stream stream)
+static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q, int n_q_heads,
+                                  const void *hidden, const void *lm_head, int d_model, int vocab,
+                                  const int32_t *draft_tokens, void *attn_out, int32_t *argmax, float *top1,
+                                  float *entropy, const tb_typical *typ, tb_result *result, void *workspace,
+                                  size_t workspace_bytes, int flags, tb_stream stream, const char *fn)
 {
-    const char *fn = "verify_step";
     AttnArgs a{bank, bank_id, kv, 0, kv ? kv->n_layers : 0, q, n_q_heads, attn_out};
     AttnPlan aplan;
     tb_status st = attn_validate(a, fn, &aplan);
@@ -713,12 +806,23 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
         return st;
     if (!draft_tokens || !result)
         return fail(TB_EINVAL, "%s: draft_tokens / result is NULL", fn);
+    if (typ && (st = check_typical(typ, fn)) != TB_OK)
+        return st;
     const size_t attn_bytes = attn_part_bytes(sm_count(bank->device), kv->head_dim);
     const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
     if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
         return st;
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = (cudaStream_t)stream;
+    const TypRows tr = typ_rows(ws);
+    LmTypical lt{};
+    if (typ) {
+        lt.temperature = typ->temperature;
+        lt.logz_t = tr.logz_t;
+        lt.ent_t = tr.ent_t;
+        lt.gather.n_seq = 1;
+        lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, tr.draft_logit, 0, N};
+    }
     {
         // attention on the caller's stream; the LM head forked onto the bank's
         // helper stream fills the SMs that attention CTAs release; join before acceptance
@@ -731,7 +835,7 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
         if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
             return st;
         if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                             bank->aux, fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0)) != TB_OK)
+                             bank->aux, fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr)) != TB_OK)
             return st;
         e = cudaEventRecord(bank->ev_join, bank->aux);
         if (e == cudaSuccess)
@@ -741,6 +845,8 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
     }
     AcceptParams p =
         accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
+    if (typ)
+        add_typical(p, typ, tr.logz_t, tr.ent_t, tr.draft_logit);
     if (!(flags & TB_NO_COMPACT))
         add_compaction(p, kv);
     cudaError_t e = accept_launch(p, sm_count(bank->device), s);
@@ -749,12 +855,36 @@ extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *
     return ok();
 }
 
-extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
-                                         const void *hidden, const void *lm_head, int d_model, int vocab,
-                                         int32_t *argmax, float *top1, float *entropy, void *workspace,
-                                         size_t workspace_bytes, int flags, tb_stream stream)
+extern "C" tb_status verify_step(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q, int n_q_heads,
+                                 const void *hidden, const void *lm_head, int d_model, int vocab,
+                                 const int32_t *draft_tokens, void *attn_out, int32_t *argmax, float *top1,
+                                 float *entropy, tb_result *result, void *workspace, size_t workspace_bytes, int flags,
+                                 tb_stream stream)
 {
-    const char *fn = "verify_step_batched";
+    return verify_step_impl(bank, bank_id, kv, q, n_q_heads, hidden, lm_head, d_model, vocab, draft_tokens, attn_out,
+                            argmax, top1, entropy, nullptr, result, workspace, workspace_bytes, flags, stream,
+                            "verify_step");
+}
+
+extern "C" tb_status verify_step_typical(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q,
+                                         int n_q_heads, const void *hidden, const void *lm_head, int d_model,
+                                         int vocab, const int32_t *draft_tokens, void *attn_out, int32_t *argmax,
+                                         float *top1, float *entropy, const tb_typical *params, tb_result *result,
+                                         void *workspace, size_t workspace_bytes, int flags, tb_stream stream)
+{
+    const char *fn = "verify_step_typical";
+    if (!params)
+        return fail(TB_EINVAL, "%s: typical-acceptance parameters are NULL", fn);
+    return verify_step_impl(bank, bank_id, kv, q, n_q_heads, hidden, lm_head, d_model, vocab, draft_tokens, attn_out,
+                            argmax, top1, entropy, params, result, workspace, workspace_bytes, flags, stream, fn);
+}
+
+static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                          const void *hidden, const void *lm_head, int d_model, int vocab,
+                                          int32_t *argmax, float *top1, float *entropy, const tb_typical *typ,
+                                          void *workspace, size_t workspace_bytes, int flags, tb_stream stream,
+                                          const char *fn)
+{
     if (!bank)
         return fail(TB_EINVAL, "%s: bank is NULL", fn);
     if (batch < 1 || batch > TB_MAX_BATCH || !seqs)
@@ -784,8 +914,10 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
     for (int b = 0; b < batch; ++b)
         if (Ns[b] * group > 256)
             return fail(TB_EUNSUPPORTED, "%s: sequence %d: N * group = %d > 256", fn, b, Ns[b] * group);
-    if (rows_total > 4 * 256)
-        return fail(TB_EUNSUPPORTED, "%s: %d LM-head rows > 1024", fn, rows_total);
+    if (rows_total > kMaxTypRows)
+        return fail(TB_EUNSUPPORTED, "%s: %d LM-head rows > %d", fn, rows_total, kMaxTypRows);
+    if (typ && (st = check_typical(typ, fn)) != TB_OK)
+        return st;
     LmPlan lplan;
     const int chunk = rows_total < 256 ? rows_total : 256;
     if ((st = lm_validate(hidden, chunk, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
@@ -838,12 +970,30 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
                 return st;
         }
     }
-    // LM head over every row of the batch, in chunks of up to 256 rows
+    // LM head over every row of the batch, in chunks of up to 256 rows; in
+    // typical mode each chunk gathers the draft logits of the edges whose
+    // parent row it holds
+    const TypRows tr = typ_rows(ws);
     const uint8_t *h8 = static_cast<const uint8_t *>(hidden);
     for (int r0 = 0; r0 < rows_total; r0 += 256) {
         const int rc = rows_total - r0 < 256 ? rows_total - r0 : 256;
+        LmTypical lt{};
+        if (typ) {
+            lt.temperature = typ->temperature;
+            lt.logz_t = tr.logz_t + r0;
+            lt.ent_t = tr.ent_t + r0;
+            int sr = 0;
+            for (int b = 0; b < batch; ++b) {
+                if (sr < r0 + rc && sr + Ns[b] > r0)
+                    lt.gather.seq[lt.gather.n_seq++] = LmGatherSeq{bank->d_desc + seqs[b].bank_id,
+                                                                   seqs[b].draft_tokens, tr.draft_logit + sr, sr - r0,
+                                                                   Ns[b]};
+                sr += Ns[b];
+            }
+        }
         if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
-                             entropy + r0, ws, kPartBase + attn_bytes, bank->aux, fn)) != TB_OK)
+                             entropy + r0, ws, kPartBase + attn_bytes, bank->aux, fn, 0, typ ? &lt : nullptr)) !=
+            TB_OK)
             return st;
     }
     e = cudaEventRecord(bank->ev_join, bank->aux);
@@ -857,6 +1007,8 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
     for (int b = 0; b < batch; ++b) {
         ps[b] = accept_params(bank, seqs[b].bank_id, seqs[b].draft_tokens, argmax + r0, vocab, seqs[b].kv.L,
                               seqs[b].result, reinterpret_cast<const int *>(ws));
+        if (typ)
+            add_typical(ps[b], typ, tr.logz_t + r0, tr.ent_t + r0, tr.draft_logit + r0);
         if (!(flags & TB_NO_COMPACT))
             add_compaction(ps[b], &seqs[b].kv);
         r0 += Ns[b];
@@ -865,6 +1017,29 @@ extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const t
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
+}
+
+extern "C" tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                         const void *hidden, const void *lm_head, int d_model, int vocab,
+                                         int32_t *argmax, float *top1, float *entropy, void *workspace,
+                                         size_t workspace_bytes, int flags, tb_stream stream)
+{
+    return verify_step_batched_impl(bank, batch, seqs, n_q_heads, hidden, lm_head, d_model, vocab, argmax, top1,
+                                    entropy, nullptr, workspace, workspace_bytes, flags, stream,
+                                    "verify_step_batched");
+}
+
+extern "C" tb_status verify_step_batched_typical(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
+                                                 const void *hidden, const void *lm_head, int d_model, int vocab,
+                                                 int32_t *argmax, float *top1, float *entropy,
+                                                 const tb_typical *params, void *workspace, size_t workspace_bytes,
+                                                 int flags, tb_stream stream)
+{
+    const char *fn = "verify_step_batched_typical";
+    if (!params)
+        return fail(TB_EINVAL, "%s: typical-acceptance parameters are NULL", fn);
+    return verify_step_batched_impl(bank, batch, seqs, n_q_heads, hidden, lm_head, d_model, vocab, argmax, top1,
+                                    entropy, params, workspace, workspace_bytes, flags, stream, fn);
 }
 
 // ------------------------------------------------------------------ per-step tree selection

@@ -30,15 +30,18 @@ def bits(t) -> np.ndarray:
     return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
 
-def gap_filtered_hidden(seed: int, n: int, W):
-    """n hidden rows whose oracle top-2 logit gap exceeds GAP_MIN, with their oracle stats."""
+def gap_filtered_hidden(seed: int, n: int, W, want_logits: bool = False):
+    """n hidden rows whose oracle top-2 logit gap exceeds GAP_MIN, with their oracle
+    stats (and their fp64 logits when want_logits)."""
     D = W.shape[1]
     for attempt in range(8):
         pool = synth.gen_hidden_pool(seed + 1000 * attempt, n + max(8, n // 2), D)
-        am, t1, en, gap = oracle.lm_head(pool, W)
+        out = oracle.lm_head(pool, W, want_logits=want_logits)
+        am, t1, en, gap = out[:4]
         keep = np.nonzero(gap > GAP_MIN)[0][:n]
         if len(keep) == n:
-            return pool[keep], am[keep], t1[keep], en[keep]
+            rows = (pool[keep], am[keep], t1[keep], en[keep])
+            return rows + (out[4][keep],) if want_logits else rows
     raise RuntimeError("could not draw hidden rows with a clear top-2 gap")
 
 
@@ -81,3 +84,56 @@ def check_attention(got: np.ndarray, ref: np.ndarray, what: str = "attention"):
     assert err.max() <= ATT_MAX, f"{what}: max |err| {err.max():.3e} > {ATT_MAX}"
     assert err.mean() <= ATT_MEAN, f"{what}: mean |err| {err.mean():.3e} > {ATT_MEAN}"
     return float(err.max()), float(err.mean())
+
+
+# typical acceptance: the paper's settings (temperature, posterior threshold, mixing coefficient)
+TYPICAL = (0.7, 0.09, 0.3)
+MARGIN_MIN = 1e-3  # |p - threshold| / threshold of every edge, so fp32 and fp64 decide alike
+LL_GAP_MIN = 1e-3  # path log-likelihood gap between the best deepest accepted node and any other
+LOGIT_TOL = 1e-3   # gathered draft logits and tempered log-partitions: abs
+
+
+def typical_ambiguity(parent, drafts, logits, T, eps, alpha):
+    """Edges whose decision sits within MARGIN_MIN of the threshold, and whether the
+    choice among the deepest accepted nodes is within LL_GAP_MIN (different tokens)."""
+    k, path, bonus, det = oracle.typical_accept(parent, drafts, logits, T, eps, alpha, detail=True)
+    close = [j for j in range(1, len(parent)) if abs(det["margin"][j]) < MARGIN_MIN]
+    depth = synth.depth_of(parent)
+    cand = [i for i in range(len(parent)) if det["accepted"][i] and depth[i] == k - 1]
+    lls = sorted((det["loglik"][i] for i in cand), reverse=True)
+    tie = len(lls) > 1 and 0 < lls[0] - lls[1] < LL_GAP_MIN
+    return close, tie
+
+
+def typical_drafts(seed: int, parent, logits, T, eps, alpha, p_likely: float = 0.7):
+    """Draft tokens whose typical-acceptance decisions are all clear of the threshold.
+
+    Each non-root node proposes, with probability p_likely, a token drawn from its
+    parent's tempered target distribution (what a trained head tends to propose),
+    else a uniform token.  Tokens whose edge margin is within MARGIN_MIN are redrawn;
+    a near-tie between equally deep accepted paths redraws everything."""
+    parent = np.asarray(parent)
+    n, V = logits.shape
+    w = np.exp((logits - logits.max(axis=1, keepdims=True)) / T)
+    w /= w.sum(axis=1, keepdims=True)
+    for attempt in range(20):
+        g = synth.rng(seed + 7919 * attempt, 9)
+        drafts = np.zeros(n, dtype=np.int32)
+
+        def draw(j):
+            if g.random() < p_likely:
+                return int(g.choice(V, p=w[parent[j]]))
+            return int(g.integers(0, V))
+
+        for j in range(1, n):
+            drafts[j] = draw(j)
+        for _ in range(20):
+            close, tie = typical_ambiguity(parent, drafts, logits, T, eps, alpha)
+            if not close:
+                break
+            for j in close:
+                drafts[j] = draw(j)
+        close, tie = typical_ambiguity(parent, drafts, logits, T, eps, alpha)
+        if not close and not tie:
+            return drafts
+    raise RuntimeError("could not draw unambiguous drafts")

@@ -14,6 +14,7 @@ from fractions import Fraction
 import networkx as nx
 import numpy as np
 import pytest
+import scipy.special
 import torch
 
 import oracle
@@ -232,3 +233,45 @@ def test_matches_brute_force(seed):
     if np.abs(det["margin"][1:]).min() < 1e-9:
         pytest.skip("an edge sits on the threshold")
     assert (k, path, bonus) == _brute_force(parent, draft, z, T, EPS, ALPHA)
+
+
+# ---------------------------------------------------------------- tempered statistics
+
+def test_tempered_stats_closed_form():
+    base = np.log([0.5, 0.25, 0.125, 0.125])
+    logz, ent = oracle.tempered_stats(base[None], 0.5)
+    # sum_v e^(2 ln p_v) = sum p_v^2 = 22/64; entropy of (16, 4, 1, 1)/22
+    q = np.array([16, 4, 1, 1]) / 22
+    assert logz[0] == pytest.approx(math.log(22 / 64), rel=1e-14)
+    assert ent[0] == pytest.approx(-(q * np.log(q)).sum(), rel=1e-14)
+    logz, ent = oracle.tempered_stats(base[None], 1.0)
+    assert logz[0] == pytest.approx(0.0, abs=1e-15)
+    assert ent[0] == pytest.approx(1.75 * math.log(2), rel=1e-14)
+    logz, ent = oracle.tempered_stats(np.full((1, 1000), 3.0), 0.7)
+    assert logz[0] == pytest.approx(3.0 / 0.7 + math.log(1000), rel=1e-14)
+    assert ent[0] == pytest.approx(math.log(1000), rel=1e-14)
+
+
+@pytest.mark.parametrize("T_", [0.3, 0.7, 1.0, 2.0])
+def test_tempered_stats_match_libraries(T_):
+    # against scipy's logsumexp and torch's Categorical entropy; at T = 1 the
+    # entropy also equals the (separately pinned) LM-head entropy
+    g = synth.rng(400)
+    z = g.standard_normal((9, 777)) * 2.5
+    logz, ent = oracle.tempered_stats(z, T_)
+    np.testing.assert_allclose(logz, scipy.special.logsumexp(z / T_, axis=1), rtol=1e-12)
+    cat = torch.distributions.Categorical(logits=torch.from_numpy(z) / T_)
+    np.testing.assert_allclose(ent, cat.entropy().numpy(), rtol=1e-11, atol=1e-12)
+    # logits and temperature scaled together: unchanged
+    logz2, ent2 = oracle.tempered_stats(z * 3.0, T_ * 3.0)
+    np.testing.assert_allclose(logz2, logz, rtol=1e-12)
+    np.testing.assert_allclose(ent2, ent, rtol=1e-12)
+
+
+def test_tempered_entropy_at_one_equals_lm_head_entropy():
+    g = synth.rng(401)
+    W = synth.normal_bf16(g, (300, 64), 0.3)
+    h = synth.normal_bf16(g, (5, 64))
+    _, _, ent1, _, logits = oracle.lm_head(h, W, want_logits=True)
+    _, ent = oracle.tempered_stats(logits, 1.0)
+    np.testing.assert_allclose(ent, ent1, rtol=1e-12)
