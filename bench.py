@@ -531,6 +531,118 @@ def run_gpu_bank_loop(args):
     print(json.dumps(line), flush=True)
 
 
+def expected_accept_len(parent, p_match: float) -> float:
+    """E[accept_len] when every edge matches independently with probability
+    p_match (the synthetic draft model: a node copies its parent's greedy token
+    with probability p_match).  With f_u(k) = P(the deepest fully matched path
+    below an accepted node u is >= k edges long), f_u(0) = 1 and
+    f_u(k) = 1 - prod over children c of (1 - p f_c(k - 1)); then
+    E[accept_len] = 1 + sum_{k >= 1} f_root(k)."""
+    parent = list(parent)
+    n = len(parent)
+    kids = [[] for _ in range(n)]
+    for i in range(1, n):
+        kids[parent[i]].append(i)
+    depth_max = int(synth.depth_of(parent).max())
+    f = [[1.0] + [0.0] * depth_max for _ in range(n)]
+    for u in range(n - 1, -1, -1):  # parent[i] < i: children before parents
+        for k in range(1, depth_max + 1):
+            miss = 1.0
+            for c in kids[u]:
+                miss *= 1.0 - p_match * f[c][k - 1]
+            f[u][k] = 1.0 - miss
+    return 1.0 + sum(f[0][1:])
+
+
+def run_gpu_sweep(args):
+    """Verify cost against tree size over the 8-tree bank (the kernel-side
+    counterpart of the paper's throughput frontier, Sec. 3.2): for each tree,
+    the device time of one verify_step at the 7B single-layer shape (L=2048)
+    and at the long-context shape (32 layers, L=16384), with the expected
+    accept length of the synthetic draft model at several match rates and the
+    resulting accepted tokens per second."""
+    import torch
+
+    import paper_2606_27550_gb300 as tv
+    from paper_2606_27550_gb300 import build as tvbuild
+
+    world, rank, local = dist_info()
+    tvbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device(f"cuda:{local}")
+    bf = torch.bfloat16
+    trees = synth.bank_trees()
+    bank = tv.Bank(16, local)
+    ids = [bank.add(t)[0] for t in trees]
+    ps = (0.5, 0.6, 0.7, 0.8, 0.9)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    rows = []
+    shapes = {"7b-1layer-L2048": (1, 2048), "7b-32layer-L16384": (32, 16384)}
+    for sname, (nl, L) in shapes.items():
+        H, d, D, V = 32, 128, 4096, 32000
+        seed = 99 + nl
+        k = synth.device_normal_bf16_(torch.empty((nl, H, L + 64, d), dtype=bf, device=dev), seed)
+        v = synth.device_normal_bf16_(torch.empty((nl, H, L + 64, d), dtype=bf, device=dev), seed + 1)
+        W = synth.device_normal_bf16_(torch.empty((V, D), dtype=bf, device=dev), seed + 2, std=0.02)
+        q = synth.device_normal_bf16_(torch.empty((nl, 64, H, d), dtype=bf, device=dev), seed + 3)
+        hid = synth.device_normal_bf16_(torch.empty((64, D), dtype=bf, device=dev), seed + 4)
+        am = torch.empty(64, dtype=torch.int32, device=dev)
+        t1 = torch.empty(64, dtype=torch.float32, device=dev)
+        en = torch.empty(64, dtype=torch.float32, device=dev)
+        ws = tv.make_workspace(tv.tb_workspace_size(64, nl, H, H, d, V, local), dev)
+        res = tv.make_result(dev)
+        drafts = torch.zeros(64, dtype=torch.int32, device=dev)
+        for j, t in enumerate(trees):
+            n = len(t)
+            qn = q[:, :n].contiguous()
+            out = torch.empty((nl, n, H, d), dtype=bf, device=dev)
+            kv = tv.KvCache(k, v, L)
+            n_steps = max(10, min(args.steps, 100))
+            for _ in range(args.warmup):
+                tv.verify_step(bank, ids[j], kv, qn, hid[:n], W, drafts[:n], out, am[:n], t1[:n], en[:n], res, ws,
+                               tv.TB_NO_COMPACT, stream)
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(n_steps)]
+            for i in range(n_steps):
+                flush.zero_()
+                ev[i][0].record(stream)
+                tv.verify_step(bank, ids[j], kv, qn, hid[:n], W, drafts[:n], out, am[:n], t1[:n], en[:n], res, ws,
+                               tv.TB_NO_COMPACT, stream)
+                ev[i][1].record(stream)
+            torch.cuda.synchronize()
+            ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+            taus = {str(pm): round(expected_accept_len(t, pm), 4) for pm in ps}
+            rows.append({"shape": sname, "tree_nodes": n, "tree_depth": int(synth.depth_of(t).max()),
+                         "ms_per_step": round(ms, 4),
+                         "accepted_tokens_per_s": {pm: round(tau / (ms * 1e-3), 1) for pm, tau in taus.items()},
+                         "expected_accept_len": taus})
+        del k, v, W, q, hid, ws
+        torch.cuda.empty_cache()
+    bank.close()
+    if rank != 0:
+        return
+    best = {}
+    for sname in shapes:
+        for pm in ps:
+            cand = [r for r in rows if r["shape"] == sname]
+            top = max(cand, key=lambda r: r["accepted_tokens_per_s"][str(pm)])
+            best[f"{sname} p={pm}"] = top["tree_nodes"]
+    c4_64 = [r for r in rows if r["shape"] == "7b-32layer-L16384" and r["tree_nodes"] == 64][0]
+    line = {
+        "metric": "verify-steps/s", "value": round(1e3 / c4_64["ms_per_step"], 3), "unit": "verify-steps/s",
+        "n_gpus": 1, "steps": max(10, min(args.steps, 100)), "warmup": args.warmup,
+        "ms_per_step": c4_64["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded); accept lengths from the independent-match draft model",
+        "config": {"workload": "bank sweep: 8 trees x {7B 1 layer L=2048, 7B 32 layers L=16384}",
+                   "l2": "256 MB flush before every timed step"},
+        "sweep": rows,
+        "throughput_optimal_tree": best,
+        "gpu_launches": 4 * max(10, min(args.steps, 100)) * len(rows),
+    }
+    print(json.dumps(line), flush=True)
+
+
 # ----------------------------------------------------------------------------- CPU oracle (reference arm)
 
 
@@ -626,7 +738,7 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--config", default="c4", choices=["c1", "c2", "c3", "c4", "c5", "sweep"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
@@ -634,8 +746,10 @@ def main(argv=None):
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
                     help="verification rule: greedy (default) or typical acceptance at T=0.7, eps=0.09, alpha=0.3")
     args = ap.parse_args(argv)
-    if args.accept == "typical" and (args.impl == "reference" or args.config == "c3"):
+    if args.accept == "typical" and (args.impl == "reference" or args.config in ("c3", "sweep")):
         ap.error("--accept typical applies to the GPU arm of c1, c2, c4 and c5")
+    if args.impl == "reference" and args.config == "sweep":
+        ap.error("the sweep has no reference arm")
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
@@ -644,6 +758,8 @@ def main(argv=None):
         run_gpu_batched(args)
     elif args.config == "c3":
         run_gpu_bank_loop(args)
+    elif args.config == "sweep":
+        run_gpu_sweep(args)
     else:
         run_gpu(args)
 
