@@ -498,6 +498,9 @@ def run_gpu_bank_loop(args):
             L = int(res_h[2])
         return L, kix, toks, kv_b, accepted, hist
 
+    if args.scheduled:
+        return bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs, drafts, am, t1, en, res,
+                                   ws, trace, steps, L0, sh, rank, world)
     L, kix, *_ = loop(0, args.warmup, L0, 0)
     sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]
                            if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
@@ -527,6 +530,81 @@ def run_gpu_bank_loop(args):
                          "peak_src": peak_src},
         "gpu_launches": 4 * steps,
         "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs, drafts, am, t1, en, res, ws, trace,
+                        steps, L0, sh, rank, world):
+    """The bank-switching loop driven from the device (verify_step_scheduled):
+    the tree and the prefix length of each step live in device memory and the
+    acceptance kernel takes the ladder decision (trace feature, up below 1.5,
+    down above 2.5), so G steps are captured into one CUDA graph and replayed
+    with no host read between steps."""
+    bf = torch.bfloat16
+    H, d = sh.n_q_heads, sh.head_dim
+    n_max = 64
+    pool = qs.shape[0]
+    G = 48  # steps per graph (a multiple of the input pool)
+    tab = []
+    for i in range(pool):
+        t_ = torch.zeros((len(trees), n_max), dtype=torch.int32, device=dev)
+        for j, t in enumerate(trees):
+            t_[j, :len(t)] = drafts[(i, j)]
+        tab.append(t_)
+    trace_d = torch.from_numpy(np.asarray(trace, dtype=np.float32)).to(dev)
+    pol = tv.make_policy(tv.TB_POLICY_HYSTERETIC_LADDER, tv.TB_FEATURE_TRACE, ids, a=1.5, b=2.5, trace=trace_d,
+                         node_stride=n_max)
+    state = tv.make_state(0, L0, dev)
+    out = torch.empty((1, n_max, H, d), dtype=bf, device=dev)
+    kv = tv.KvCache(k, v, 0)
+
+    def sstep(t, s):
+        i = t % pool
+        tv.verify_step_scheduled(bank, pol, state, kv, qs[i], hs[i], W, tab[i], out, am, t1, en, res, ws, 0, s)
+
+    stream = torch.cuda.current_stream()
+    for t in range(max(args.warmup, 3)):
+        sstep(t, stream)
+    torch.cuda.synchronize()
+    cs = torch.cuda.Stream()
+    cs.wait_stream(stream)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cs):
+        for t in range(G):
+            sstep(t, cs)
+    n_rep = (steps + G - 1) // G
+    state.copy_(tv.make_state(0, L0, dev))
+    torch.cuda.synchronize()
+    sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(dev.index)).split(",")[dev.index]
+                           if os.environ.get("CUDA_VISIBLE_DEVICES") else str(dev.index))
+    sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n_rep):
+        g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    el = e0.elapsed_time(e1) / 1e3
+    clocks = sampler.stop()
+    st = tv.parse_state(state)
+    bank.close()
+    if rank != 0:
+        return
+    done = n_rep * G
+    peaks, peak_src = load_peaks()
+    line = {
+        "metric": "verify-steps/s", "value": round(done / el, 3), "unit": "verify-steps/s", "n_gpus": world,
+        "steps": done, "warmup": max(args.warmup, 3), "ms_per_step": round(el / done * 1e3, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded), AR(1) entropy trace",
+        "config": {"workload": sh.name + "-device-driven", "bank_sizes": [len(t) for t in trees], "L_start": L0,
+                   "L_end": st["L"], "policy": "hysteretic step ladder on the device: up below 1.5, down above 2.5",
+                   "host_read_per_step": False, "cuda_graph_steps": G},
+        "tau_mean_accept_len": round((st["L"] - L0) / done, 4),
+        "gpu_launches": 4 * done,
+        "clocks": clocks,
+        "hbm_roofline": {"peak_gbs": float(peaks["hbm_gbs"]), "peak_src": peak_src},
     }
     print(json.dumps(line), flush=True)
 
@@ -743,11 +821,15 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--scheduled", action="store_true",
+                    help="c3 only: the device-driven loop (tree and L on the device, CUDA-graph replay)")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
                     help="verification rule: greedy (default) or typical acceptance at T=0.7, eps=0.09, alpha=0.3")
     args = ap.parse_args(argv)
     if args.accept == "typical" and (args.impl == "reference" or args.config in ("c3", "sweep")):
         ap.error("--accept typical applies to the GPU arm of c1, c2, c4 and c5")
+    if args.scheduled and (args.config != "c3" or args.impl == "reference"):
+        ap.error("--scheduled applies to the GPU arm of c3")
     if args.impl == "reference" and args.config == "sweep":
         ap.error("the sweep has no reference arm")
     if args.warmup < 3:

@@ -348,6 +348,72 @@ TB_API tb_status verify_step_batched_typical(const tb_bank *bank, int batch, con
                                              int32_t *argmax, float *top1, float *entropy, const tb_typical *params,
                                              void *workspace, size_t workspace_bytes, int flags, tb_stream stream);
 
+/* ------------------------------------------------------------------------
+ * Device-driven decode loop: the per-step tree selection of Sec. 4 ("Policy",
+ * "Cost") taken on the GPU.  The prefix length and the tree of the next step
+ * live in device memory (tb_state); the acceptance kernel's last CTA updates
+ * them after each step, so consecutive verify_step_scheduled calls need no
+ * host read in between and a sequence of them can be captured into one CUDA
+ * graph.  head_dim 128 only.
+ * ---------------------------------------------------------------------- */
+
+/* Device-resident state (caller-allocated device memory, 4-byte aligned). */
+typedef struct tb_state {
+    int32_t rung;        /* index into tb_policy.bank_ids of the tree the next step verifies */
+    int32_t L;           /* prefix length of the next step */
+    int32_t step;        /* steps completed */
+    float feature;       /* feature value of the last policy decision */
+    int32_t accept_len;  /* accepted length of the last step */
+    int32_t reserved[3];
+} tb_state;
+
+#define TB_POLICY_HYSTERETIC_LADDER 0 /* one rung up when feature < a, one down when feature > b */
+#define TB_POLICY_BINARY 1            /* rung 1 when feature > a (tau_on), rung 0 when feature <= b (tau_off) */
+#define TB_POLICY_THRESHOLD_LADDER 2  /* rung = number of edges[0..n_rungs-2] that are <= feature */
+
+#define TB_FEATURE_TRACE 0      /* feature = trace[min(step, n_trace - 1)] (a per-step feature series) */
+#define TB_FEATURE_PATH_VALUE 1 /* s = max(p0, g_1 .. g_D), g_d = p0 * prod_{i <= d} p_i: p0 = top1 of the last accepted
+                                   node, p_i = trace[min(step, n_trace - 1) * n_heads + i - 1] (Sec. 4 "Path-value score") */
+#define TB_FEATURE_ENTROPY 2    /* feature = entropy of the last accepted node (nats, temperature 1) */
+
+/* Policy of the device-driven loop (host struct, read at call time). */
+typedef struct tb_policy {
+    int32_t kind;          /* TB_POLICY_* */
+    int32_t feature;       /* TB_FEATURE_* */
+    int32_t n_rungs;       /* 1..8 (TB_POLICY_BINARY: 2) */
+    int32_t bank_ids[8];   /* the tree of each rung, smallest first */
+    float a, b;            /* ladder: up_below, down_above; binary: tau_on, tau_off (b <= a) */
+    float edges[7];        /* threshold ladder: n_rungs - 1 ascending edges */
+    const float *trace;    /* device array for TB_FEATURE_TRACE / TB_FEATURE_PATH_VALUE, else NULL */
+    int32_t n_trace;       /* entries (rows of n_heads for TB_FEATURE_PATH_VALUE), >= 1 when trace is used */
+    int32_t n_heads;       /* head probabilities per row (TB_FEATURE_PATH_VALUE), 0..8 */
+    int32_t node_stride;   /* nodes per layer / per draft row of the per-node arrays; 0: the largest tree of the
+                              policy; otherwise at least that */
+} tb_policy;
+
+/* One verification step whose tree and prefix length come from *state:
+ * tree = policy->bank_ids[state->rung], L = state->L (kv->L is ignored).
+ * N_max is policy->node_stride (0: the largest node count among the policy's
+ * trees); per-node arrays are laid out for N_max nodes and the step uses the
+ * first N of them:
+ *   q, attn_out   bf16 [kv->n_layers][N_max][n_q_heads][128]
+ *   hidden        bf16 [N_max][d_model]
+ *   draft_tokens  int32 [n_rungs][N_max]: row r holds the drafts of rung r's tree
+ *   argmax/top1/entropy [N_max] (rows >= N are scratch)
+ * After tree_attention, the LM head and greedy acceptance (+ compaction unless
+ * TB_NO_COMPACT), the last CTA of the acceptance kernel evaluates the feature
+ * and the policy and writes the next rung, L + accept_len, step + 1, the
+ * feature and accept_len into *state; *result is written as by verify_step.
+ * A state whose L + N exceeds kv->L_cap, or whose rung is out of range, makes
+ * the step report TB_ECAPACITY / TB_EINVAL in result->status and leaves
+ * *state unchanged. */
+TB_API tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy *policy, tb_state *state,
+                                       const tb_kv *kv, const void *q, int n_q_heads, const void *hidden,
+                                       const void *lm_head, int d_model, int vocab, const int32_t *draft_tokens,
+                                       void *attn_out, int32_t *argmax, float *top1, float *entropy,
+                                       tb_result *result, void *workspace, size_t workspace_bytes, int flags,
+                                       tb_stream stream);
+
 /* Message for the last failing call on this thread ("" if none). */
 TB_API const char *tb_last_error(void);
 

@@ -184,3 +184,42 @@ def tempered_stats(logits, temperature: float):
     if _load().oracle_tempered_stats(_ptr(logits), R, V, temperature, _ptr(logz), _ptr(ent)) != 0:
         raise ValueError("bad shape or temperature")
     return logz, ent
+
+
+# ---------------------------------------------------------------- per-step tree selection (Sec. 4)
+
+def path_value(p0: float, head_probs) -> float:
+    """Path-value score (Sec. 4): g_d = p0 * p_1 * ... * p_d and
+    s = max(p0, g_1, ..., g_D).  Evaluated in float64."""
+    s = g = float(p0)
+    for p in head_probs:
+        g *= float(p)
+        s = max(s, g)
+    return s
+
+
+def policy_next(kind: str, rung: int, n_rungs: int, feature: float, a: float = 0.0, b: float = 0.0, edges=()):
+    """Next rung of the per-step policies (Sec. 4 "Policy"):
+      'ladder'    hysteretic step ladder: one rung up when feature < a, one down
+                  when feature > b, else stay (clamped to the rungs);
+      'binary'    rung 1 (aggressive tree) when feature > a = tau_on, rung 0 when
+                  feature <= b = tau_off, else unchanged;
+      'threshold' threshold_ladder: the number of edges that are <= feature."""
+    if kind == "ladder":
+        if feature < a:
+            return min(rung + 1, n_rungs - 1)
+        if feature > b:
+            return max(rung - 1, 0)
+        return rung
+    if kind == "binary":
+        if feature > a:
+            return 1
+        if feature <= b:
+            return 0
+        return rung
+    if kind == "threshold":
+        k = 0
+        while k < n_rungs - 1 and feature >= edges[k]:
+            k += 1
+        return k
+    raise ValueError(kind)

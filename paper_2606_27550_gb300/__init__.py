@@ -31,7 +31,8 @@ API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
        "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error",
        "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
-       "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical")
+       "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical",
+       "verify_step_scheduled")
 
 
 class TreeVerifyError(RuntimeError):
@@ -54,6 +55,18 @@ class TbSeq(ctypes.Structure):
 class TbTypical(ctypes.Structure):
     _fields_ = [("temperature", ctypes.c_float), ("eps", ctypes.c_float), ("alpha", ctypes.c_float),
                 ("reserved", ctypes.c_int32)]
+
+
+TB_POLICY_HYSTERETIC_LADDER, TB_POLICY_BINARY, TB_POLICY_THRESHOLD_LADDER = 0, 1, 2
+TB_FEATURE_TRACE, TB_FEATURE_PATH_VALUE, TB_FEATURE_ENTROPY = 0, 1, 2
+STATE_INTS = 8  # sizeof(tb_state) / 4
+
+
+class TbPolicy(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("feature", ctypes.c_int32), ("n_rungs", ctypes.c_int32),
+                ("bank_ids", ctypes.c_int32 * 8), ("a", ctypes.c_float), ("b", ctypes.c_float),
+                ("edges", ctypes.c_float * 7), ("trace", ctypes.c_void_p), ("n_trace", ctypes.c_int32),
+                ("n_heads", ctypes.c_int32), ("node_stride", ctypes.c_int32)]
 
 
 # the paper's verification settings (temperature, posterior threshold, mixing coefficient)
@@ -94,6 +107,7 @@ def load(path: str = LIB_PATH):
         "typical_accept": [P, i32, P, P, P, P, P, i32, i32, P, P, P],
         "verify_step_typical": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, P, sz, i32, P],
         "verify_step_batched_typical": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, P, sz, i32, P],
+        "verify_step_scheduled": [P, P, P, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -359,6 +373,55 @@ def verify_step_batched_typical(bank: Bank, seqs, hidden, lm_head, argmax, top1,
                                               _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(argmax),
                                               _ptr(top1), _ptr(entropy), ctypes.byref(t), _ptr(ws), ws.numel(),
                                               flags, _stream(stream)), "verify_step_batched_typical")
+
+
+# --------------------------------------------------------------------- device-driven loop
+
+
+def make_policy(kind: int, feature: int, bank_ids, a: float = 0.0, b: float = 0.0, edges=(), trace=None,
+                n_heads: int = 0, node_stride: int = 0) -> TbPolicy:
+    """tb_policy; `trace` is a device float tensor (kept alive by the caller)."""
+    pol = TbPolicy()
+    pol.kind, pol.feature, pol.n_rungs = kind, feature, len(bank_ids)
+    for i, x in enumerate(bank_ids):
+        pol.bank_ids[i] = int(x)
+    pol.a, pol.b = float(a), float(b)
+    for i, x in enumerate(edges):
+        pol.edges[i] = float(x)
+    if trace is not None:
+        pol.trace = _ptr(trace)
+        pol.n_trace = trace.numel() // max(1, n_heads) if feature == TB_FEATURE_PATH_VALUE else trace.numel()
+    pol.n_heads = n_heads
+    pol.node_stride = node_stride
+    return pol
+
+
+def make_state(rung: int, L: int, device="cuda"):
+    """A device tb_state (int32 words) at the given rung and prefix length."""
+    import torch
+
+    t = torch.zeros(STATE_INTS, dtype=torch.int32)
+    t[0], t[1] = rung, L
+    return t.to(device)
+
+
+def parse_state(st) -> dict:
+    import numpy as np
+
+    h = st.cpu().numpy()
+    return {"rung": int(h[0]), "L": int(h[1]), "step": int(h[2]), "feature": float(h[3:4].view(np.float32)[0]),
+            "accept_len": int(h[4])}
+
+
+def verify_step_scheduled(bank: Bank, policy: TbPolicy, state, kv: KvCache, q, hidden, lm_head, drafts, attn_out,
+                          argmax, top1, entropy, result, ws, flags: int = 0, stream=None):
+    """q / attn_out [n_layers][N_max][Hq][128]; hidden [N_max][d_model]; drafts [n_rungs][N_max]."""
+    c = kv.as_c()
+    _check(load().verify_step_scheduled(bank.handle, ctypes.byref(policy), _ptr(state), ctypes.byref(c), _ptr(q),
+                                        q.shape[2], _ptr(hidden), _ptr(lm_head), hidden.shape[1], lm_head.shape[0],
+                                        _ptr(drafts), _ptr(attn_out), _ptr(argmax), _ptr(top1), _ptr(entropy),
+                                        _ptr(result), _ptr(ws), ws.numel(), flags, _stream(stream)),
+           "verify_step_scheduled")
 
 
 # --------------------------------------------------------------------- per-step tree selection

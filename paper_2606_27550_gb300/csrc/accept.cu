@@ -48,6 +48,49 @@ struct AcceptBatch {
     AcceptParams seq[TB_MAX_BATCH];
 };
 
+// Per-step tree selection on the device (Sec. 4, "Path-value score" and
+// "Policy"): the feature of the step just verified, then the next rung.
+// Writes the state words rung, L, step, feature (bits), accept_len.
+__device__ void policy_step(const AcceptParams &p, int rung, int L, int len, int jstar)
+{
+    const int step = p.sched[2];
+    const int row = p.n_trace > 0 ? min(step, p.n_trace - 1) : 0;
+    float f = 0.f;
+    if (p.pol_feature == TB_FEATURE_TRACE) {
+        f = p.trace[row];
+    } else if (p.pol_feature == TB_FEATURE_PATH_VALUE) {
+        // s = max(p0, g_1 .. g_D), g_d = p0 * p_1 * ... * p_d
+        const float p0 = p.top1[jstar];
+        float g = p0, sv = p0;
+        for (int i = 0; i < p.n_heads; ++i) {
+            g *= p.trace[(size_t)row * p.n_heads + i];
+            sv = fmaxf(sv, g);
+        }
+        f = sv;
+    } else {
+        f = p.entropy[jstar];
+    }
+    const int nr = p.n_rungs;
+    int next = rung;
+    if (p.pol_kind == TB_POLICY_HYSTERETIC_LADDER) {
+        if (f < p.pol_a)
+            next = min(rung + 1, nr - 1);
+        else if (f > p.pol_b)
+            next = max(rung - 1, 0);
+    } else if (p.pol_kind == TB_POLICY_BINARY) {
+        next = f > p.pol_a ? 1 : (f <= p.pol_b ? 0 : (rung == 1 ? 1 : 0));
+    } else {
+        next = 0;
+        while (next < nr - 1 && f >= p.pol_edges[next])
+            ++next;
+    }
+    p.sched[0] = next;
+    p.sched[1] = L + len;
+    p.sched[2] = step + 1;
+    p.sched[3] = __float_as_int(f);
+    p.sched[4] = len;
+}
+
 // blockIdx.y selects the sequence; every CTA of a sequence recomputes its acceptance.
 __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__ AcceptBatch pb)
 {
@@ -55,7 +98,32 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
     __shared__ int s_path[kMaxNodes];
     __shared__ float s_lp[kMaxNodes];
     __shared__ int s_len;
+    __shared__ int s_rung, s_L, s_err;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    const TreeDesc *tree = p.tree;
+    const int32_t *draft = p.draft;
+    int L = p.L;
+    if (p.sched) {
+        if (threadIdx.x == 0) {
+            int rung = p.sched[0];
+            const int Ls = p.sched[1];
+            int err = TB_OK;
+            if (rung < 0 || rung >= p.n_rungs) {
+                err = TB_EINVAL;
+                rung = 0;
+            } else if (Ls < 0 || Ls + p.rung_tree[rung]->n > p.L_cap) {
+                err = TB_ECAPACITY;
+            }
+            s_rung = rung;
+            s_L = err == TB_OK ? Ls : 0;
+            s_err = err;
+        }
+        __syncthreads();
+        tree = p.rung_tree[s_rung];
+        draft = p.draft + (size_t)s_rung * p.n_max;
+        L = s_L;
+    }
 
     if (p.from_result) {
         if (threadIdx.x < kMaxNodes)
@@ -65,7 +133,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
         __syncthreads();
     } else {
         if (warp == 0) {
-            const TreeDesc *t = p.tree;
+            const TreeDesc *t = tree;
             const int n = t->n;
             uint64_t match = 0;
             bool bad = false;
@@ -74,7 +142,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                 const int i = lane + 32 * h;
                 bool m = false;
                 if (i >= 1 && i < n) {
-                    const int tok = p.draft[i];
+                    const int tok = draft[i];
                     const bool bad_tok = (tok < 0 || tok >= p.vocab);
                     bad |= bad_tok;
                     if (!p.typical) {
@@ -174,13 +242,15 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                     tb_result *r = p.result;
                     r->accept_len = len;
                     r->bonus_token = p.argmax[jstar];
-                    r->new_L = p.L + len;
                     int st = TB_OK;
                     const int ws = p.ws_status ? *p.ws_status : 0;
-                    if (ws & kStatusTimeout)
+                    if (p.sched && s_err != TB_OK)
+                        st = s_err;
+                    else if (ws & kStatusTimeout)
                         st = TB_ETIMEOUT;
                     else if (any_bad || (ws & kStatusBadToken))
                         st = TB_EINVAL;
+                    r->new_L = (p.sched && s_err != TB_OK) ? p.sched[1] : L + len;
                     r->status = st;
                 }
             }
@@ -192,20 +262,32 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
         __syncthreads();
     }
 
-    if (p.n_layers == 0)
-        return;
     const int k = s_len;
-    if (k <= 1)
+    const bool compact = p.n_layers > 0 && k > 1 && !(p.sched && s_err != TB_OK);
+    if (compact) {
+        const int units = p.n_layers * p.n_kv_heads * 2;
+        const int warps_per_cta = blockDim.x >> 5;
+        for (int unit = blockIdx.x * warps_per_cta + warp; unit < units; unit += gridDim.x * warps_per_cta) {
+            const int which = unit & 1;
+            const int lh = unit >> 1;
+            const int head = lh % p.n_kv_heads, layer = lh / p.n_kv_heads;
+            uint8_t *base = (which ? p.v : p.k) + layer * p.layer_stride_b + head * p.head_stride_b +
+                            (size_t)L * p.row_bytes;
+            copy_rows(base, s_path, k, p.row_bytes, p.L_cap - L, lane);
+        }
+    }
+    if (!p.sched)
         return;
-    const int units = p.n_layers * p.n_kv_heads * 2;
-    const int warps_per_cta = blockDim.x >> 5;
-    for (int unit = blockIdx.x * warps_per_cta + warp; unit < units; unit += gridDim.x * warps_per_cta) {
-        const int which = unit & 1;
-        const int lh = unit >> 1;
-        const int head = lh % p.n_kv_heads, layer = lh / p.n_kv_heads;
-        uint8_t *base = (which ? p.v : p.k) + layer * p.layer_stride_b + head * p.head_stride_b +
-                        (size_t)p.L * p.row_bytes;
-        copy_rows(base, s_path, k, p.row_bytes, p.L_cap - p.L, lane);
+    // ---------------- scheduled mode: the last CTA to arrive takes the policy step
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const int ticket = atomicAdd(p.ticket, 1);
+        if (ticket == (int)gridDim.x - 1) {
+            *p.ticket = 0;
+            if (s_err == TB_OK)
+                policy_step(p, s_rung, L, k, s_path[k - 1]);
+        }
     }
 }
 

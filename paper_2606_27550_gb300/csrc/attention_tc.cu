@@ -57,10 +57,11 @@ constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by
 // [tile_base, tile_base + n_units * T) of the flattened tile space.
 struct TcSeq {
     long long tile_base;
-    const __nv_bfloat16 *q;  // [n_layers][N][Hq][128]
+    const __nv_bfloat16 *q;  // [n_layers][nstride][Hq][128]
     __nv_bfloat16 *out;      // same layout
     const TreeDesc *tree;
     int L, N, rows, row_blocks, T, unit_base;
+    int nstride;             // nodes per layer in q / out (N, or the largest tree of a scheduled loop)
 };
 
 struct TcParams {
@@ -73,7 +74,34 @@ struct TcParams {
     float *part;
     int *counters;
     int *status;
+    // scheduled mode (sched != null): the tree and the prefix length come from
+    // device memory (sched[0] = rung into rung_tree, sched[1] = L) and every
+    // CTA derives the work split itself; seq[0] carries q, out and nstride
+    const int32_t *sched;
+    const TreeDesc *rung_tree[8];
+    int n_rungs, n_layers, L_cap;
 };
+
+// Scheduled mode: the sequence of this step from the device state.  An
+// out-of-range rung or a prefix that does not fit the cache gives no work
+// (the acceptance kernel reports it).
+__device__ void sched_plan(const TcParams &p, TcSeq *sq, long long *total)
+{
+    *sq = p.seq[0];
+    sq->tile_base = 0;
+    sq->unit_base = 0;
+    const int rung = p.sched[0], L = p.sched[1];
+    const bool ok = rung >= 0 && rung < p.n_rungs && L >= 0;
+    const TreeDesc *tr = p.rung_tree[ok ? rung : 0];
+    const int N = tr->n;
+    sq->tree = tr;
+    sq->L = ok ? L : 0;
+    sq->N = N;
+    sq->rows = N * p.group;
+    sq->row_blocks = (sq->rows + 127) / 128;
+    sq->T = (sq->L + N + kBN - 1) / kBN;
+    *total = (ok && L + N <= p.L_cap) ? (long long)p.n_layers * p.Hkv * sq->row_blocks * sq->T : 0;
+}
 
 // Sequence holding flattened tile t, searching forward from `b` (tiles are
 // visited in increasing order by every role).  kBatched = false: sequence 0.
@@ -89,14 +117,14 @@ __device__ __forceinline__ int seq_at(const TcParams &p, long long t, int b)
     }
 }
 
-__device__ __forceinline__ long long tc_seg_begin(const TcParams &p, int c)
+__device__ __forceinline__ long long tc_seg_begin(long long total, int P, int c)
 {
-    return (long long)c * p.total / p.P;
+    return (long long)c * total / P;
 }
 
-__device__ __forceinline__ int tc_cta_of(const TcParams &p, long long t)
+__device__ __forceinline__ int tc_cta_of(long long total, int P, long long t)
 {
-    return (int)(((t + 1) * (long long)p.P - 1) / p.total);
+    return total > 0 ? (int)(((t + 1) * (long long)P - 1) / total) : 0;
 }
 
 // MN-major (N contiguous) 128-byte-swizzled operand: lbo = stride between
@@ -117,13 +145,24 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
     __shared__ __align__(8) uint64_t q_full, o_free, drain_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
+    __shared__ TcSeq s_seq;
+    __shared__ long long s_total;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sKV = smem;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
-    const long long t0 = tc_seg_begin(p, c), t1 = tc_seg_begin(p, c + 1);
+    const TcSeq *seqs = p.seq;
+    long long total = p.total;
+    if (p.sched) {
+        if (threadIdx.x == 0)
+            sched_plan(p, &s_seq, &s_total);
+        __syncthreads();
+        seqs = &s_seq;
+        total = s_total;
+    }
+    const long long t0 = tc_seg_begin(total, p.P, c), t1 = tc_seg_begin(total, p.P, c + 1);
     const long long n_tiles = t1 - t0;
 
     if (threadIdx.x == 0) {
@@ -168,7 +207,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                     break;
                 const long long t = t0 + it;
                 sb = seq_at<kBatched>(p, t, sb);
-                const TcSeq &sq = p.seq[sb];
+                const TcSeq &sq = seqs[sb];
                 const long long tl = t - sq.tile_base;
                 const int u = (int)(tl / sq.T);
                 const int j = (int)(tl % sq.T);
@@ -222,7 +261,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             for (long long it = 0; it < n_tiles && ok; ++it) {
                 const long long t = t0 + it;
                 sb = seq_at<kBatched>(p, t, sb);
-                const bool first = (it == 0) || ((t - p.seq[sb].tile_base) % p.seq[sb].T == 0);
+                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
                 if (first)
                     ++sg;
                 const int s = (int)(it % kStages);
@@ -273,7 +312,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 
         struct Seg {
             long long start, end, u_first, u_last;  // flattened tile indices
-            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N;
+            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N, ns;
             bool valid;
             uint64_t anc;
             const __nv_bfloat16 *q;
@@ -283,7 +322,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         auto describe = [&](long long t) {
             Seg g;
             sb = seq_at<kBatched>(p, t, sb);
-            const TcSeq &sq = p.seq[sb];
+            const TcSeq &sq = seqs[sb];
             g.b = sb;
             g.start = t;
             g.u = (int)((t - sq.tile_base) / sq.T);
@@ -302,6 +341,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             g.anc = g.valid ? sq.tree->anc[g.node] : 0ull;
             g.L = sq.L;
             g.N = sq.N;
+            g.ns = sq.nstride;
             g.q = sq.q;
             g.out = sq.out;
             return g;
@@ -310,7 +350,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         // operand of QK^T); zeros for padding rows
         auto write_q = [&](const Seg &g) {
             const uint4 *src =
-                reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
+                reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.ns + g.node) * p.Hq + g.qh) * kD);
 #pragma unroll 1
             for (int qc = 0; qc < 4; ++qc) {
                 uint32_t w[16];
@@ -463,7 +503,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             {
                 const float inv = 1.f / l;
                 uint4 *dst =
-                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.N + g.node) * p.Hq + g.qh) * kD);
+                    reinterpret_cast<uint4 *>(g.out + (((size_t)g.layer_rel * g.ns + g.node) * p.Hq + g.qh) * kD);
                 float4 *pdst = reinterpret_cast<float4 *>(slot + rloc * kD);
 #pragma unroll 1
                 for (int c0 = 0; c0 < kD; c0 += 32) {
@@ -526,20 +566,31 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 template <bool kBatched>
 __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__ TcParams p)
 {
+    __shared__ TcSeq s_seq;
+    __shared__ long long s_total;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const TcSeq *seqs = p.seq;
+    long long total = p.total;
+    if (p.sched) {
+        if (threadIdx.x == 0)
+            sched_plan(p, &s_seq, &s_total);
+        __syncthreads();
+        seqs = &s_seq;
+        total = s_total;
+    }
     const int cb = blockIdx.x + 1;  // CTA range starting at tile t_c
-    const long long tc = tc_seg_begin(p, cb);
+    const long long tc = tc_seg_begin(total, p.P, cb);
     int b = 0;
     if constexpr (kBatched) {
-        while (b + 1 < p.n_seq && tc >= p.seq[b + 1].tile_base)
+        while (b + 1 < p.n_seq && tc >= seqs[b + 1].tile_base)
             ++b;
     }
-    const TcSeq &sq = p.seq[b];
+    const TcSeq &sq = seqs[b];
     const int u = (int)((tc - sq.tile_base) / sq.T);
     const long long u_first = sq.tile_base + (long long)u * sq.T, u_last = u_first + sq.T;
     if (tc == u_first)
         return;  // the boundary is a unit boundary
-    const int c_lo = tc_cta_of(p, u_first), c_hi = tc_cta_of(p, u_last - 1);
+    const int c_lo = tc_cta_of(total, p.P, u_first), c_hi = tc_cta_of(total, p.P, u_last - 1);
     if (cb != c_lo + 1)
         return;  // an earlier boundary inside this unit handles it
     const int nseg = c_hi - c_lo + 1;
@@ -555,7 +606,7 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
     for (int j0 = 0; j0 < nseg; j0 += 32) {
         const int cc = c_lo + j0 + lane;
         if (j0 + lane < nseg) {
-            const float *sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
+            const float *sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, p.P, cc) >= u_first ? 0 : 1)) * kSlot;
             M = fmaxf(M, __ldcg(sl + 128 * kD + r));
         }
     }
@@ -569,7 +620,7 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
         const float *sl = p.part;
         float w = 0.f;
         if (j0 + lane < nseg) {
-            sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(p, cc) >= u_first ? 0 : 1)) * kSlot;
+            sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, p.P, cc) >= u_first ? 0 : 1)) * kSlot;
             const float ms = __ldcg(sl + 128 * kD + r);
             w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             lsum += w * __ldcg(sl + 128 * kD + 128 + r);
@@ -603,7 +654,7 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
     const int grow = rb * 128 + r;
     const int node = grow / p.group;
     const int qh = head * p.group + grow % p.group;
-    uint2 *dst = reinterpret_cast<uint2 *>(sq.out + (((size_t)layer_rel * sq.N + node) * p.Hq + qh) * kD) + lane;
+    uint2 *dst = reinterpret_cast<uint2 *>(sq.out + (((size_t)layer_rel * sq.nstride + node) * p.Hq + qh) * kD) + lane;
     *dst = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
 }
 
@@ -680,6 +731,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
         sq.row_blocks = pl.row_blocks;
         sq.T = pl.T;
         sq.unit_base = units;
+        sq.nstride = seqs[b].N;
         tiles += pl.total;
         units += pl.n_units;
         max_rows = pl.rows < 128 ? (pl.rows > max_rows ? pl.rows : max_rows) : 128;
@@ -713,6 +765,56 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
         if (p.P > 1)
             k1_merge_split<true><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
+                                 cudaStream_t stream, const char **err)
+{
+    if (sc.n_rungs < 1 || sc.n_rungs > 8) {
+        *err = "scheduled attention: 1..8 rungs";
+        return cudaErrorInvalidValue;
+    }
+    const tb_kv *kv = sc.kv;
+    TcParams p{};
+    // the cache's whole capacity: keys past L + N are masked by the kernel
+    if (!make_tmap_kv(&p.tmap[0], kv->k, kD, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+                      kv->layer_stride, kBN, err) ||
+        !make_tmap_kv(&p.tmap[1], kv->v, kD, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+                      kv->layer_stride, kBN, err))
+        return cudaErrorInvalidValue;
+    TcSeq &sq = p.seq[0];
+    sq.q = static_cast<const __nv_bfloat16 *>(sc.q);
+    sq.out = static_cast<__nv_bfloat16 *>(sc.out);
+    sq.tree = sc.rung_tree[0];
+    sq.nstride = sc.N_max;
+    sq.T = 1;
+    sq.row_blocks = 1;
+    p.n_seq = 1;
+    p.Hq = Hq;
+    p.Hkv = kv->n_kv_heads;
+    p.group = Hq / kv->n_kv_heads;
+    p.layer_begin = 0;
+    p.n_layers = kv->n_layers;
+    p.L_cap = kv->L_cap;
+    p.P = n_sm;
+    p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
+    p.part = part;
+    p.counters = counters;
+    p.status = status;
+    p.sched = sc.sched;
+    p.n_rungs = sc.n_rungs;
+    for (int r = 0; r < sc.n_rungs; ++r)
+        p.rung_tree[r] = sc.rung_tree[r];
+    const int max_rows = sc.N_max * p.group < 128 ? sc.N_max * p.group : 128;
+    cudaError_t e;
+    if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
+        return e;
+    k1_tree_attention_tc<false><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+    if ((e = cudaGetLastError()) != cudaSuccess)
+        return e;
+    if (p.P > 1)
+        k1_merge_split<false><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

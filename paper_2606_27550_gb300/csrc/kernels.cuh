@@ -62,6 +62,18 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
 bool attn_tc_supported(int d, int rows);
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
 size_t attn_tc_slot_floats();
+// scheduled mode: the tree (rung_tree[sched[0]]) and L (sched[1]) are read on
+// the device; q / out hold N_max nodes per layer; all kv->n_layers layers
+struct AttnSched {
+    const tb_kv *kv;
+    const TreeDesc *rung_tree[8];
+    int n_rungs, N_max;
+    const int32_t *sched;
+    const void *q;
+    void *out;
+};
+cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
+                                 cudaStream_t stream, const char **err);
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
                            const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
                            cudaStream_t stream, const char **err);
@@ -86,6 +98,18 @@ struct AcceptParams {
     int n_layers, n_kv_heads, row_bytes;
     int L_cap;        // slots per head: copies touching slots >= L_cap are skipped
     int from_result;  // compaction driven by an existing result (kv_compact): no acceptance
+    // scheduled mode (sched != null, one sequence): tree = rung_tree[sched[0]],
+    // drafts = draft + sched[0] * n_max, L = sched[1]; the last CTA to finish
+    // (arrival ticket) evaluates the feature and the policy and writes the
+    // next state: rung, L + accept_len, step + 1, feature bits, accept_len
+    int32_t *sched;
+    const TreeDesc *rung_tree[8];
+    int n_rungs, n_max;
+    int *ticket;
+    int pol_kind, pol_feature, n_trace, n_heads;
+    float pol_a, pol_b, pol_edges[7];
+    const float *trace;
+    const float *top1, *entropy;
 };
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
 cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream);

@@ -145,6 +145,7 @@ bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_h
 // Counters sit at fixed offsets so that calls of different shapes sharing one
 // workspace always find them zero; partials are written before they are read.
 
+constexpr size_t kTicketOff = 128;  // scheduled acceptance: arrival ticket, inside the status page
 constexpr size_t kAttnCounterOff = 256;
 constexpr int kMaxAttnUnits = 16384;
 constexpr size_t kLmCounterOff = kAttnCounterOff + (size_t)kMaxAttnUnits * 4;
@@ -1040,6 +1041,149 @@ extern "C" tb_status verify_step_batched_typical(const tb_bank *bank, int batch,
         return fail(TB_EINVAL, "%s: typical-acceptance parameters are NULL", fn);
     return verify_step_batched_impl(bank, batch, seqs, n_q_heads, hidden, lm_head, d_model, vocab, argmax, top1,
                                     entropy, params, workspace, workspace_bytes, flags, stream, fn);
+}
+
+// ------------------------------------------------------------------ device-driven loop
+
+static tb_status check_policy(const tb_bank *bank, const tb_policy *pol, const char *fn, int *n_max)
+{
+    if (!pol)
+        return fail(TB_EINVAL, "%s: policy is NULL", fn);
+    if (pol->n_rungs < 1 || pol->n_rungs > 8)
+        return fail(TB_EINVAL, "%s: %d rungs (1..8)", fn, pol->n_rungs);
+    if (pol->kind < TB_POLICY_HYSTERETIC_LADDER || pol->kind > TB_POLICY_THRESHOLD_LADDER)
+        return fail(TB_EINVAL, "%s: policy kind %d", fn, pol->kind);
+    if (pol->feature < TB_FEATURE_TRACE || pol->feature > TB_FEATURE_ENTROPY)
+        return fail(TB_EINVAL, "%s: feature %d", fn, pol->feature);
+    if (pol->kind == TB_POLICY_BINARY && (pol->n_rungs != 2 || !(pol->b <= pol->a)))
+        return fail(TB_EINVAL, "%s: the binary policy takes 2 rungs and tau_off <= tau_on", fn);
+    if (pol->kind != TB_POLICY_THRESHOLD_LADDER && !(std::isfinite(pol->a) && std::isfinite(pol->b)))
+        return fail(TB_EINVAL, "%s: thresholds must be finite", fn);
+    if (pol->kind == TB_POLICY_THRESHOLD_LADDER)
+        for (int i = 0; i + 1 < pol->n_rungs; ++i)
+            if (!std::isfinite(pol->edges[i]) || (i > 0 && pol->edges[i] < pol->edges[i - 1]))
+                return fail(TB_EINVAL, "%s: ladder edges must be finite and ascending", fn);
+    const bool uses_trace = pol->feature == TB_FEATURE_TRACE ||
+                            (pol->feature == TB_FEATURE_PATH_VALUE && pol->n_heads > 0);
+    if (pol->feature == TB_FEATURE_PATH_VALUE && (pol->n_heads < 0 || pol->n_heads > 8))
+        return fail(TB_EINVAL, "%s: %d head probabilities per step (0..8)", fn, pol->n_heads);
+    if (uses_trace && (!pol->trace || pol->n_trace < 1))
+        return fail(TB_EINVAL, "%s: the feature needs a device trace with at least one entry", fn);
+    int nm = 0;
+    for (int r = 0; r < pol->n_rungs; ++r) {
+        tb_status st = check_bank(bank, pol->bank_ids[r], fn);
+        if (st != TB_OK)
+            return st;
+        const int n = bank->h_desc[pol->bank_ids[r]].n;
+        nm = n > nm ? n : nm;
+    }
+    if (pol->node_stride != 0 && (pol->node_stride < nm || pol->node_stride > kMaxNodes))
+        return fail(TB_EINVAL, "%s: node_stride %d below the largest tree (%d) or above %d", fn, pol->node_stride,
+                    nm, kMaxNodes);
+    *n_max = pol->node_stride != 0 ? pol->node_stride : nm;
+    return TB_OK;
+}
+
+extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy *policy, tb_state *state,
+                                           const tb_kv *kv, const void *q, int n_q_heads, const void *hidden,
+                                           const void *lm_head, int d_model, int vocab, const int32_t *draft_tokens,
+                                           void *attn_out, int32_t *argmax, float *top1, float *entropy,
+                                           tb_result *result, void *workspace, size_t workspace_bytes, int flags,
+                                           tb_stream stream)
+{
+    const char *fn = "verify_step_scheduled";
+    if (!bank)
+        return fail(TB_EINVAL, "%s: bank is NULL", fn);
+    int N_max = 0;
+    tb_status st = check_policy(bank, policy, fn, &N_max);
+    if (st != TB_OK)
+        return st;
+    if (!state || (reinterpret_cast<uintptr_t>(state) & 3u))
+        return fail(TB_EINVAL, "%s: state NULL or not 4-byte aligned", fn);
+    if (!kv)
+        return fail(TB_EINVAL, "%s: kv is NULL", fn);
+    tb_kv kv0 = *kv;
+    kv0.L = 0;  // the prefix length lives in *state
+    if ((st = check_kv(&kv0, N_max, fn)) != TB_OK)
+        return st;
+    if (kv->head_dim != 128)
+        return fail(TB_EUNSUPPORTED, "%s: head_dim %d (the device-driven loop runs head_dim 128)", fn, kv->head_dim);
+    if (n_q_heads < kv->n_kv_heads || n_q_heads % kv->n_kv_heads)
+        return fail(TB_EINVAL, "%s: n_q_heads %d not a multiple of n_kv_heads %d", fn, n_q_heads, kv->n_kv_heads);
+    if (N_max * (n_q_heads / kv->n_kv_heads) > 256)
+        return fail(TB_EUNSUPPORTED, "%s: N_max * group = %d > 256", fn, N_max * (n_q_heads / kv->n_kv_heads));
+    if (!q || !attn_out || !aligned16(q) || !aligned16(attn_out))
+        return fail(TB_EINVAL, "%s: q / attn_out NULL or not 16-byte aligned", fn);
+    if (!draft_tokens || !result)
+        return fail(TB_EINVAL, "%s: draft_tokens / result is NULL", fn);
+    LmPlan lplan;
+    if ((st = lm_validate(hidden, N_max, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
+        return st;
+    const int nsm = sm_count(bank->device);
+    const size_t attn_bytes = attn_part_bytes(nsm, kv->head_dim);
+    if ((st = check_ws(workspace, workspace_bytes, kPartBase + attn_bytes + lplan.ws_bytes, fn)) != TB_OK)
+        return st;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = (cudaStream_t)stream;
+    AttnSched sc{};
+    sc.kv = kv;
+    sc.n_rungs = policy->n_rungs;
+    sc.N_max = N_max;
+    sc.sched = reinterpret_cast<const int32_t *>(state);
+    sc.q = q;
+    sc.out = attn_out;
+    for (int r = 0; r < policy->n_rungs; ++r)
+        sc.rung_tree[r] = bank->d_desc + policy->bank_ids[r];
+    {
+        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
+        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step_scheduled: fork");
+        const char *err = "";
+        e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
+                                 reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
+                                 &err);
+        if (e == cudaErrorInvalidValue && err[0])
+            return fail(TB_EINVAL, "%s: %s", fn, err);
+        if (e != cudaSuccess)
+            return cuda_fail(e, fn);
+        if ((st = lm_enqueue(hidden, N_max, lm_head, d_model, vocab, argmax, top1, entropy, ws,
+                             kPartBase + attn_bytes, bank->aux, fn)) != TB_OK)
+            return st;
+        e = cudaEventRecord(bank->ev_join, bank->aux);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step_scheduled: join");
+    }
+    AcceptParams p = accept_params(bank, policy->bank_ids[0], draft_tokens, argmax, vocab, 0, result,
+                                   reinterpret_cast<const int *>(ws));
+    if (!(flags & TB_NO_COMPACT))
+        add_compaction(p, kv);
+    p.L_cap = kv->L_cap;
+    p.sched = reinterpret_cast<int32_t *>(state);
+    p.n_rungs = policy->n_rungs;
+    for (int r = 0; r < policy->n_rungs; ++r)
+        p.rung_tree[r] = sc.rung_tree[r];
+    p.n_max = N_max;
+    p.ticket = reinterpret_cast<int *>(ws + kTicketOff);
+    p.pol_kind = policy->kind;
+    p.pol_feature = policy->feature;
+    p.n_trace = policy->n_trace;
+    p.n_heads = policy->feature == TB_FEATURE_PATH_VALUE ? policy->n_heads : 0;
+    p.pol_a = policy->a;
+    p.pol_b = policy->b;
+    for (int i = 0; i < 7; ++i)
+        p.pol_edges[i] = policy->edges[i];
+    p.trace = policy->trace;
+    p.top1 = top1;
+    p.entropy = entropy;
+    cudaError_t e = accept_launch(p, nsm, s);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return ok();
 }
 
 // ------------------------------------------------------------------ per-step tree selection
