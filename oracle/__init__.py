@@ -50,6 +50,10 @@ def _load():
             lib.oracle_typical_accept.argtypes = [P, i32, P, P, i32, d, d, d, P, P, P, P, P, P]
             lib.oracle_typical_accept.restype = ctypes.c_int
             lib.oracle_tempered_stats.argtypes = [P, i32, i32, d, P, P]
+            lib.oracle_rope.argtypes = [P, i32, i32, P, d, P]
+            lib.oracle_rope.restype = ctypes.c_int
+            lib.oracle_tree_attention_rope.argtypes = [P, P, P, i64, i32, i32, i32, i32, i32, P, d, P, P]
+            lib.oracle_tree_attention_rope.restype = ctypes.c_int
             lib.oracle_tempered_stats.restype = ctypes.c_int
             for f in (lib.oracle_tree, lib.oracle_tree_attention, lib.oracle_lm_head,
                       lib.oracle_accept, lib.oracle_num_threads):
@@ -223,3 +227,39 @@ def policy_next(kind: str, rung: int, n_rungs: int, feature: float, a: float = 0
             k += 1
         return k
     raise ValueError(kind)
+
+
+# ---------------------------------------------------------------- rotary position embedding
+
+def rope(x, pos, base: float = 10000.0):
+    """Rotary embedding of bf16 rows x [rows][d] at positions pos[rows] (float64 out)."""
+    x = np.ascontiguousarray(x, dtype=np.uint16)
+    rows, d = x.shape
+    pos = np.ascontiguousarray(pos, dtype=np.int32)
+    y = np.zeros((rows, d))
+    if _load().oracle_rope(_ptr(x), rows, d, _ptr(pos), base, _ptr(y)) != 0:
+        raise ValueError("bad shape or base")
+    return y
+
+
+def tree_attention_rope(q, k, v, L: int, parent, base: float = 10000.0):
+    """One layer of tree-masked attention with the rotary embedding at the tree's
+    position offsets (node i at L + depth(i)); q and the tree slots of k are
+    pre-rotary, the prefix keys already rotated.
+
+    Returns (out float64 [N][Hq][d], rotated tree keys as bf16 bits [Hkv][N][d])."""
+    q = np.ascontiguousarray(q, dtype=np.uint16)
+    k = np.ascontiguousarray(k, dtype=np.uint16)
+    v = np.ascontiguousarray(v, dtype=np.uint16)
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    N, Hq, d = q.shape
+    Hkv = k.shape[0]
+    if k.shape[1] < L + N or k.shape != v.shape or k.shape[2] != d:
+        raise ValueError("bad kv shape")
+    out = np.zeros((N, Hq, d))
+    k_rot = np.zeros((Hkv, N, d), dtype=np.uint16)
+    rc = _load().oracle_tree_attention_rope(_ptr(q), _ptr(k), _ptr(v), k.shape[1] * d, L, N, Hq, Hkv, d,
+                                            _ptr(parent), base, _ptr(out), _ptr(k_rot))
+    if rc != 0:
+        raise ValueError(f"oracle_tree_attention_rope rc={rc}")
+    return out, k_rot

@@ -386,3 +386,123 @@ int oracle_tempered_stats(const double *logits, int R, int V, double temperature
     }
     return 0;
 }
+
+static uint16_t bf16_round(double x)
+{
+    /* float64 -> float32 (round to nearest) -> bf16 bits (round to nearest even); finite inputs */
+    float f = (float)x;
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+/*
+ * Rotary position embedding of the base model (Llama: frequencies
+ * theta_i = base^(-2i/d), i < d/2, element i paired with element i + d/2):
+ *   y_i       = x_i cos(p theta_i) - x_{i+d/2} sin(p theta_i)
+ *   y_{i+d/2} = x_{i+d/2} cos(p theta_i) + x_i sin(p theta_i)
+ * for row r at position pos[r].  x: bf16 bits [rows][d]; y: double [rows][d].
+ */
+int oracle_rope(const uint16_t *x, int rows, int d, const int32_t *pos, double base, double *y)
+{
+    if (rows < 0 || d < 2 || d % 2 || !(base > 0.0))
+        return -1;
+    const int h = d / 2;
+    for (int r = 0; r < rows; ++r)
+        for (int i = 0; i < h; ++i) {
+            const double th = pow(base, -2.0 * i / d);
+            const double a = (double)pos[r] * th;
+            const double c = cos(a), s = sin(a);
+            const double x1 = bf16_value(x[(size_t)r * d + i]), x2 = bf16_value(x[(size_t)r * d + i + h]);
+            y[(size_t)r * d + i] = x1 * c - x2 * s;
+            y[(size_t)r * d + i + h] = x2 * c + x1 * s;
+        }
+    return 0;
+}
+
+/*
+ * Tree-masked attention with the rotary embedding applied at the tree's
+ * position offsets (TopologyBank "position offsets", Sec. 1 / 2.3): node i sits
+ * at position L + depth(i).  Inputs are pre-rotary for the step's tokens:
+ * q [N][Hq][d] and the tree slots L + j of k; the prefix slots [0, L) of k hold
+ * keys already rotated at their own positions (as a KV cache does).  The
+ * rotated tree keys are stored back into the bf16 cache, so they are rounded
+ * to bf16 (written to k_rot [Hkv][N][d] as bits); q stays in double.
+ *   k, v  [Hkv][head_stride] rows as in oracle_tree_attention
+ *   out   [N][Hq][d] double
+ */
+int oracle_tree_attention_rope(const uint16_t *q, const uint16_t *k, const uint16_t *v, int64_t head_stride, int L,
+                               int N, int Hq, int Hkv, int d, const int32_t *parent, double base, double *out,
+                               uint16_t *k_rot)
+{
+    if (Hkv < 1 || Hq % Hkv != 0 || d < 2 || d % 2 || L < 0 || !(base > 0.0))
+        return -1;
+    uint8_t in_anc[ORACLE_MAX_NODES * ORACLE_MAX_NODES];
+    int32_t depth[ORACLE_MAX_NODES];
+    if (oracle_tree(parent, N, depth, in_anc) != 0)
+        return -1;
+    int32_t pos[ORACLE_MAX_NODES];
+    for (int i = 0; i < N; ++i)
+        pos[i] = L + depth[i];
+    /* rotated tree keys, rounded to the cache's bf16 */
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)N * d);
+    if (!tmp)
+        return -2;
+    for (int g = 0; g < Hkv; ++g) {
+        oracle_rope(k + (size_t)g * head_stride + (size_t)L * d, N, d, pos, base, tmp);
+        for (size_t e = 0; e < (size_t)N * d; ++e)
+            k_rot[(size_t)g * N * d + e] = bf16_round(tmp[e]);
+    }
+    free(tmp);
+    const int group = Hq / Hkv;
+    const double scale = 1.0 / sqrt((double)d);
+#pragma omp parallel
+    {
+        double *score = (double *)malloc(sizeof(double) * (size_t)(L + N));
+        double *qr = (double *)malloc(sizeof(double) * (size_t)d);
+        const double *kp[1];
+        (void)kp;
+#pragma omp for schedule(dynamic)
+        for (int ih = 0; ih < N * Hq; ++ih) {
+            const int i = ih / Hq, h = ih % Hq, g = h / group;
+            oracle_rope(q + ((size_t)i * Hq + h) * d, 1, d, &pos[i], base, qr);
+            const uint16_t *kg = k + (size_t)g * head_stride;
+            const uint16_t *vg = v + (size_t)g * head_stride;
+            const uint16_t *kt = k_rot + (size_t)g * N * d;
+            double mx = -INFINITY;
+            int n = 0;
+            for (int s = 0; s < L + N; ++s) {
+                if (s >= L && !in_anc[(size_t)i * N + (s - L)])
+                    continue;
+                const uint16_t *ks = s < L ? kg + (size_t)s * d : kt + (size_t)(s - L) * d;
+                double dot = 0.0;
+                for (int c = 0; c < d; ++c)
+                    dot += qr[c] * bf16_value(ks[c]);
+                score[s] = dot * scale;
+                if (score[s] > mx)
+                    mx = score[s];
+                ++n;
+            }
+            double denom = 0.0;
+            for (int s = 0; s < L + N; ++s)
+                if (s < L || in_anc[(size_t)i * N + (s - L)]) {
+                    score[s] = exp(score[s] - mx);
+                    denom += score[s];
+                }
+            double *o = out + ((size_t)i * Hq + h) * d;
+            for (int c = 0; c < d; ++c)
+                o[c] = 0.0;
+            for (int s = 0; s < L + N; ++s)
+                if (s < L || in_anc[(size_t)i * N + (s - L)]) {
+                    const uint16_t *vs = vg + (size_t)s * d;
+                    const double w = score[s] / denom;
+                    for (int c = 0; c < d; ++c)
+                        o[c] += w * bf16_value(vs[c]);
+                }
+        }
+        free(score);
+        free(qr);
+    }
+    return 0;
+}
