@@ -175,7 +175,9 @@ def run_gpu(args):
 
     bank = tv.Bank(16, local)
     bid, order = bank.add(sh.parent)
-    kv = tv.KvCache(k, v, L)
+    # --rope: the queries and tree keys are pre-rotary and every call applies the rotary
+    # embedding at L + depth (the tree slots are rotated in place again each step: timing only)
+    kv = tv.KvCache(k, v, L, rope_theta=10000.0 if args.rope else 0.0)
     out = torch.empty((nl, N, H, d), dtype=bf, device=dev)
     am = torch.empty(N, dtype=torch.int32, device=dev)
     t1 = torch.empty(N, dtype=torch.float32, device=dev)
@@ -303,7 +305,7 @@ def run_gpu(args):
         "config": {"workload": sh.name, "layers": nl, "q_heads": H, "kv_heads": Hkv, "head_dim": d, "L": L,
                    "tree_nodes": N, "tree_depth": int(synth.depth_of(sh.parent).max()), "d_model": D, "vocab": V,
                    "batch": 1, "l2": f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)",
-                   "acceptance": acceptance_label(args)},
+                   "acceptance": acceptance_label(args), "rope": "in-kernel, theta 10000" if args.rope else "none"},
         "tree_tokens_per_s": round(value * N, 1),
         "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
                          "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
@@ -318,7 +320,8 @@ def run_gpu(args):
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         # per step: LM head, attention, split-unit merge (head_dim 128), acceptance + compaction
-        "gpu_launches": (4 if d == 128 else 3) * args.steps,
+        # (+ the rotary table and tree-key rotation with --rope)
+        "gpu_launches": ((4 if d == 128 else 3) + (2 if args.rope else 0)) * args.steps,
         "clocks": clocks,
     }
     if args.layers:
@@ -821,6 +824,8 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=None, help="override the layer count (smaller profiling cases)")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--rope", action="store_true",
+                    help="c1/c2/c4: pre-rotary inputs, rotary embedding applied by the library (head_dim 128)")
     ap.add_argument("--scheduled", action="store_true",
                     help="c3 only: the device-driven loop (tree and L on the device, CUDA-graph replay)")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],

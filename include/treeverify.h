@@ -109,7 +109,18 @@ TB_API tb_status tb_destroy(tb_bank *bank);
  * Slots [0, L) hold the prefix; the N tree nodes of the step occupy slots
  * [L, L + N) in canonical node order (the keys/values of the draft tokens,
  * produced by the model's K/V projection before the call).  Strides are in
- * elements and must be multiples of 8; head_dim is 64 or 128. */
+ * elements and must be multiples of 8; head_dim is 64 or 128.
+ *
+ * rope_theta = 0: the queries and every key are already rotary-embedded.
+ * rope_theta > 0 (head_dim 128): the calls apply the base model's rotary
+ * embedding (Llama convention: frequencies rope_theta^(-2i/d), element i
+ * paired with element i + d/2) at the tree's position offsets, node i at
+ * position L + depth(i): the queries are passed pre-rotary, and the tree
+ * slots [L, L + N) of K hold pre-rotary keys when the call starts; the call
+ * rotates them in place (the cache then holds rotated keys, as for the
+ * prefix, and the accepted ones keep their positions after compaction: path
+ * index i has depth i).  A second call on the same tree slots would rotate
+ * them again. */
 typedef struct tb_kv {
     void *k;
     void *v;
@@ -118,8 +129,9 @@ typedef struct tb_kv {
     int32_t n_layers;
     int32_t n_kv_heads;
     int32_t head_dim;
-    int32_t L;     /* prefix length of this step */
-    int32_t L_cap; /* slots per head: L + N <= L_cap */
+    int32_t L;          /* prefix length of this step */
+    int32_t L_cap;      /* slots per head: L + N <= L_cap */
+    float rope_theta;   /* 0, or the rotary base (e.g. 10000) applied by the call */
 } tb_kv;
 
 /* Device-resident result of one verification, written by the GPU. */

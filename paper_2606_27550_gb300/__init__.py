@@ -44,7 +44,8 @@ class TreeVerifyError(RuntimeError):
 class TbKv(ctypes.Structure):
     _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("layer_stride", ctypes.c_int64),
                 ("head_stride", ctypes.c_int64), ("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
-                ("head_dim", ctypes.c_int32), ("L", ctypes.c_int32), ("L_cap", ctypes.c_int32)]
+                ("head_dim", ctypes.c_int32), ("L", ctypes.c_int32), ("L_cap", ctypes.c_int32),
+                ("rope_theta", ctypes.c_float)]
 
 
 class TbSeq(ctypes.Structure):
@@ -218,11 +219,13 @@ class KvCache:
     k: object
     v: object
     L: int
+    rope_theta: float = 0.0  # > 0: the call rotary-embeds q and the tree keys at L + depth
 
     def as_c(self) -> TbKv:
         n_layers, n_kv_heads, L_cap, head_dim = self.k.shape
         s = self.k.stride()
-        return TbKv(self.k.data_ptr(), self.v.data_ptr(), s[0], s[1], n_layers, n_kv_heads, head_dim, self.L, L_cap)
+        return TbKv(self.k.data_ptr(), self.v.data_ptr(), s[0], s[1], n_layers, n_kv_heads, head_dim, self.L, L_cap,
+                    float(self.rope_theta))
 
 
 def tb_workspace_size(max_rows: int, n_layers: int, n_kv_heads: int, n_q_heads: int, head_dim: int, vocab: int,

@@ -80,6 +80,9 @@ struct TcParams {
     const int32_t *sched;
     const TreeDesc *rung_tree[8];
     int n_rungs, n_layers, L_cap;
+    // rotary embedding (null: the queries are already rotated): per sequence a
+    // table of (cos, sin) at position L + depth for every pair of head elements
+    const float2 *rope_tab;
 };
 
 // Scheduled mode: the sequence of this step from the device state.  An
@@ -312,7 +315,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
 
         struct Seg {
             long long start, end, u_first, u_last;  // flattened tile indices
-            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N, ns;
+            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N, ns, dep;
             bool valid;
             uint64_t anc;
             const __nv_bfloat16 *q;
@@ -339,6 +342,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
             g.node = g.valid ? grow / p.group : 0;
             g.qh = g.head * p.group + grow % p.group;
             g.anc = g.valid ? sq.tree->anc[g.node] : 0ull;
+            g.dep = g.valid ? sq.tree->depth[g.node] : 0;
             g.L = sq.L;
             g.N = sq.N;
             g.ns = sq.nstride;
@@ -351,18 +355,45 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         auto write_q = [&](const Seg &g) {
             const uint4 *src =
                 reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.ns + g.node) * p.Hq + g.qh) * kD);
+            if (!p.rope_tab) {
 #pragma unroll 1
-            for (int qc = 0; qc < 4; ++qc) {
-                uint32_t w[16];
+                for (int qc = 0; qc < 4; ++qc) {
+                    uint32_t w[16];
 #pragma unroll
-                for (int ch = 0; ch < 4; ++ch) {
-                    const uint4 v = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
-                    w[4 * ch] = v.x;
-                    w[4 * ch + 1] = v.y;
-                    w[4 * ch + 2] = v.z;
-                    w[4 * ch + 3] = v.w;
+                    for (int ch = 0; ch < 4; ++ch) {
+                        const uint4 v = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
+                        w[4 * ch] = v.x;
+                        w[4 * ch + 1] = v.y;
+                        w[4 * ch + 2] = v.z;
+                        w[4 * ch + 3] = v.w;
+                    }
+                    tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, w);
                 }
-                tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, w);
+            } else {
+                // pre-rotary query: element i pairs with i + 64, rotated at position
+                // L + depth(node) with the sequence's (cos, sin) table
+                const float2 *tab = p.rope_tab + (size_t)g.b * kRopeTableEntries + (size_t)g.dep * kRopeMaxHalf;
+#pragma unroll 1
+                for (int qc = 0; qc < 2; ++qc) {
+                    uint32_t wl[16], wh[16];
+#pragma unroll
+                    for (int ch = 0; ch < 4; ++ch) {
+                        const uint4 lo = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
+                        const uint4 hi = g.valid ? src[(qc + 2) * 4 + ch] : make_uint4(0, 0, 0, 0);
+                        const uint32_t lw[4] = {lo.x, lo.y, lo.z, lo.w}, hw[4] = {hi.x, hi.y, hi.z, hi.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int i0 = 32 * qc + 8 * ch + 2 * e;
+                            const float2 c0 = tab[i0], c1 = tab[i0 + 1];
+                            const float a0 = __uint_as_float(lw[e] << 16), a1 = __uint_as_float(lw[e] & 0xffff0000u);
+                            const float b0 = __uint_as_float(hw[e] << 16), b1 = __uint_as_float(hw[e] & 0xffff0000u);
+                            wl[4 * ch + e] = pack_bf16x2(a0 * c0.x - b0 * c0.y, a1 * c1.x - b1 * c1.y);
+                            wh[4 * ch + e] = pack_bf16x2(b0 * c0.x + a0 * c0.y, b1 * c1.x + a1 * c1.y);
+                        }
+                    }
+                    tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, wl);
+                    tmem_st_32x32b_x16(lane_addr + kColQ + (qc + 2) * 16, wh);
+                }
             }
             tmem_st_wait();
             tc_fence_before();
@@ -702,7 +733,8 @@ int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers)
 }
 
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
-                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err)
+                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
+                                 const float2 *rope_tab)
 {
     if (n_seq < 1 || n_seq > kMaxSeqPerLaunch) {
         *err = "too many sequences for one attention launch";
@@ -747,6 +779,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     p.part = part;
     p.counters = counters;
     p.status = status;
+    p.rope_tab = rope_tab;
     cudaError_t e;
     if (n_seq == 1) {
         if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
@@ -803,6 +836,7 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
     p.counters = counters;
     p.status = status;
     p.sched = sc.sched;
+    p.rope_tab = sc.rope_tab;
     p.n_rungs = sc.n_rungs;
     for (int r = 0; r < sc.n_rungs; ++r)
         p.rung_tree[r] = sc.rung_tree[r];
@@ -820,10 +854,11 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
 
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
                            const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                           cudaStream_t stream, const char **err)
+                           cudaStream_t stream, const char **err, const float2 *rope_tab)
 {
     AttnSeq one{kv, d_tree, N, q, out};
-    return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, counters, status, n_sm, stream, err);
+    return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, counters, status, n_sm, stream, err,
+                                rope_tab);
 }
 
 }  // namespace tv

@@ -46,6 +46,30 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
                         const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
                         cudaStream_t stream, const char **err);
 
+// rotary embedding at the tree's position offsets (rope.cu)
+constexpr int kRopeMaxHalf = 64;                                // pairs per head (head_dim <= 128)
+constexpr int kRopeTableEntries = kMaxNodes * kRopeMaxHalf;    // cos / sin per (depth, pair)
+struct RopeSeq {
+    __nv_bfloat16 *k;
+    long long layer_stride, head_stride;  // elements
+    const TreeDesc *tree;
+    int L;
+};
+struct RopeParams {
+    RopeSeq seq[TB_MAX_BATCH];
+    int layer_begin, Hkv, d;
+    double inv_freq[kRopeMaxHalf];
+    float2 *table;  // [n_seq][kRopeTableEntries]: (cos, sin) at position L + depth
+    // scheduled mode: tree = rung_tree[sched[0]], L = sched[1]
+    const int32_t *sched;
+    const TreeDesc *rung_tree[8];
+    int n_rungs, L_cap;
+};
+void rope_inv_freq(double theta, int d, double *inv_freq);
+// the table, then the in-place rotation of every sequence's tree keys in
+// layers [layer_begin, layer_begin + n_layers)
+cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_layers, cudaStream_t stream);
+
 // tree attention on tcgen05 (attention_tc.cu): head_dim 128, one or several
 // sequences (each with its own cache, prefix length and tree) per launch
 constexpr int kMaxSeqPerLaunch = TB_MAX_BATCH;
@@ -57,8 +81,11 @@ struct AttnSeq {
     void *out;
 };
 int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers);
+// rope_tab: null, or the (cos, sin) tables of rope.cu: the queries are then
+// pre-rotary and are rotated at L + depth while they are staged
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
-                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err);
+                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
+                                 const float2 *rope_tab = nullptr);
 bool attn_tc_supported(int d, int rows);
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
 size_t attn_tc_slot_floats();
@@ -71,12 +98,13 @@ struct AttnSched {
     const int32_t *sched;
     const void *q;
     void *out;
+    const float2 *rope_tab;  // null, or the rotary tables (pre-rotary queries)
 };
 cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
                                  cudaStream_t stream, const char **err);
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
                            const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                           cudaStream_t stream, const char **err);
+                           cudaStream_t stream, const char **err, const float2 *rope_tab = nullptr);
 
 // acceptance + compaction (accept.cu)
 struct AcceptParams {

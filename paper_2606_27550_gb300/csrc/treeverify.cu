@@ -141,6 +141,7 @@ bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_h
 //   [256, 256 + 64 KiB)         attention unit counters (16384 int32)
 //   [.., + 4 KiB)               LM-head group counters (1024 int32)
 //   [.., + 12 KiB)              typical acceptance: logZ_T, H_T, draft logits (3 x 1024 float)
+//   [.., + 512 KiB)             rotary tables: (cos, sin) per (depth, pair), one per sequence
 //   [kPartBase, ..)             attention partials, then LM-head partials
 // Counters sit at fixed offsets so that calls of different shapes sharing one
 // workspace always find them zero; partials are written before they are read.
@@ -152,7 +153,8 @@ constexpr size_t kLmCounterOff = kAttnCounterOff + (size_t)kMaxAttnUnits * 4;
 constexpr int kMaxLmCounters = 1024;
 constexpr int kMaxTypRows = 1024;
 constexpr size_t kTypOff = kLmCounterOff + (size_t)kMaxLmCounters * 4;
-constexpr size_t kPartBase = kTypOff + (size_t)3 * kMaxTypRows * 4;
+constexpr size_t kRopeOff = kTypOff + (size_t)3 * kMaxTypRows * 4;
+constexpr size_t kPartBase = kRopeOff + (size_t)TB_MAX_BATCH * kRopeTableEntries * sizeof(float2);
 
 static size_t align256(size_t x)
 {
@@ -524,6 +526,8 @@ struct AttnArgs {
     void *out;
 };
 
+static tb_status check_rope(const tb_kv *kv, const char *fn);
+
 static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan)
 {
     tb_status st = check_bank(a.bank, a.bank_id, fn);
@@ -534,6 +538,8 @@ static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan
         return st;
     if (!a.q || !a.out || !aligned16(a.q) || !aligned16(a.out))
         return fail(TB_EINVAL, "%s: q / out NULL or not 16-byte aligned", fn);
+    if ((st = check_rope(a.kv, fn)) != TB_OK)
+        return st;
     if (a.layer_begin < 0 || a.n_layers < 1 || a.layer_begin + a.n_layers > a.kv->n_layers)
         return fail(TB_EINVAL, "%s: layers [%d, %d) outside the cache's %d", fn, a.layer_begin,
                     a.layer_begin + a.n_layers, a.kv->n_layers);
@@ -551,15 +557,67 @@ static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan
     return TB_OK;
 }
 
+static tb_status check_rope(const tb_kv *kv, const char *fn)
+{
+    if (kv->rope_theta == 0.f)
+        return TB_OK;
+    if (!(kv->rope_theta > 0.f) || !std::isfinite(kv->rope_theta))
+        return fail(TB_EINVAL, "%s: rope_theta %g (0, or a positive base)", fn, (double)kv->rope_theta);
+    if (kv->head_dim != 128)
+        return fail(TB_EUNSUPPORTED, "%s: the rotary embedding runs with head_dim 128 (got %d)", fn, kv->head_dim);
+    return TB_OK;
+}
+
+static float2 *rope_table(uint8_t *ws)
+{
+    return reinterpret_cast<float2 *>(ws + kRopeOff);
+}
+
+// Rotary tables and in-place rotation of the tree keys of n_seq sequences
+// (layers [layer_begin, layer_begin + n_layers)), before their attention.
+static tb_status rope_enqueue(RopeParams &rp, const tb_kv *kv0, int n_seq, int layer_begin, int n_layers,
+                              int max_nodes, uint8_t *ws, cudaStream_t s, const char *fn)
+{
+    rp.layer_begin = layer_begin;
+    rp.Hkv = kv0->n_kv_heads;
+    rp.d = kv0->head_dim;
+    rope_inv_freq((double)kv0->rope_theta, kv0->head_dim, rp.inv_freq);
+    rp.table = rope_table(ws);
+    cudaError_t e = rope_launch(rp, n_seq, max_nodes, n_layers, s);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return TB_OK;
+}
+
+static RopeSeq rope_seq(const tb_kv *kv, const TreeDesc *tree)
+{
+    return RopeSeq{static_cast<__nv_bfloat16 *>(kv->k), (long long)kv->layer_stride, (long long)kv->head_stride,
+                   tree, kv->L};
+}
+
 static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn)
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
     const int rows = N * (a.Hq / a.kv->n_kv_heads);
-    auto launch = use_tc_attention(a.kv->head_dim, rows) ? attn_tc_launch : attn_launch;
-    cudaError_t e = launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
+    const bool rope = a.kv->rope_theta != 0.f;
+    if (rope) {
+        RopeParams rp{};
+        rp.seq[0] = rope_seq(a.kv, a.bank->d_desc + a.bank_id);
+        tb_status st = rope_enqueue(rp, a.kv, 1, a.layer_begin, a.n_layers, N, ws, stream, fn);
+        if (st != TB_OK)
+            return st;
+    }
+    cudaError_t e;
+    if (use_tc_attention(a.kv->head_dim, rows))
+        e = attn_tc_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
                            reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                           reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
+                           reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err,
+                           rope ? rope_table(ws) : nullptr);
+    else
+        e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
+                        reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
+                        reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -900,8 +958,10 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
         Ns[b] = bank->h_desc[sq.bank_id].n;
         if ((st = check_kv(&sq.kv, Ns[b], fn)) != TB_OK)
             return st;
+        if ((st = check_rope(&sq.kv, fn)) != TB_OK)
+            return st;
         if (sq.kv.n_layers != seqs[0].kv.n_layers || sq.kv.n_kv_heads != seqs[0].kv.n_kv_heads ||
-            sq.kv.head_dim != seqs[0].kv.head_dim)
+            sq.kv.head_dim != seqs[0].kv.head_dim || sq.kv.rope_theta != seqs[0].kv.rope_theta)
             return fail(TB_EINVAL, "%s: sequence %d has another layer / head / head_dim count than sequence 0", fn,
                         b);
         if (!sq.q || !sq.attn_out || !sq.draft_tokens || !sq.result || !aligned16(sq.q) || !aligned16(sq.attn_out))
@@ -948,15 +1008,26 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
         e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
     if (e != cudaSuccess)
         return cuda_fail(e, "verify_step_batched: fork");
-    // tree attention of every sequence
+    // tree attention of every sequence (after the rotary embedding of their tree keys)
     if (tc) {
+        const bool rope = kv0.rope_theta != 0.f;
+        if (rope) {
+            RopeParams rp{};
+            int max_nodes = 1;
+            for (int b = 0; b < batch; ++b) {
+                rp.seq[b] = rope_seq(&seqs[b].kv, bank->d_desc + seqs[b].bank_id);
+                max_nodes = Ns[b] > max_nodes ? Ns[b] : max_nodes;
+            }
+            if ((st = rope_enqueue(rp, &kv0, batch, 0, kv0.n_layers, max_nodes, ws, s, fn)) != TB_OK)
+                return st;
+        }
         AttnSeq as[TB_MAX_BATCH];
         for (int b = 0; b < batch; ++b)
             as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
         const char *err = "";
         e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err);
+                                 &err, rope ? rope_table(ws) : nullptr);
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
@@ -1108,6 +1179,8 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
         return st;
     if (kv->head_dim != 128)
         return fail(TB_EUNSUPPORTED, "%s: head_dim %d (the device-driven loop runs head_dim 128)", fn, kv->head_dim);
+    if ((st = check_rope(kv, fn)) != TB_OK)
+        return st;
     if (n_q_heads < kv->n_kv_heads || n_q_heads % kv->n_kv_heads)
         return fail(TB_EINVAL, "%s: n_q_heads %d not a multiple of n_kv_heads %d", fn, n_q_heads, kv->n_kv_heads);
     if (N_max * (n_q_heads / kv->n_kv_heads) > 256)
@@ -1141,6 +1214,18 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
             e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
         if (e != cudaSuccess)
             return cuda_fail(e, "verify_step_scheduled: fork");
+        if (kv->rope_theta != 0.f) {
+            RopeParams rp{};
+            rp.seq[0] = rope_seq(kv, sc.rung_tree[0]);
+            rp.sched = sc.sched;
+            rp.n_rungs = sc.n_rungs;
+            rp.L_cap = kv->L_cap;
+            for (int r = 0; r < sc.n_rungs; ++r)
+                rp.rung_tree[r] = sc.rung_tree[r];
+            if ((st = rope_enqueue(rp, kv, 1, 0, kv->n_layers, N_max, ws, s, fn)) != TB_OK)
+                return st;
+            sc.rope_tab = rope_table(ws);
+        }
         const char *err = "";
         e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
