@@ -30,15 +30,39 @@
 
 namespace tv {
 
+// Slot L + j takes slot L + path[j] for 1 <= j < k (slot L + path[0] = L is the
+// root itself).  path is strictly increasing with path[j] >= j, so in a chunk
+// of consecutive j no copy reads a slot that a copy of a later chunk writes,
+// and a chunk's writes land below every source of the later chunks: each chunk
+// loads all of its source rows, then stores them.  A warp covers 512 bytes per
+// pass: 512 / row_bytes rows side by side (row_bytes a multiple of 16, <= 512).
 __device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k, int row_bytes, int room, int lane)
 {
-    for (int j = 1; j < k; ++j) {
-        const int src = path[j];
-        if (src != j && src > j && src < room) {
-            const uint8_t *s = base + (size_t)src * row_bytes;
-            uint8_t *d = base + (size_t)j * row_bytes;
-            for (int off = lane * 16; off < row_bytes; off += 32 * 16)
-                *reinterpret_cast<uint4 *>(d + off) = *reinterpret_cast<const uint4 *>(s + off);
+    constexpr int kChunk = 8;
+    const int lanes_per_row = row_bytes >> 4;
+    const int rows_per_pass = 32 / lanes_per_row;
+    const int r_in = lane / lanes_per_row;
+    const int off = (lane - r_in * lanes_per_row) * 16;
+    for (int j0 = 1; j0 < k; j0 += kChunk) {
+        uint4 buf[kChunk];
+#pragma unroll
+        for (int m = 0; m < kChunk; ++m) {
+            const int j = j0 + r_in + m * rows_per_pass;
+            if (m * rows_per_pass < kChunk && j < k && j < j0 + kChunk) {
+                const int src = path[j];
+                if (src > j && src < room)
+                    buf[m] = *reinterpret_cast<const uint4 *>(base + (size_t)src * row_bytes + off);
+            }
+        }
+        __syncwarp();
+#pragma unroll
+        for (int m = 0; m < kChunk; ++m) {
+            const int j = j0 + r_in + m * rows_per_pass;
+            if (m * rows_per_pass < kChunk && j < k && j < j0 + kChunk) {
+                const int src = path[j];
+                if (src > j && src < room)
+                    *reinterpret_cast<uint4 *>(base + (size_t)j * row_bytes + off) = buf[m];
+            }
         }
         __syncwarp();
     }
