@@ -50,6 +50,8 @@ def _load():
             lib.oracle_typical_accept.argtypes = [P, i32, P, P, i32, d, d, d, P, P, P, P, P, P]
             lib.oracle_typical_accept.restype = ctypes.c_int
             lib.oracle_tempered_stats.argtypes = [P, i32, i32, d, P, P]
+            lib.oracle_spec_sample.argtypes = [P, i32, P, P, P, i32, d, P, P, P, P, P, P]
+            lib.oracle_spec_sample.restype = ctypes.c_int
             lib.oracle_rope.argtypes = [P, i32, i32, P, d, P]
             lib.oracle_rope.restype = ctypes.c_int
             lib.oracle_tree_attention_rope.argtypes = [P, P, P, i64, i32, i32, i32, i32, i32, P, d, P, P]
@@ -263,3 +265,34 @@ def tree_attention_rope(q, k, v, L: int, parent, base: float = 10000.0):
     if rc != 0:
         raise ValueError(f"oracle_tree_attention_rope rc={rc}")
     return out, k_rot
+
+
+# ---------------------------------------------------------------- speculative sampling (Sec. 2.1)
+
+def spec_sample(parent, draft, logits, q, temperature: float, unif, detail: bool = False):
+    """Speculative sampling on the tree: (accept_len, path, token[, detail]).
+
+    logits, q: float64 [N][V] (target logits per node; draft distribution of each
+    node's children); unif: [2N] uniforms in [0, 1) (unif[c] decides child c,
+    unif[N + u] draws the token after the final node u)."""
+    parent = np.ascontiguousarray(parent, dtype=np.int32)
+    draft = np.ascontiguousarray(draft, dtype=np.int32)
+    logits = np.ascontiguousarray(logits, dtype=np.float64)
+    q = np.ascontiguousarray(q, dtype=np.float64)
+    unif = np.ascontiguousarray(unif, dtype=np.float64)
+    n, V = logits.shape
+    if q.shape != logits.shape or len(unif) < 2 * n or len(parent) != n:
+        raise ValueError("shapes")
+    path = np.zeros(max(n, 1), dtype=np.int32)
+    alen = np.zeros(1, dtype=np.int32)
+    tok = np.zeros(1, dtype=np.int32)
+    rm = np.zeros(n)
+    cm = np.zeros(1)
+    if _load().oracle_spec_sample(_ptr(parent), n, _ptr(draft), _ptr(logits), _ptr(q), V, temperature, _ptr(unif),
+                                  _ptr(alen), _ptr(path), _ptr(tok), _ptr(rm), _ptr(cm)) != 0:
+        raise ValueError("bad tree, vocab or temperature")
+    k = int(alen[0])
+    out = (k, [int(x) for x in path[:k]], int(tok[0]))
+    if detail:
+        return out + ({"ratio_margin": rm, "cdf_margin": float(cm[0])},)
+    return out

@@ -506,3 +506,114 @@ int oracle_tree_attention_rope(const uint16_t *q, const uint16_t *k, const uint1
     }
     return 0;
 }
+
+/*
+ * Speculative sampling on a draft tree.  The rule of Sec. 2.1 (tokens accepted
+ * left to right with probability min(1, p(t) / q(t)); at the first rejection
+ * the replacement is drawn from norm(max(0, p - q))) applied at every node to
+ * its children in increasing id order, the residual replacing the target after
+ * each rejected sibling (the multi-candidate form of the rule):
+ *   - target p_u = softmax(z_u / T) for every node u;
+ *   - q_u [V]: the draft distribution the children of u were drawn from;
+ *   - at node u with residual r (= p_u on arrival), child c with token t_c is
+ *     accepted when unif[c] < r(t_c) / q_u(t_c) (q_u(t_c) = 0: accepted when
+ *     r(t_c) > 0); the walk moves to c;
+ *   - on rejection r <- max(0, r - q_u) / sum_v max(0, r(v) - q_u(v)) and the
+ *     next child is tried;
+ *   - when no child of u is accepted (or u is a leaf) the walk stops: the
+ *     token after u is drawn from r by inverse CDF: the smallest v with
+ *     sum_{w <= v} r(w) > unif[N + u].
+ * accept_len = depth(u) + 1, path = root .. u, token = the drawn token.
+ *   logits [N][V], q [N][V] (double); unif [2N]
+ *   ratio_margin[c] (NULL ok): r(t_c) / q_u(t_c) - unif[c] for the children tried, NAN otherwise
+ *   cdf_margin (NULL ok): distance of unif[N + u] to the nearest CDF value of r
+ * A draft token outside [0, V) has r = 0 and is rejected.
+ */
+int oracle_spec_sample(const int32_t *parent, int N, const int32_t *draft, const double *logits, const double *q,
+                       int V, double temperature, const double *unif, int32_t *accept_len, int32_t *path,
+                       int32_t *token, double *ratio_margin, double *cdf_margin)
+{
+    uint8_t in_anc[ORACLE_MAX_NODES * ORACLE_MAX_NODES];
+    int32_t depth[ORACLE_MAX_NODES];
+    if (oracle_tree(parent, N, depth, in_anc) != 0 || V < 1 || !(temperature > 0.0))
+        return -1;
+    double *r = (double *)malloc(sizeof(double) * (size_t)V);
+    if (!r)
+        return -2;
+    if (ratio_margin)
+        for (int j = 0; j < N; ++j)
+            ratio_margin[j] = NAN;
+    int u = 0;
+    for (;;) {
+        /* r = p_u */
+        const double *z = logits + (size_t)u * V;
+        double m = z[0];
+        for (int v = 1; v < V; ++v)
+            if (z[v] > m)
+                m = z[v];
+        double s = 0.0;
+        for (int v = 0; v < V; ++v) {
+            r[v] = exp((z[v] - m) / temperature);
+            s += r[v];
+        }
+        for (int v = 0; v < V; ++v)
+            r[v] /= s;
+        int next = -1;
+        const double *qu = q + (size_t)u * V;
+        for (int c = u + 1; c < N && next < 0; ++c) {
+            if (parent[c] != u)
+                continue;
+            const int t = draft[c];
+            const double rt = (t >= 0 && t < V) ? r[t] : 0.0;
+            const double qt = (t >= 0 && t < V) ? qu[t] : 0.0;
+            const double ratio = qt > 0.0 ? rt / qt : (rt > 0.0 ? INFINITY : 0.0);
+            if (ratio_margin)
+                ratio_margin[c] = ratio - unif[c];
+            if (unif[c] < ratio) {
+                next = c;
+                break;
+            }
+            /* rejected: residual */
+            double zr = 0.0;
+            for (int v = 0; v < V; ++v) {
+                r[v] = r[v] > qu[v] ? r[v] - qu[v] : 0.0;
+                zr += r[v];
+            }
+            if (zr > 0.0)
+                for (int v = 0; v < V; ++v)
+                    r[v] /= zr;
+        }
+        if (next < 0)
+            break;
+        u = next;
+    }
+    /* inverse CDF at u */
+    const double x = unif[N + u];
+    double cum = 0.0, best = INFINITY;
+    int tok = V - 1;
+    for (int v = 0; v < V; ++v) {
+        const double before = cum;
+        cum += r[v];
+        const double dist = fabs(cum - x);
+        if (dist < best && r[v] > 0.0)
+            best = dist;
+        if (cum > x && before <= x) {
+            tok = v;
+            const double d0 = fabs(before - x);
+            if (d0 < best)
+                best = d0;
+            break;
+        }
+    }
+    if (cdf_margin)
+        *cdf_margin = best;
+    const int len = depth[u] + 1;
+    for (int j = u, pos = len - 1; pos >= 0; --pos) {
+        path[pos] = j;
+        j = (j == 0) ? -1 : parent[j];
+    }
+    *accept_len = len;
+    *token = tok;
+    free(r);
+    return 0;
+}
