@@ -145,6 +145,8 @@ def kernel_source_hash(files: str) -> str:
 def acceptance_label(args) -> str:
     if getattr(args, "accept", "greedy") == "typical":
         return "typical (T=0.7, eps=0.09, alpha=0.3)"
+    if getattr(args, "accept", "greedy") == "sampled":
+        return "speculative sampling (T=0.7; drafts drawn from a synthetic head distribution)"
     return "greedy"
 
 
@@ -192,10 +194,27 @@ def run_gpu(args):
     drafts = torch.from_numpy(synth.gen_drafts(seed, sh.parent, am.cpu().numpy(), V, sh.p_match)).to(dev)
 
     typical = args.accept == "typical"
+    sampled = args.accept == "sampled"
     lz, et, dl = (torch.empty(N, dtype=torch.float32, device=dev) for _ in range(3))
+    if sampled:
+        # untimed: draft distributions = the target sharpened plus noise (a head that mostly
+        # agrees with the model), drafts drawn from them, seeded uniforms
+        g = torch.Generator(device=dev)
+        g.manual_seed(seed + 9)
+        zf = (hidden.float() @ W.float().t()) / 0.7
+        qd = torch.softmax(zf * 1.3 + 0.5 * torch.randn(zf.shape, generator=g, device=dev), dim=1).contiguous()
+        par = torch.from_numpy(np.asarray(sh.parent, np.int64)).to(dev)
+        drafts = torch.zeros(N, dtype=torch.int32, device=dev)
+        drafts[1:] = torch.multinomial(qd[par[1:]], 1, generator=g).squeeze(1).int()
+        unif = torch.rand(2 * N, generator=g, device=dev)
+        lgs = torch.empty((N + 1, V), dtype=torch.float32, device=dev)
+        del zf
 
     def step():
-        if typical:
+        if sampled:
+            tv.verify_step_sampled(bank, bid, kv, q, hidden, W, drafts, qd, unif, 0.7, out, am, t1, en, lgs, res, ws,
+                                   0, stream)
+        elif typical:
             tv.verify_step_typical(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, *tv.PAPER_TYPICAL,
                                    0, stream)
         else:
@@ -230,7 +249,7 @@ def run_gpu(args):
     torch.cuda._sleep(200_000_000)
     for i in range(n_k):
         ev[i][0].record(stream)
-        if typical:
+        if typical or sampled:
             tv.lm_head_stats_typical(bank, bid, hidden, W, tv.PAPER_TYPICAL[0], drafts, am, t1, en, lz, et, dl, ws,
                                      stream)
         else:
@@ -238,7 +257,9 @@ def run_gpu(args):
         ev[i][1].record(stream)
         tv.tree_attention(bank, bid, kv, q, out, ws, 0, nl, stream)
         ev[i][2].record(stream)
-        if typical:
+        if sampled:
+            tv.spec_sample_accept(bank, bid, drafts, lgs[:N], lz, qd, unif, L, 0.7, lgs[N], res, stream)
+        elif typical:
             tv.typical_accept(bank, bid, drafts, am, lz, et, dl, V, L, res, *tv.PAPER_TYPICAL, stream=stream)
         else:
             tv.greedy_accept(bank, bid, drafts, am, V, L, res, stream)
@@ -320,8 +341,9 @@ def run_gpu(args):
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         # per step: LM head, attention, split-unit merge (head_dim 128), acceptance + compaction
-        # (+ the rotary table and tree-key rotation with --rope)
-        "gpu_launches": ((4 if d == 128 else 3) + (2 if args.rope else 0)) * args.steps,
+        # (+ the rotary table and tree-key rotation with --rope; sampled: the walk, then compaction)
+        "gpu_launches": ((4 if d == 128 else 3) + (2 if args.rope else 0) + (1 if args.accept == "sampled" else 0))
+                        * args.steps,
         "clocks": clocks,
     }
     if args.layers:
@@ -828,11 +850,14 @@ def main(argv=None):
                     help="c1/c2/c4: pre-rotary inputs, rotary embedding applied by the library (head_dim 128)")
     ap.add_argument("--scheduled", action="store_true",
                     help="c3 only: the device-driven loop (tree and L on the device, CUDA-graph replay)")
-    ap.add_argument("--accept", default="greedy", choices=["greedy", "typical"],
-                    help="verification rule: greedy (default) or typical acceptance at T=0.7, eps=0.09, alpha=0.3")
+    ap.add_argument("--accept", default="greedy", choices=["greedy", "typical", "sampled"],
+                    help="verification rule: greedy (default), typical acceptance at T=0.7, eps=0.09, alpha=0.3, "
+                         "or speculative sampling at T=0.7")
     args = ap.parse_args(argv)
-    if args.accept == "typical" and (args.impl == "reference" or args.config in ("c3", "sweep")):
-        ap.error("--accept typical applies to the GPU arm of c1, c2, c4 and c5")
+    if args.accept != "greedy" and (args.impl == "reference" or args.config in ("c3", "sweep")):
+        ap.error("--accept typical / sampled apply to the GPU arm of c1, c2, c4 and c5")
+    if args.accept == "sampled" and args.config == "c5":
+        ap.error("--accept sampled runs one sequence per step (c1, c2, c4)")
     if args.scheduled and (args.config != "c3" or args.impl == "reference"):
         ap.error("--scheduled applies to the GPU arm of c3")
     if args.impl == "reference" and args.config == "sweep":

@@ -361,6 +361,45 @@ TB_API tb_status verify_step_batched_typical(const tb_bank *bank, int batch, con
                                              void *workspace, size_t workspace_bytes, int flags, tb_stream stream);
 
 /* ------------------------------------------------------------------------
+ * Speculative sampling: the stochastic verification rule of Sec. 2.1 (accept
+ * a drafted token t with probability min(1, p(t) / q(t)); at the first
+ * rejection draw the replacement from norm(max(0, p - q))), applied on the
+ * tree: at every node the children are tried in increasing canonical id
+ * order, the residual norm(max(0, r - q_u)) replacing the target r after each
+ * rejected sibling; the walk stops at the node none of whose children is
+ * accepted and the token after it is drawn from r by inverse CDF (the
+ * smallest v with sum_{w <= v} r(w) > uniforms[N + u] * sum_w r(w)).  The
+ * target at node u is p_u = softmax(z_u / T).  Lossless when the children of
+ * each node u are independent draws from q_u.
+ * ---------------------------------------------------------------------- */
+
+/* The walk alone, from the target logits:
+ *   draft_tokens int32 [N]; logits float [N][vocab]; logz_t float [N] =
+ *   ln sum_v e^(z_v / T) (lm_head_stats_typical); draft_probs float [N][vocab]:
+ *   row u = the distribution the children of u were drawn from (rows of
+ *   leaves unused); uniforms float [2N] in [0, 1): uniforms[c] decides child
+ *   c, uniforms[N + u] draws the token at the final node u; scratch float
+ *   [vocab].  All device memory.  *result: accept_len, path, bonus_token = the
+ *   drawn token, new_L = L + accept_len, status (a draft token outside
+ *   [0, vocab) is never accepted and sets TB_EINVAL).  One CTA. */
+TB_API tb_status spec_sample_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens, const float *logits,
+                                    const float *logz_t, const float *draft_probs, const float *uniforms, int vocab,
+                                    int L, float temperature, float *scratch, tb_result *result, tb_stream stream);
+
+/* One verification step with speculative sampling: tree_attention, the LM
+ * head (greedy statistics, tempered log-partition, and the logits of every
+ * node written to logits[0 .. N) -- the sampling needs whole rows), the walk
+ * (scratch: logits row N), then (unless TB_NO_COMPACT) kv_compact.
+ *   logits float [N + 1][vocab] (device scratch written by the call);
+ *   draft_probs, uniforms as for spec_sample_accept; the rest as verify_step. */
+TB_API tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q,
+                                     int n_q_heads, const void *hidden, const void *lm_head, int d_model, int vocab,
+                                     const int32_t *draft_tokens, const float *draft_probs, const float *uniforms,
+                                     float temperature, void *attn_out, int32_t *argmax, float *top1, float *entropy,
+                                     float *logits, tb_result *result, void *workspace, size_t workspace_bytes,
+                                     int flags, tb_stream stream);
+
+/* ------------------------------------------------------------------------
  * Device-driven decode loop: the per-step tree selection of Sec. 4 ("Policy",
  * "Cost") taken on the GPU.  The prefix length and the tree of the next step
  * live in device memory (tb_state); the acceptance kernel's last CTA updates

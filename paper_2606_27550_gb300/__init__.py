@@ -32,7 +32,7 @@ API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb
        "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error",
        "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
        "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical",
-       "verify_step_scheduled")
+       "verify_step_scheduled", "spec_sample_accept", "verify_step_sampled")
 
 
 class TreeVerifyError(RuntimeError):
@@ -109,6 +109,9 @@ def load(path: str = LIB_PATH):
         "verify_step_typical": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, P, sz, i32, P],
         "verify_step_batched_typical": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, P, sz, i32, P],
         "verify_step_scheduled": [P, P, P, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
+        "spec_sample_accept": [P, i32, P, P, P, P, P, i32, i32, ctypes.c_float, P, P, P],
+        "verify_step_sampled": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, ctypes.c_float, P, P, P, P, P, P, P, sz,
+                                i32, P],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
@@ -376,6 +379,29 @@ def verify_step_batched_typical(bank: Bank, seqs, hidden, lm_head, argmax, top1,
                                               _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(argmax),
                                               _ptr(top1), _ptr(entropy), ctypes.byref(t), _ptr(ws), ws.numel(),
                                               flags, _stream(stream)), "verify_step_batched_typical")
+
+
+# --------------------------------------------------------------------- speculative sampling
+
+
+def spec_sample_accept(bank: Bank, bank_id: int, draft, logits, logz_t, draft_probs, uniforms, L: int,
+                       temperature: float, scratch, result, stream=None):
+    """logits, draft_probs float [N][V]; logz_t [N]; uniforms [2N]; scratch [V]."""
+    _check(load().spec_sample_accept(bank.handle, bank_id, _ptr(draft), _ptr(logits), _ptr(logz_t),
+                                     _ptr(draft_probs), _ptr(uniforms), logits.shape[1], L, float(temperature),
+                                     _ptr(scratch), _ptr(result), _stream(stream)), "spec_sample_accept")
+
+
+def verify_step_sampled(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft, draft_probs, uniforms,
+                        temperature: float, attn_out, argmax, top1, entropy, logits, result, ws, flags: int = 0,
+                        stream=None):
+    """logits: float [N + 1][V] scratch (rows 0..N-1 receive the target logits)."""
+    c = kv.as_c()
+    _check(load().verify_step_sampled(bank.handle, bank_id, ctypes.byref(c), _ptr(q), q.shape[2], _ptr(hidden),
+                                      _ptr(lm_head), hidden.shape[1], lm_head.shape[0], _ptr(draft),
+                                      _ptr(draft_probs), _ptr(uniforms), float(temperature), _ptr(attn_out),
+                                      _ptr(argmax), _ptr(top1), _ptr(entropy), _ptr(logits), _ptr(result), _ptr(ws),
+                                      ws.numel(), flags, _stream(stream)), "verify_step_sampled")
 
 
 # --------------------------------------------------------------------- device-driven loop

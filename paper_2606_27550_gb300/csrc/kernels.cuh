@@ -30,6 +30,7 @@ struct LmTypical {
     float *logz_t;
     float *ent_t;
     LmGather gather;
+    float *logits_out;  // null, or [R][V] fp32: the logits themselves (speculative sampling needs whole rows)
 };
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
@@ -141,6 +142,22 @@ struct AcceptParams {
 };
 cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
 cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream);
+
+// speculative sampling on the tree (sample.cu): one CTA walks the tree
+struct SampleParams {
+    const TreeDesc *tree;
+    const int32_t *draft;
+    const float *logits;  // [N][V]
+    const float *logz_t;  // [N]: ln sum_v e^(z_v / T)
+    const float *q;       // [N][V]: the draft distribution of each node's children
+    const float *unif;    // [2N]
+    float *resid;         // [V] scratch
+    int V, L;
+    float inv_t;
+    tb_result *result;
+    const int *ws_status;  // may be null
+};
+cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once
 // per (kernel, device) (treeverify.cu).

@@ -54,6 +54,7 @@ struct LmParams {
     float *logz_t;        // [R] m / T + ln sT
     float *ent_t;         // [R] ln sT - tT / sT
     LmGather gather;
+    float *logits_out;    // typical mode, optional: [R][V] fp32 logits
 };
 
 struct RowStat {
@@ -406,6 +407,14 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
             }
         }
         if constexpr (kTyp) {
+            if (p.logits_out) {
+                // whole logit rows for speculative sampling: 128 consecutive floats per row
+                for (int e = threadIdx.x; e < p.R * 128; e += blockDim.x) {
+                    const int r = e >> 7, j = e & 127;
+                    if (j < nvalid)
+                        p.logits_out[(size_t)r * p.V + v0 + j] = logits[r * ld + j];
+                }
+            }
             const int nhit = s_nhit;
             if (nhit <= kHitCap) {
                 for (int i = threadIdx.x; i < nhit; i += blockDim.x) {
@@ -547,6 +556,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         p.logz_t = typ->logz_t;
         p.ent_t = typ->ent_t;
         p.gather = typ->gather;
+        p.logits_out = typ->logits_out;
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
         if (e != cudaSuccess)
             return e;

@@ -830,6 +830,119 @@ extern "C" tb_status typical_accept(const tb_bank *bank, int bank_id, const int3
     return ok();
 }
 
+static tb_status sample_enqueue(const tb_bank *bank, int bank_id, const int32_t *draft, const float *logits,
+                                const float *logz_t, const float *q, const float *unif, int vocab, int L,
+                                float temperature, float *scratch, tb_result *result, const int *ws_status,
+                                cudaStream_t s, const char *fn)
+{
+    SampleParams sp{};
+    sp.tree = bank->d_desc + bank_id;
+    sp.draft = draft;
+    sp.logits = logits;
+    sp.logz_t = logz_t;
+    sp.q = q;
+    sp.unif = unif;
+    sp.resid = scratch;
+    sp.V = vocab;
+    sp.L = L;
+    sp.inv_t = 1.0f / temperature;
+    sp.result = result;
+    sp.ws_status = ws_status;
+    cudaError_t e = sample_launch(sp, s);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
+    return TB_OK;
+}
+
+extern "C" tb_status spec_sample_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens,
+                                        const float *logits, const float *logz_t, const float *draft_probs,
+                                        const float *uniforms, int vocab, int L, float temperature, float *scratch,
+                                        tb_result *result, tb_stream stream)
+{
+    const char *fn = "spec_sample_accept";
+    tb_status st = check_bank(bank, bank_id, fn);
+    if (st != TB_OK)
+        return st;
+    if (!draft_tokens || !logits || !logz_t || !draft_probs || !uniforms || !scratch || !result)
+        return fail(TB_EINVAL, "%s: NULL argument", fn);
+    if (vocab < 1 || L < 0)
+        return fail(TB_EINVAL, "%s: vocab=%d L=%d", fn, vocab, L);
+    const tb_typical t{temperature, 0.f, 0.f, 0};
+    if ((st = check_typical(&t, fn)) != TB_OK)
+        return st;
+    if ((st = sample_enqueue(bank, bank_id, draft_tokens, logits, logz_t, draft_probs, uniforms, vocab, L,
+                             temperature, scratch, result, nullptr, (cudaStream_t)stream, fn)) != TB_OK)
+        return st;
+    return ok();
+}
+
+extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const tb_kv *kv, const void *q,
+                                         int n_q_heads, const void *hidden, const void *lm_head, int d_model,
+                                         int vocab, const int32_t *draft_tokens, const float *draft_probs,
+                                         const float *uniforms, float temperature, void *attn_out, int32_t *argmax,
+                                         float *top1, float *entropy, float *logits, tb_result *result,
+                                         void *workspace, size_t workspace_bytes, int flags, tb_stream stream)
+{
+    const char *fn = "verify_step_sampled";
+    AttnArgs a{bank, bank_id, kv, 0, kv ? kv->n_layers : 0, q, n_q_heads, attn_out};
+    AttnPlan aplan;
+    tb_status st = attn_validate(a, fn, &aplan);
+    if (st != TB_OK)
+        return st;
+    const int N = bank->h_desc[bank_id].n;
+    LmPlan lplan;
+    if ((st = lm_validate(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
+        return st;
+    if (!draft_tokens || !draft_probs || !uniforms || !logits || !result)
+        return fail(TB_EINVAL, "%s: NULL draft_tokens / draft_probs / uniforms / logits / result", fn);
+    const tb_typical tt{temperature, 0.f, 0.f, 0};
+    if ((st = check_typical(&tt, fn)) != TB_OK)
+        return st;
+    const size_t attn_bytes = attn_part_bytes(sm_count(bank->device), kv->head_dim);
+    if ((st = check_ws(workspace, workspace_bytes, kPartBase + attn_bytes + lplan.ws_bytes, fn)) != TB_OK)
+        return st;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    cudaStream_t s = (cudaStream_t)stream;
+    const TypRows tr = typ_rows(ws);
+    LmTypical lt{};
+    lt.temperature = temperature;
+    lt.logz_t = tr.logz_t;
+    lt.ent_t = tr.ent_t;
+    lt.logits_out = logits;
+    {
+        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
+        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step_sampled: fork");
+        if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+            return st;
+        if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                             bank->aux, fn, 0, &lt)) != TB_OK)
+            return st;
+        e = cudaEventRecord(bank->ev_join, bank->aux);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
+        if (e != cudaSuccess)
+            return cuda_fail(e, "verify_step_sampled: join");
+    }
+    if ((st = sample_enqueue(bank, bank_id, draft_tokens, logits, tr.logz_t, draft_probs, uniforms, vocab, kv->L,
+                             temperature, logits + (size_t)N * vocab, result, reinterpret_cast<const int *>(ws), s,
+                             fn)) != TB_OK)
+        return st;
+    if (!(flags & TB_NO_COMPACT)) {
+        AcceptParams p{};
+        p.result = result;
+        p.from_result = 1;
+        add_compaction(p, kv);
+        cudaError_t e = accept_launch(p, sm_count(bank->device), s);
+        if (e != cudaSuccess)
+            return cuda_fail(e, fn);
+    }
+    return ok();
+}
+
 extern "C" tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream)
 {
     const char *fn = "kv_compact";
