@@ -163,9 +163,25 @@ template <bool kTyp>
 __device__ void merge_partials(const LmParams &p, const float4 *src, const float2 *src_t, int count, float4 *sbuf,
                                float4 *dst, float2 *dst_t)
 {
+    // staging with eight loads in flight per thread: the partials are in L2,
+    // and a load-then-store loop would pay one round trip per element
+    constexpr int kInFlight = 8;
     const int n = count * p.R_pad;
-    for (int i = threadIdx.x; i < n; i += blockDim.x)
-        sbuf[i] = __ldcg(src + i);
+    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kInFlight) {
+        float4 v[kInFlight];
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            const int i = i0 + u * (int)blockDim.x;
+            if (i < n)
+                v[u] = __ldcg(src + i);
+        }
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            const int i = i0 + u * (int)blockDim.x;
+            if (i < n)
+                sbuf[i] = v[u];
+        }
+    }
     __syncthreads();
     const int tpr = threads_per_row(p.R_pad);
     const int sub = threadIdx.x % tpr;
@@ -182,20 +198,33 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
                 }
             }
             if (st.idx != 0x7fffffff) {
-                for (int k = sub; k < count; k += tpr) {
-                    const float4 v = sbuf[k * p.R_pad + r];
-                    if (v.z > 0.f) {
-                        const float delta = v.x - st.m;
-                        const float e = ex2_approx(delta * kLog2e);
-                        st.s += v.z * e;
-                        st.t += (v.w + delta * v.z) * e;
-                        if constexpr (kTyp) {
-                            // the tempered sums are read once, straight from L2
-                            const float2 w = __ldcg(src_t + (size_t)k * p.R_pad + r);
-                            const float dT = delta * p.inv_t;
-                            const float eT = ex2_approx(dT * kLog2e);
-                            st.sT += w.x * eT;
-                            st.tT += (w.y + dT * w.x) * eT;
+                for (int k0 = sub; k0 < count; k0 += tpr * kInFlight) {
+                    // the tempered sums are read once, straight from L2, eight at a time
+                    float2 w[kInFlight];
+                    if constexpr (kTyp) {
+#pragma unroll
+                        for (int u = 0; u < kInFlight; ++u) {
+                            const int k = k0 + u * tpr;
+                            w[u] = k < count ? __ldcg(src_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < kInFlight; ++u) {
+                        const int k = k0 + u * tpr;
+                        if (k >= count)
+                            break;
+                        const float4 v = sbuf[k * p.R_pad + r];
+                        if (v.z > 0.f) {
+                            const float delta = v.x - st.m;
+                            const float e = ex2_approx(delta * kLog2e);
+                            st.s += v.z * e;
+                            st.t += (v.w + delta * v.z) * e;
+                            if constexpr (kTyp) {
+                                const float dT = delta * p.inv_t;
+                                const float eT = ex2_approx(dT * kLog2e);
+                                st.sT += w[u].x * eT;
+                                st.tT += (w[u].y + dT * w[u].x) * eT;
+                            }
                         }
                     }
                 }
