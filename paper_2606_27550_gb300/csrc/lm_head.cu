@@ -13,8 +13,9 @@
 // N = R_pad B operand.  tcgen05.mma (kind::f16, f32 accumulate) builds the
 // 128 x R_pad logit tile in TMEM over d_model/64 k-blocks fed by a multi-stage
 // TMA ring.  Warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, then all
-// four warps read TMEM (lane = vocab entry), transpose through shared memory
-// and reduce each row.  Per-tile statistics are merged in two levels by
+// eight warps read TMEM (lane = vocab entry; two warps per lane quadrant, each
+// taking half of the columns), transpose through shared memory and reduce
+// each row.  Per-tile statistics are merged in two levels by
 // atomic arrival tickets (the last CTA of a group merges the group; the last
 // group merges everything); no CTA ever waits for another.
 //
@@ -67,6 +68,11 @@ struct RowStat {
 };
 
 constexpr float kLog2e = 1.4426950408889634f;
+
+// Threads per CTA: warp 0 lane 0 issues TMA, warp 1 lane 0 the MMAs; all eight
+// warps then share the epilogue (warps w and w + 4 read the same TMEM lane
+// quadrant and split its columns) and the per-row scans.
+constexpr int kLmThreads = 256;
 
 __device__ __forceinline__ RowStat stat_empty()
 {
@@ -122,12 +128,13 @@ __device__ __forceinline__ RowStat stat_unpack(float4 v)
     return RowStat{v.x, __float_as_int(v.y), v.z, v.w, 0.f, 0.f};
 }
 
-// Threads per row for per-row scans by the 128 threads of a CTA: the largest
-// power of two with tpr x R_pad <= 128 (at least 1).
+// Threads per row for per-row scans by the CTA's threads: the largest power
+// of two with tpr x R_pad <= blockDim.x, at most 8 (the transposed tile's row
+// stride 128 + tpr is sized for 8).
 __device__ __forceinline__ int threads_per_row(int R_pad)
 {
     int tpr = 1;
-    while (tpr * 2 * R_pad <= 128)
+    while (tpr < 8 && tpr * 2 * R_pad <= (int)blockDim.x)
         tpr *= 2;
     return tpr;
 }
@@ -185,7 +192,7 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
     __syncthreads();
     const int tpr = threads_per_row(p.R_pad);
     const int sub = threadIdx.x % tpr;
-    for (int r0 = 0; r0 < p.R; r0 += 128 / tpr) {
+    for (int r0 = 0; r0 < p.R; r0 += (int)blockDim.x / tpr) {
         const int r = r0 + threadIdx.x / tpr;
         RowStat st = stat_empty();
         if (r < p.R) {
@@ -252,7 +259,7 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
 }
 
 template <bool kTyp>
-__global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmParams p)
+__global__ void __launch_bounds__(kLmThreads, 1) k2_lm_head(const __grid_constant__ LmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[8];
@@ -354,10 +361,11 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
         }
         tc_commit(&acc_bar);
     } else if (kTyp && warp >= 2) {
-        // ---------------- edges to gather (warps 2-3 are otherwise idle here)
+        // ---------------- edges to gather (warps 2.. are otherwise idle here)
         const int nvalid = min(128, p.V - v0);
+        const int helpers = (int)blockDim.x - 64;
         for (int b = 0; b < p.gather.n_seq; ++b) {
-            for (int j = 1 + (threadIdx.x - 64); j < p.gather.seq[b].n; j += 64) {
+            for (int j = 1 + (threadIdx.x - 64); j < p.gather.seq[b].n; j += helpers) {
                 int row, col;
                 if (gather_hit(p.gather, b, j, p.R, v0, nvalid, &row, &col)) {
                     const int slot = atomicAdd(&s_nhit, 1);
@@ -380,14 +388,17 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     const int ld = 128 + tpr;
     float *logits = reinterpret_cast<float *>(smem);  // aliases the drained ring
     if (ok) {
-        const uint32_t row_addr = tmem + ((uint32_t)(32 * warp) << 16);
-        for (int c0 = 0; c0 < p.R_pad; c0 += 16) {
+        // warps w and w + 4 read TMEM lane quadrant w % 4 (vocab rows 32 (w % 4) ..)
+        // and split the columns (tree rows) in alternate 16-column chunks
+        const int quad = warp & 3, half = warp >> 2, halves = (int)blockDim.x >> 7;
+        const uint32_t row_addr = tmem + ((uint32_t)(32 * quad) << 16);
+        for (int c0 = 16 * half; c0 < p.R_pad; c0 += 16 * halves) {
             uint32_t r[16];
             tmem_ld_32x32b_x16(row_addr + (uint32_t)c0, r);
             tmem_ld_wait();
 #pragma unroll
             for (int j = 0; j < 16; ++j)
-                logits[(c0 + j) * ld + 32 * warp + lane] = __uint_as_float(r[j]);
+                logits[(c0 + j) * ld + 32 * quad + lane] = __uint_as_float(r[j]);
         }
     } else if (warp == 1 && lane == 0) {
         mbar_wait_drain(&acc_bar, 0);  // MMAs issued before giving up must finish before dealloc
@@ -403,7 +414,7 @@ __global__ void __launch_bounds__(128, 1) k2_lm_head(const __grid_constant__ LmP
     {
         const int sub = threadIdx.x % tpr;
         const int nvalid = min(128, p.V - v0);
-        for (int r0 = 0; r0 < p.R; r0 += 128 / tpr) {
+        for (int r0 = 0; r0 < p.R; r0 += (int)blockDim.x / tpr) {
             const int r = r0 + threadIdx.x / tpr;
             RowStat st = stat_empty();
             if (r < p.R) {
@@ -589,13 +600,13 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
         if (e != cudaSuccess)
             return e;
-        k2_lm_head<true><<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+        k2_lm_head<true><<<pl.n_tiles, kLmThreads, pl.smem_bytes, stream>>>(p);
     } else {
         p.inv_t = 1.0f;
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
         if (e != cudaSuccess)
             return e;
-        k2_lm_head<false><<<pl.n_tiles, 128, pl.smem_bytes, stream>>>(p);
+        k2_lm_head<false><<<pl.n_tiles, kLmThreads, pl.smem_bytes, stream>>>(p);
     }
     return cudaGetLastError();
 }
