@@ -105,7 +105,8 @@ def test_tree_attention_large_L_multilayer(dev, bank):
     _run_attention(bank, dev, synth.bank_trees()[-1], 5000, 3, 8, 8, 128, seed=4)
 
 
-LM_CASES = [(1, 256, 1000), (7, 256, 1000), (26, 4096, 4099), (64, 4096, 32000), (200, 512, 3000), (256, 256, 129)]
+LM_CASES = [(1, 256, 1000), (7, 256, 1000), (26, 4096, 4099), (64, 4096, 32000), (200, 512, 3000), (256, 256, 129),
+            (232, 256, 4099)]
 
 
 @pytest.mark.parametrize("R,D,V", LM_CASES)
