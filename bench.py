@@ -210,15 +210,16 @@ def run_gpu(args):
         lgs = torch.empty((N + 1, V), dtype=torch.float32, device=dev)
         del zf
 
-    def step():
+    def step(qq=q, hh=hidden, dd=drafts, st=None):
+        st = stream if st is None else st
         if sampled:
-            tv.verify_step_sampled(bank, bid, kv, q, hidden, W, drafts, qd, unif, 0.7, out, am, t1, en, lgs, res, ws,
-                                   0, stream)
+            tv.verify_step_sampled(bank, bid, kv, qq, hh, W, dd, qd, unif, 0.7, out, am, t1, en, lgs, res, ws,
+                                   0, st)
         elif typical:
-            tv.verify_step_typical(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, *tv.PAPER_TYPICAL,
-                                   0, stream)
+            tv.verify_step_typical(bank, bid, kv, qq, hh, W, dd, out, am, t1, en, res, ws, *tv.PAPER_TYPICAL,
+                                   0, st)
         else:
-            tv.verify_step(bank, bid, kv, q, hidden, W, drafts, out, am, t1, en, res, ws, 0, stream)
+            tv.verify_step(bank, bid, kv, qq, hh, W, dd, out, am, t1, en, res, ws, 0, st)
 
     visible = os.environ.get("CUDA_VISIBLE_DEVICES")
     sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
@@ -270,7 +271,11 @@ def run_gpu(args):
     t_at = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
     t_ac = statistics.mean(e[2].elapsed_time(e[3]) for e in ev)
 
-    # end to end: per step, pinned host -> device inputs, verify_step, device -> host result, host sync
+    # end to end: every step copies its inputs from pinned host memory and reads its result
+    # back with a host synchronisation.  Inputs are double-buffered: step i + 1's copy runs on
+    # a copy stream while step i computes (events keep a buffer from being overwritten while
+    # a step still reads it); each buffer's verify_step call is captured once into a CUDA
+    # graph, so the host enqueues one replay per step.
     q_h = torch.empty(q.shape, dtype=bf, pin_memory=True).copy_(q)
     h_h = torch.empty(hidden.shape, dtype=bf, pin_memory=True).copy_(hidden)
     d_h = torch.empty(drafts.shape, dtype=torch.int32, pin_memory=True).copy_(drafts)
@@ -278,16 +283,43 @@ def run_gpu(args):
     stats_h = torch.empty((3, N), dtype=torch.float32, pin_memory=True)
     h2d = q_h.numel() * 2 + h_h.numel() * 2 + d_h.numel() * 4
     d2h = res_h.numel() * 4 + stats_h.numel() * 4
+    bufs = [(q, hidden, drafts), (torch.empty_like(q), torch.empty_like(hidden), torch.empty_like(drafts))]
+    copy_stream = torch.cuda.Stream()
+    ev_copied = [torch.cuda.Event(), torch.cuda.Event()]
+    ev_used = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def upload(b):
+        copy_stream.wait_event(ev_used[b])  # the step that last read these buffers is done
+        with torch.cuda.stream(copy_stream):
+            bufs[b][0].copy_(q_h, non_blocking=True)
+            bufs[b][1].copy_(h_h, non_blocking=True)
+            bufs[b][2].copy_(d_h, non_blocking=True)
+            ev_copied[b].record(copy_stream)
+
     n_e2e = max(3, min(args.steps, 50))
+    graphs = []
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    for b in range(2):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap):
+            step(*bufs[b], st=cap)
+        graphs.append(g)
+    torch.cuda.synchronize()
+    for b in range(2):
+        ev_used[b].record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     t0 = time.perf_counter()
-    for _ in range(n_e2e):
-        q.copy_(q_h, non_blocking=True)
-        hidden.copy_(h_h, non_blocking=True)
-        drafts.copy_(d_h, non_blocking=True)
-        step()
+    upload(0)
+    for i in range(n_e2e):
+        b = i % 2
+        if i + 1 < n_e2e:
+            upload(1 - b)
+        stream.wait_event(ev_copied[b])
+        graphs[b].replay()
+        ev_used[b].record(stream)
         res_h.copy_(res, non_blocking=True)
         stats_h[0].copy_(am.view(torch.float32), non_blocking=True)
         stats_h[1].copy_(t1, non_blocking=True)
