@@ -39,6 +39,7 @@ import numpy as np  # noqa: E402
 from paper_2606_27550_gb300 import synth  # noqa: E402
 
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+NOMINAL_HBM_GBS = 8000.0  # nominal HBM3e bandwidth, for context beside the measured copy peak
 
 
 def load_peaks():
@@ -362,7 +363,14 @@ def run_gpu(args):
         "tree_tokens_per_s": round(value * N, 1),
         "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
                          "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
-                         "peak_gbs": hbm, "peak_src": peak_src},
+                         "peak_gbs": hbm, "peak_src": peak_src,
+                         "frac_nominal": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
+                         "nominal_gbs": NOMINAL_HBM_GBS},
+        "compute_roofline": {"flops_per_step": flops,
+                             "t_ms": round(flops / (float(peaks.get("bf16_tflops_sustained", 1713.0)) * 1e12) * 1e3, 4),
+                             "frac": round(flops / (float(peaks.get("bf16_tflops_sustained", 1713.0)) * 1e12)
+                                           / (ms * 1e-3), 4),
+                             "peak_tflops": float(peaks.get("bf16_tflops_sustained", 1713.0))},
         "roofline": {"kernel": k1_name, "bound": "hbm", "achieved": round(at_gbs, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(at_gbs / hbm, 4), "traffic": traffic_from_profiles(k1_name),
                      "algorithmic_bytes": kv_bytes, "avg_launch_ms": round(t_at, 4)},
@@ -817,16 +825,43 @@ def cpu_sample_step(cfg: str, attn_units: int, vocab_slices: int, seed: int = 0)
     return full, sample, t_attn + t_lm
 
 
+def cpu_model() -> str:
+    try:
+        for ln in open("/proc/cpuinfo"):
+            key = ln.split(":")[0].strip().lower()
+            if key in ("model name", "cpu model", "hardware"):
+                return ln.split(":", 1)[1].strip()
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+
+    return platform.processor() or platform.machine()
+
+
 def cpu_baseline(cfg: str, budget_s: float = 20.0):
-    """The oracle timed on this host's cores on a bounded sample of the workload."""
+    """The oracle timed on this host's cores on a bounded sample of the workload (all
+    cores, and one thread on a smaller sample)."""
     import oracle
 
     oracle.build()
     _, _, probe = cpu_sample_step(cfg, 1, 1)
     n = int(max(1, min(64, budget_s / max(probe, 1e-6))))
-    full, sample, _ = cpu_sample_step(cfg, n, n, seed=1)
-    return {"value": round(1.0 / full, 6), "unit": "verify-steps/s", "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": sample, "s_per_full_step": round(full, 3)}
+    sh, _, _, _ = workload(cfg)
+    full, sample, _ = cpu_sample_step(cfg, min(n, sh.n_layers * sh.n_kv_heads), min(n, 32), seed=1)
+    cores = oracle.num_threads()
+    prev = oracle.set_num_threads(1)
+    try:
+        full1, sample1, _ = cpu_sample_step(cfg, 1, 1, seed=2)
+    finally:
+        oracle.set_num_threads(prev)
+    return {"value": round(1.0 / full, 6), "unit": "verify-steps/s", "cores": cores, "kind": "oracle",
+            "sample": sample, "s_per_full_step": round(full, 3),
+            "single_thread": {"value": round(1.0 / full1, 7), "s_per_full_step": round(full1, 2), "sample": sample1},
+            "nproc": os.cpu_count(), "cpu_model": cpu_model()}
 
 
 def run_reference(args):

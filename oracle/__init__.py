@@ -46,6 +46,8 @@ def _load():
             lib.oracle_lm_head.argtypes = [P, P, i32, i32, i32, P, P, P, P, P]
             lib.oracle_accept.argtypes = [P, i32, P, P, P, P, P]
             lib.oracle_num_threads.argtypes = []
+            lib.oracle_set_num_threads.argtypes = [i32]
+            lib.oracle_set_num_threads.restype = ctypes.c_int
             d = ctypes.c_double
             lib.oracle_typical_accept.argtypes = [P, i32, P, P, i32, d, d, d, P, P, P, P, P, P]
             lib.oracle_typical_accept.restype = ctypes.c_int
@@ -70,6 +72,11 @@ def _ptr(a: np.ndarray):
 
 def num_threads() -> int:
     return int(_load().oracle_num_threads())
+
+
+def set_num_threads(n: int) -> int:
+    """Threads of the oracle's OpenMP loops from now on; returns the previous count."""
+    return int(_load().oracle_set_num_threads(int(n)))
 
 
 def tree(parent):

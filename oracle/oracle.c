@@ -60,6 +60,17 @@ int oracle_num_threads(void)
 #endif
 }
 
+/* Threads of the OpenMP loops that follow (n >= 1); returns the previous count. */
+int oracle_set_num_threads(int n)
+{
+    const int prev = oracle_num_threads();
+#ifdef _OPENMP
+    if (n >= 1)
+        omp_set_num_threads(n);
+#endif
+    return prev;
+}
+
 /*
  * Tree bookkeeping.  in_anc[i * n + j] = 1 when j is i or an ancestor of i.
  * depth[i] = number of edges from the root.  Returns 0, or -1 when parent[]
