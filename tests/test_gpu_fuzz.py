@@ -1,0 +1,149 @@
+"""Randomised verification steps against the fp64 oracle: random trees (in
+and out of breadth-first order), prefix lengths (including 0), head_dim 64
+and 128, GQA groups, d_model not a multiple of 64, vocabularies from 1 token
+up, single and batched steps.  Same tolerances as the other parity tests."""
+import numpy as np
+import pytest
+
+import oracle
+from helpers import STAT_TOL, bits, check_attention, to_dev
+from paper_2606_27550_gb300 import synth
+
+torch = pytest.importorskip("torch")
+tv = pytest.importorskip("paper_2606_27550_gb300")
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    from paper_2606_27550_gb300 import build
+
+    build.build()
+    torch.cuda.set_device(0)
+    return torch.device("cuda:0")
+
+
+def _hidden(g, n, W, gap_min=1e-2):
+    """n hidden rows with a clear top-2 gap (V = 1 has a single token: no gap to keep)."""
+    D, V = W.shape[1], W.shape[0]
+    for _ in range(20):
+        pool = synth.normal_bf16(g, (n + 16, D))
+        am, t1, en, gap = oracle.lm_head(pool, W)
+        keep = np.arange(len(gap)) if V == 1 else np.nonzero(gap > gap_min)[0]
+        if len(keep) >= n:
+            keep = keep[:n]
+            return pool[keep], am[keep], t1[keep], en[keep]
+    raise RuntimeError("no rows with a clear gap")
+
+
+def _random_case(g):
+    n = int(g.integers(1, 65))
+    bfs = g.random() < 0.5
+    parent = synth.random_tree(g, n)
+    if bfs:
+        parent = np.sort(parent)
+        parent[0] = -1
+    d = int(g.choice([64, 128]))
+    Hkv = int(g.choice([1, 2, 4]))
+    group = int(g.choice([1, 2, 4]))
+    while n * group > 256:
+        group //= 2
+    Hq = Hkv * max(group, 1)
+    L = int(g.choice([0, 1, 63, 128, 300, 1000, 2500]))
+    D = int(g.choice([64, 200, 256, 520]))
+    V = int(g.choice([1, 2, 127, 128, 129, 1000, 3001]))
+    return parent, bfs, d, Hkv, Hq, L, D, V
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_random_verify_step(dev, seed):
+    g = synth.rng(9000 + seed)
+    parent, bfs, d, Hkv, Hq, L, D, V = _random_case(g)
+    b = tv.Bank(4, 0)
+    bid, order = b.add(parent)
+    # the library canonicalises: per-node inputs follow its breadth-first order
+    canon = np.asarray(b.get(bid)[0], np.int32)
+    N = len(canon)
+    layers = int(g.integers(1, 3))
+    k, v = synth.gen_kv(seed, layers, Hkv, L + N + 2, d, L + N)
+    q = synth.gen_q(seed, layers, N, Hq, d)
+    W = synth.normal_bf16(g, (V, D), 0.05)
+    hidden, am, t1, en = _hidden(g, N, W)
+    drafts = synth.gen_drafts(seed, canon, am, V, 0.7) if V > 1 else np.zeros(N, np.int32)
+    kd, vd = to_dev(k, dev), to_dev(v, dev)
+    out = torch.empty((layers, N, Hq, d), dtype=torch.bfloat16, device=dev)
+    g_am = torch.empty(N, dtype=torch.int32, device=dev)
+    g_t1 = torch.empty(N, dtype=torch.float32, device=dev)
+    g_en = torch.empty(N, dtype=torch.float32, device=dev)
+    res = tv.make_result(dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(N, layers, Hkv, Hq, d, V, 0), dev)
+    tv.verify_step(b, bid, tv.KvCache(kd, vd, L), to_dev(q, dev), to_dev(hidden, dev), to_dev(W, dev),
+                   to_dev(drafts.astype(np.int32), dev), out, g_am, g_t1, g_en, res, ws)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    for layer in range(layers):
+        check_attention(got[layer], oracle.tree_attention(q[layer], k[layer], v[layer], L, canon),
+                        f"seed {seed} layer {layer} (N={N} L={L} d={d} Hq={Hq} Hkv={Hkv})")
+    assert np.array_equal(g_am.cpu().numpy(), am), seed
+    assert np.abs(g_t1.cpu().numpy() - t1).max() <= STAT_TOL
+    assert np.abs(g_en.cpu().numpy() - en).max() <= STAT_TOL
+    ka, path, bonus = oracle.accept(canon, drafts, am)
+    r = tv.parse_result(res)
+    assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (ka, path, bonus, L + ka, 0)
+    assert np.array_equal(bits(kd), oracle.kv_compact(k, L, path))
+    assert np.array_equal(bits(vd), oracle.kv_compact(v, L, path))
+    b.close()
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_batched_step(dev, seed):
+    g = synth.rng(9500 + seed)
+    d, Hkv = 128, int(g.choice([1, 2, 4]))
+    group = int(g.choice([1, 2, 4]))
+    Hq = Hkv * group
+    D, V = int(g.choice([64, 256, 520])), int(g.choice([129, 1000, 3001]))
+    batch = int(g.integers(1, 9))
+    b = tv.Bank(16, 0)
+    W = synth.normal_bf16(g, (V, D), 0.05)
+    seqs, host, rows = [], [], []
+    for i in range(batch):
+        n = int(g.integers(1, 65))
+        while n * group > 256:
+            n //= 2
+        parent = np.sort(synth.random_tree(g, max(n, 1)))
+        parent[0] = -1
+        L = int(g.choice([0, 5, 130, 777, 2000]))
+        bid, _ = b.add(parent)
+        k, v = synth.gen_kv(100 * seed + i, 1, Hkv, L + n + 1, d, L + n)
+        q = synth.gen_q(100 * seed + i, 1, n, Hq, d)
+        seqs.append((bid, parent, L, k, v, q))
+        rows.append(n)
+    R = sum(rows)
+    hidden, am, t1, en = _hidden(g, R, W)
+    r0 = 0
+    tseqs = []
+    for i, (bid, parent, L, k, v, q) in enumerate(seqs):
+        n = len(parent)
+        drafts = synth.gen_drafts(i, parent, am[r0:r0 + n], V, 0.7)
+        s = tv.Seq(bid, tv.KvCache(to_dev(k, dev), to_dev(v, dev), L), to_dev(q, dev), to_dev(drafts, dev),
+                   torch.empty((1, n, Hq, d), dtype=torch.bfloat16, device=dev), tv.make_result(dev))
+        tseqs.append(s)
+        host.append((parent, L, k, v, q, drafts, r0))
+        r0 += n
+    g_am = torch.empty(R, dtype=torch.int32, device=dev)
+    g_t1 = torch.empty(R, dtype=torch.float32, device=dev)
+    g_en = torch.empty(R, dtype=torch.float32, device=dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(R, 1, Hkv, Hq, d, V, 0), dev)
+    tv.verify_step_batched(b, tseqs, to_dev(hidden, dev), to_dev(W, dev), g_am, g_t1, g_en, ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(g_am.cpu().numpy(), am)
+    assert np.abs(g_en.cpu().numpy() - en).max() <= STAT_TOL
+    for s, (parent, L, k, v, q, drafts, r0) in zip(tseqs, host):
+        n = len(parent)
+        check_attention(s.attn_out[0].float().cpu().numpy(), oracle.tree_attention(q[0], k[0], v[0], L, parent))
+        ka, path, bonus = oracle.accept(parent, drafts, am[r0:r0 + n])
+        r = tv.parse_result(s.result)
+        assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (ka, path, bonus, L + ka, 0)
+        assert np.array_equal(bits(s.kv.k), oracle.kv_compact(k, L, path))
+    b.close()
