@@ -1,12 +1,19 @@
 """Randomised verification steps against the fp64 oracle: random trees (in
 and out of breadth-first order), prefix lengths (including 0), head_dim 64
 and 128, GQA groups, d_model not a multiple of 64, vocabularies from 1 token
-up, single and batched steps.  Same tolerances as the other parity tests."""
+up, single and batched steps.
+
+Same bars as the other parity tests, with one addition for attention: short or
+empty prefixes give rows that average a handful of values, whose outputs reach
+|x| ~ 4; there the bf16 probabilities of the P V product and the bf16 output
+alone account for about two bf16 ulps (2^-7 |x|), so an element may differ by
+max(1e-2, 2^-7 |ref|); the mean-abs bar stays 1e-3.  The workload-shaped tests
+keep the plain 1e-2 bar."""
 import numpy as np
 import pytest
 
 import oracle
-from helpers import STAT_TOL, bits, check_attention, to_dev
+from helpers import STAT_TOL, bits, to_dev
 from paper_2606_27550_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -22,6 +29,16 @@ def dev():
     build.build()
     torch.cuda.set_device(0)
     return torch.device("cuda:0")
+
+
+def check_attention_fuzz(got, ref, what):
+    got = got.astype(np.float64)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    err = np.abs(got - ref)
+    bound = np.maximum(1e-2, np.abs(ref) * 2.0 ** -7)
+    worst = np.argmax(err - bound)
+    assert (err <= bound).all(), f"{what}: |err| {err.flat[worst]:.3e} at |ref| {abs(ref.flat[worst]):.3f}"
+    assert err.mean() <= 1e-3, f"{what}: mean |err| {err.mean():.3e}"
 
 
 def _hidden(g, n, W, gap_min=1e-2):
@@ -83,8 +100,8 @@ def test_random_verify_step(dev, seed):
     torch.cuda.synchronize()
     got = out.float().cpu().numpy()
     for layer in range(layers):
-        check_attention(got[layer], oracle.tree_attention(q[layer], k[layer], v[layer], L, canon),
-                        f"seed {seed} layer {layer} (N={N} L={L} d={d} Hq={Hq} Hkv={Hkv})")
+        check_attention_fuzz(got[layer], oracle.tree_attention(q[layer], k[layer], v[layer], L, canon),
+                             f"seed {seed} layer {layer} (N={N} L={L} d={d} Hq={Hq} Hkv={Hkv})")
     assert np.array_equal(g_am.cpu().numpy(), am), seed
     assert np.abs(g_t1.cpu().numpy() - t1).max() <= STAT_TOL
     assert np.abs(g_en.cpu().numpy() - en).max() <= STAT_TOL
@@ -141,7 +158,8 @@ def test_random_batched_step(dev, seed):
     assert np.abs(g_en.cpu().numpy() - en).max() <= STAT_TOL
     for s, (parent, L, k, v, q, drafts, r0) in zip(tseqs, host):
         n = len(parent)
-        check_attention(s.attn_out[0].float().cpu().numpy(), oracle.tree_attention(q[0], k[0], v[0], L, parent))
+        check_attention_fuzz(s.attn_out[0].float().cpu().numpy(), oracle.tree_attention(q[0], k[0], v[0], L, parent),
+                             f"seed {seed} L={L} n={n}")
         ka, path, bonus = oracle.accept(parent, drafts, am[r0:r0 + n])
         r = tv.parse_result(s.result)
         assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (ka, path, bonus, L + ka, 0)
