@@ -229,6 +229,37 @@ struct tb_bank {
     std::mutex fork_mu;
 };
 
+// The helper stream of a step.  The LM head runs on the bank's helper stream,
+// forked from the caller's stream when the step starts and joined back before
+// acceptance; the bank's fork and join events are shared, so the bank's mutex
+// is held from the fork to the end of the step's enqueueing.
+class HelperFork {
+  public:
+    HelperFork(const tb_bank *bank, cudaStream_t s) : bank_(const_cast<tb_bank *>(bank)), s_(s), lk_(bank_->fork_mu)
+    {
+    }
+    cudaStream_t aux() const { return bank_->aux; }
+    tb_status fork(const char *fn)
+    {
+        cudaError_t e = cudaEventRecord(bank_->ev_fork, s_);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(bank_->aux, bank_->ev_fork, 0);
+        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: fork: %s", fn, cudaGetErrorString(e));
+    }
+    tb_status join(const char *fn)
+    {
+        cudaError_t e = cudaEventRecord(bank_->ev_join, bank_->aux);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(s_, bank_->ev_join, 0);
+        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: join: %s", fn, cudaGetErrorString(e));
+    }
+
+  private:
+    tb_bank *bank_;
+    cudaStream_t s_;
+    std::lock_guard<std::mutex> lk_;
+};
+
 extern "C" tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
                                      int32_t *depth, uint64_t *anc)
 {
@@ -909,24 +940,16 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
     lt.logz_t = tr.logz_t;
     lt.ent_t = tr.ent_t;
     lt.logits_out = logits;
-    {
-        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
-        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step_sampled: fork");
-        if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
-            return st;
-        if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                             bank->aux, fn, 0, &lt)) != TB_OK)
-            return st;
-        e = cudaEventRecord(bank->ev_join, bank->aux);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step_sampled: join");
-    }
+    HelperFork hf(bank, s);
+    if ((st = hf.fork(fn)) != TB_OK)
+        return st;
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+        return st;
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                         hf.aux(), fn, 0, &lt)) != TB_OK)
+        return st;
+    if ((st = hf.join(fn)) != TB_OK)
+        return st;
     if ((st = sample_enqueue(bank, bank_id, draft_tokens, logits, tr.logz_t, draft_probs, uniforms, vocab, kv->L,
                              temperature, logits + (size_t)N * vocab, result, reinterpret_cast<const int *>(ws), s,
                              fn)) != TB_OK)
@@ -995,26 +1018,18 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         lt.gather.n_seq = 1;
         lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, tr.draft_logit, 0, N};
     }
-    {
-        // attention on the caller's stream; the LM head forked onto the bank's
-        // helper stream fills the SMs that attention CTAs release; join before acceptance
-        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
-        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step: fork");
-        if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
-            return st;
-        if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                             bank->aux, fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr)) != TB_OK)
-            return st;
-        e = cudaEventRecord(bank->ev_join, bank->aux);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step: join");
-    }
+    // attention on the caller's stream; the LM head forked onto the bank's
+    // helper stream fills the SMs that attention CTAs release; join before acceptance
+    HelperFork hf(bank, s);
+    if ((st = hf.fork(fn)) != TB_OK)
+        return st;
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+        return st;
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                         hf.aux(), fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr)) != TB_OK)
+        return st;
+    if ((st = hf.join(fn)) != TB_OK)
+        return st;
     AcceptParams p =
         accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
     if (typ)
@@ -1115,12 +1130,10 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
 
     // attention on the caller's stream, the LM head forked onto the helper
     // stream (it fills the SMs the attention CTAs release), joined before acceptance
-    std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
-    cudaError_t e = cudaEventRecord(bank->ev_fork, s);
-    if (e == cudaSuccess)
-        e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
-    if (e != cudaSuccess)
-        return cuda_fail(e, "verify_step_batched: fork");
+    HelperFork hf(bank, s);
+    if ((st = hf.fork(fn)) != TB_OK)
+        return st;
+    cudaError_t e = cudaSuccess;
     // tree attention of every sequence (after the rotary embedding of their tree keys)
     if (tc) {
         const bool rope = kv0.rope_theta != 0.f;
@@ -1181,11 +1194,8 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             TB_OK)
             return st;
     }
-    e = cudaEventRecord(bank->ev_join, bank->aux);
-    if (e == cudaSuccess)
-        e = cudaStreamWaitEvent(s, bank->ev_join, 0);
-    if (e != cudaSuccess)
-        return cuda_fail(e, "verify_step_batched: join");
+    if ((st = hf.join(fn)) != TB_OK)
+        return st;
     // acceptance + compaction, one launch
     AcceptParams ps[TB_MAX_BATCH];
     int r0 = 0;
@@ -1321,12 +1331,9 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     for (int r = 0; r < policy->n_rungs; ++r)
         sc.rung_tree[r] = bank->d_desc + policy->bank_ids[r];
     {
-        std::lock_guard<std::mutex> lk(const_cast<tb_bank *>(bank)->fork_mu);
-        cudaError_t e = cudaEventRecord(bank->ev_fork, s);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(bank->aux, bank->ev_fork, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step_scheduled: fork");
+        HelperFork hf(bank, s);
+        if ((st = hf.fork(fn)) != TB_OK)
+            return st;
         if (kv->rope_theta != 0.f) {
             RopeParams rp{};
             rp.seq[0] = rope_seq(kv, sc.rung_tree[0]);
@@ -1340,7 +1347,7 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
             sc.rope_tab = rope_table(ws);
         }
         const char *err = "";
-        e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
+        cudaError_t e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
                                  &err);
         if (e == cudaErrorInvalidValue && err[0])
@@ -1348,13 +1355,10 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
         if ((st = lm_enqueue(hidden, N_max, lm_head, d_model, vocab, argmax, top1, entropy, ws,
-                             kPartBase + attn_bytes, bank->aux, fn)) != TB_OK)
+                             kPartBase + attn_bytes, hf.aux(), fn)) != TB_OK)
             return st;
-        e = cudaEventRecord(bank->ev_join, bank->aux);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(s, bank->ev_join, 0);
-        if (e != cudaSuccess)
-            return cuda_fail(e, "verify_step_scheduled: join");
+        if ((st = hf.join(fn)) != TB_OK)
+            return st;
     }
     AcceptParams p = accept_params(bank, policy->bank_ids[0], draft_tokens, argmax, vocab, 0, result,
                                    reinterpret_cast<const int *>(ws));
