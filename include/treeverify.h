@@ -295,8 +295,10 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
  *  - Every call clears the array's arrival counters on `stream` and reuses the
  *    array, which keeps the previous call's partial results: calls that can
  *    overlap on the GPU (different streams without ordering) race.
- *  - Shapes whose scratch exceeds the array (n_rows x vocab partials larger
- *    than 4 MiB) are rejected with TB_ECAPACITY before anything is enqueued.
+ *  - The scratch is one partial per persistent CTA and per merge group for
+ *    every row (about 2 MiB at 256 rows with 152 SMs, for any vocabulary);
+ *    a device whose SM count needs more than 4 MiB is rejected with
+ *    TB_ECAPACITY before anything is enqueued.
  * Arguments, layouts and tolerances are those of lm_head_stats.  The paper has
  * no counterpart: this is an integration convenience of this library. */
 TB_API tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,

@@ -7,11 +7,14 @@ namespace tv {
 
 // LM head (lm_head.cu)
 struct LmPlan {
-    int R_pad, n_tiles, n_kblocks, stages, tmem_cols, group_size, n_groups, bps;
+    int R_pad, n_tiles, n_kblocks, stages, acc_cols, group_size, n_groups;
+    int ctas_per_sm;  // 2 when two rings fit side by side, else 1
+    int P;            // persistent CTAs: ctas_per_sm per SM, at most one per vocab tile
+    int n_counters;   // workspace counters used (group tickets)
     size_t smem_bytes;
-    size_t ws_bytes;  // partials (tile + group), 256-byte aligned
+    size_t ws_bytes;  // partials (CTA + group), 256-byte aligned
 };
-LmPlan lm_plan(int R, int D, int V);
+LmPlan lm_plan(int R, int D, int V, int n_sm);
 // typical-acceptance inputs produced by the same pass: per-row statistics at
 // temperature T and the draft-token logit of every tree edge j, written to
 // seq[b].out[j] for edges whose parent row row_base + parent[j] is in [0, R)
@@ -33,7 +36,7 @@ struct LmTypical {
     float *logits_out;  // null, or [R][V] fp32: the logits themselves (speculative sampling needs whole rows)
 };
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
-                           float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
+                           float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
                            const char **err, int expire_wait = 0, const LmTypical *typ = nullptr);
 
 // tree attention (attention.cu)

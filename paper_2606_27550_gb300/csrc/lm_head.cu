@@ -7,25 +7,21 @@
 // the entropy feature that the EntMTP scheduler consumes (Sec. 4, "Path-value
 // score" and "Cost": computed from the verifier logits already on chip).
 //
-// Design (swap-AB): one CTA per 128-entry vocab tile.  The tile of W
+// Design (swap-AB, persistent).  The 128-entry vocab tiles are split into
+// contiguous runs over a persistent grid (two CTAs per SM when their rings fit
+// side by side, one otherwise); a CTA walks its run tile by tile.  The tile of W
 // ([128][64] bf16 per k-block, 128-byte swizzled by TMA) is the MMA's M=128 A
-// operand; the tree rows ([R_pad][64] per k-block, same swizzle) are the
-// N = R_pad B operand.  tcgen05.mma (kind::f16, f32 accumulate) builds the
-// 128 x R_pad logit tile in TMEM over d_model/64 k-blocks fed by a multi-stage
-// TMA ring.  Warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, then all
-// eight warps read TMEM (lane = vocab entry; two warps per lane quadrant, each
-// taking half of the columns), transpose through shared memory and reduce
-// each row.  Per-tile statistics are merged in two levels by
-// atomic arrival tickets (the last CTA of a group merges the group; the last
-// group merges everything); no CTA ever waits for another.
+// operand, the tree rows ([R_pad][64], same swizzle) the N = R_pad B operand;
+// tcgen05.mma (kind::f16, f32 accumulate) builds the 128 x R_pad logit tile in
+// TMEM.  Warp 0 lane 0 issues TMA into a ring that runs across tiles, warp 1
+// lane 0 the MMAs into one of two TMEM accumulators, and warps 2-9 drain the
+// other accumulator meanwhile (32 tree rows at a time: TMEM -> shared memory
+// transposed -> eight threads per row reduce its 128 logits), folding each
+// tile into per-row running statistics of the CTA.  The CTAs' statistics are
+// merged in two levels by atomic arrival tickets (the last CTA of a group
+// merges the group; the last group merges everything); no CTA ever waits for
+// another.
 //
-// Typical-acceptance mode (kTyp): the same pass also yields, per row, the
-// statistics of the tempered distribution softmax(z / T) -- its log-partition
-// logZ_T = m / T + ln sum e^((z-m)/T) and entropy H_T -- and gathers the logit
-// z_{parent(j)}[draft[j]] of every tree edge j straight from the tile's logits
-// in shared memory (the Medusa/Hydra typical-acceptance inputs, Sec. 5.1/5.2).
-// Warps 2-3, idle during the k-loop, find the edges whose token falls in this
-// CTA's vocab tile meanwhile.
 #include <math.h>
 #include <stdlib.h>
 
@@ -37,12 +33,14 @@ struct LmParams {
     CUtensorMap tmap_w;  // (d_model, vocab), box (64, 128), 128B swizzle
     CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad), 128B swizzle
     int R, R_pad, D, V;
-    int n_tiles, n_kblocks, stages, tmem_cols;
-    int bps;             // 64-column boxes per pipeline stage
+    int n_tiles, nk, stages, acc_cols;
+    int P;               // CTAs
     int group_size, n_groups;
-    float4 *part_tile;   // [n_tiles][R_pad]  (max, argmax bits, s, t)
+    float4 *part_cta;    // [P][R_pad]  (max, argmax bits, s, t)
     float4 *part_group;  // [n_groups][R_pad]
-    int *counters;       // [n_groups + 1], zero between launches
+    float2 *part_cta_t;  // [P][R_pad]  (sT, tT), typical mode
+    float2 *part_group_t;
+    int *counters;       // [n_groups + 1] group tickets, zero between launches
     int *status;
     int expire_wait;     // test hook: the epilogue waits on a barrier nothing arrives on
     int32_t *argmax;
@@ -50,8 +48,6 @@ struct LmParams {
     float *entropy;
     // typical-acceptance mode
     float inv_t;          // 1 / T
-    float2 *part_tile_t;  // [n_tiles][R_pad]  (sT, tT)
-    float2 *part_group_t; // [n_groups][R_pad]
     float *logz_t;        // [R] m / T + ln sT
     float *ent_t;         // [R] ln sT - tT / sT
     LmGather gather;
@@ -69,10 +65,14 @@ struct RowStat {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// Threads per CTA: warp 0 lane 0 issues TMA, warp 1 lane 0 the MMAs; all eight
-// warps then share the epilogue (warps w and w + 4 read the same TMEM lane
-// quadrant and split its columns) and the per-row scans.
-constexpr int kLmThreads = 256;
+// Threads per CTA: warp 0 lane 0 issues TMA, warp 1 lane 0 the MMAs, warps
+// 2-9 form the epilogue (warps w and w + 4 read the same TMEM lane quadrant
+// w % 4 and split each 32-row chunk's columns); all ten merge at the end.
+constexpr int kLmThreads = 320;
+constexpr int kEpiThreads = 256;
+constexpr int kLmChunk = 32;             // tree rows per epilogue chunk
+constexpr int kLmTpr = kEpiThreads / kLmChunk;  // threads per row in the chunk scans
+constexpr int kChunkLd = 128 + kLmTpr;   // chunk row stride (floats): conflict-free writes and scans
 
 __device__ __forceinline__ RowStat stat_empty()
 {
@@ -258,244 +258,303 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
     __syncthreads();
 }
 
+// Named barrier of the eight epilogue warps.
+__device__ __forceinline__ void epi_sync()
+{
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+}
+
+// First vocab tile of CTA c's run.
+__device__ __forceinline__ int lm_tile_begin(const LmParams &p, int c)
+{
+    return (int)((long long)c * p.n_tiles / p.P);
+}
+
+// k-block j of a tile's loop: the order is rotated by the tile index, so the
+// CTAs in flight read their W rows at spread-out column offsets rather than
+// all at the same one.
+__device__ __forceinline__ int lm_kb(const LmParams &p, int tile, int j)
+{
+    const int x = j + (int)(((long long)tile * 5) % p.nk);
+    return x >= p.nk ? x - p.nk : x;
+}
+
 template <bool kTyp>
-__global__ void __launch_bounds__(kLmThreads, 1) k2_lm_head(const __grid_constant__ LmParams p)
+__global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constant__ LmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[8];
     __shared__ __align__(8) uint64_t empty_bar[8];
-    __shared__ __align__(8) uint64_t acc_bar;
-    __shared__ __align__(8) uint64_t never_bar;
+    __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
+    __shared__ __align__(8) uint64_t drain_bar, never_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
-    __shared__ int ticket;
-    // typical mode: edges whose draft token lies in this tile, packed as
-    // (seq << 24) | (node << 16) | (row << 7) | col; overflow -> rescan in the epilogue
+    __shared__ int s_ticket, s_ok;
+    // typical mode: edges whose draft token lies in the current tile, packed as
+    // (seq << 24) | (node << 16) | (row << 7) | col; overflow -> rescan per chunk
     constexpr int kHitCap = 64;
     __shared__ int s_hit[kTyp ? kHitCap : 1];
     __shared__ int s_nhit;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = p.stages;
-    const int B = p.bps;
-    const uint32_t hb = (uint32_t)p.R_pad * 128u;  // one hidden-row box
-    const uint32_t w_stage = 16384u * B, h_stage = hb * B;
-    uint8_t *sW = smem;
-    uint8_t *sH = smem + (size_t)S * w_stage;
+    const uint32_t hb = (uint32_t)p.R_pad * 128u;  // one 64-column box of the tree rows
+    const uint32_t stage_bytes = 16384u + hb;
+    uint8_t *ring = smem;
+    float *chunk = reinterpret_cast<float *>(smem + (size_t)S * stage_bytes);  // [kLmChunk][kChunkLd]
+    RowStat *run = reinterpret_cast<RowStat *>(chunk + kLmChunk * kChunkLd);   // [R_pad] running statistics
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.x;
-    const int v0 = tile * 128;
-    const int nk = p.n_kblocks;  // stages of B boxes
+    const int c = blockIdx.x;
+    const int tile0 = lm_tile_begin(p, c), tile1 = lm_tile_begin(p, c + 1);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        mbar_init(&acc_bar, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], kEpiThreads / 32);
+        }
+        mbar_init(&drain_bar, 1);
         mbar_init(&never_bar, 1);
         abort_flag = 0;
-        s_nhit = 0;
         fence_mbar_init();
         prefetch_tmap(&p.tmap_w);
         prefetch_tmap(&p.tmap_h);
     }
     if (warp == 1) {
-        tmem_alloc(&tmem_slot, (uint32_t)p.tmem_cols);
+        tmem_alloc(&tmem_slot, 2u * (uint32_t)p.acc_cols);
         tmem_relinquish();
     }
+    for (int r = threadIdx.x; r < p.R_pad; r += blockDim.x)
+        run[r] = stat_empty();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer: one stage = B adjacent 64-column boxes of
-        // W (128 rows) and of the hidden rows, so each W row is fetched as a
-        // contiguous run of B x 128 bytes.
-        // Tiles start their k-loop at different stages so that the CTAs in
-        // flight read W rows at spread-out column offsets.
-        const int rot = (int)(((long long)tile * 5) % nk);
-        int issued = 0;
-        for (int kb = 0; kb < nk; ++kb) {
-            const int s = kb % S;
-            const uint32_t ph = (uint32_t)(kb / S) & 1u;
-            if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
-                break;
-            const int kx = (kb + rot) % nk;
-            mbar_arrive_expect_tx(&full_bar[s], w_stage + h_stage);
-            for (int b = 0; b < B; ++b) {
-                const int x = (kx * B + b) * 64;
-                tma_load_2d(sW + (size_t)s * w_stage + (size_t)b * 16384, &p.tmap_w, &full_bar[s], x, v0);
-                tma_load_2d(sH + (size_t)s * h_stage + (size_t)b * hb, &p.tmap_h, &full_bar[s], x, 0);
+    if (warp == 0) {
+        // ---------------- TMA producer: one stage = one 64-column box of W
+        // (128 rows) and of the tree rows; the ring runs across the range's tiles
+        if (lane == 0) {
+            long long g = 0;
+            bool ok = true;
+            for (int tile = tile0; tile < tile1 && ok; ++tile) {
+                for (int j = 0; j < p.nk; ++j, ++g) {
+                    const int kb = lm_kb(p, tile, j);
+                    const int s = (int)(g % S);
+                    if (!mbar_wait_bounded(&empty_bar[s], ((uint32_t)(g / S) & 1u) ^ 1u, &abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+                    tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
+                    tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                }
             }
-            issued = kb + 1;
+            if (!ok)  // gave up: the copies in flight land before the CTA exits
+                for (long long it = (g > S ? g - S : 0); it < g; ++it)
+                    mbar_wait_drain(&full_bar[it % S], (uint32_t)(it / S) & 1u);
         }
-        if (issued < nk) {
-            // gave up: let the copies already in flight land before the CTA exits
-            for (int kb = (issued > S ? issued - S : 0); kb < issued; ++kb)
-                mbar_wait_drain(&full_bar[kb % S], (uint32_t)(kb / S) & 1u);
+    } else if (warp == 1) {
+        // ---------------- MMA issuer: the CTA's i-th tile accumulates into TMEM buffer i & 1
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, p.R_pad);
+            long long g = 0;
+            bool ok = true;
+            for (int tile = tile0, i = 0; tile < tile1 && ok; ++tile, ++i) {
+                const int b = i & 1;
+                if (!mbar_wait_bounded(&acc_empty[b], ((uint32_t)(i >> 1) & 1u) ^ 1u, &abort_flag, p.status))
+                    break;
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(b * p.acc_cols);
+                for (int j = 0; j < p.nk; ++j, ++g) {
+                    const int s = (int)(g % S);
+                    if (!mbar_wait_bounded(&full_bar[s], (uint32_t)(g / S) & 1u, &abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_base = smem_u32(ring + (size_t)s * stage_bytes);
+                    const uint32_t b_base = a_base + 16384u;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const uint64_t ad = smem_desc_sw128(a_base + k * 32, 0, 1024);
+                        const uint64_t bd = smem_desc_sw128(b_base + k * 32, 0, 1024);
+                        tc_mma_f16_ss(d, ad, bd, idesc, (j != 0 || k != 0) ? 1u : 0u);
+                    }
+                    tc_commit(&empty_bar[s]);
+                }
+                if (!ok)
+                    break;
+                tc_commit(&acc_full[b]);
+            }
+            // arrives when every MMA issued above has retired (waited for before TMEM is released)
+            tc_commit(&drain_bar);
         }
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer
-        constexpr uint32_t kIdescM = 128;
-        const uint32_t idesc = idesc_bf16_f32(kIdescM, p.R_pad);
-        for (int kb = 0; kb < nk; ++kb) {
-            const int s = kb % S;
-            const uint32_t ph = (uint32_t)(kb / S) & 1u;
-            if (!mbar_wait_bounded(&full_bar[s], ph, &abort_flag, p.status))
+    } else {
+        // ---------------- epilogue (warps 2-9)
+        const int e = threadIdx.x - 64;
+        const int q = warp & 3, half = (warp - 2) >> 2;
+        const int vr = 32 * q + lane;                 // this thread's vocab entry within the tile (TMEM lane)
+        const int sub = e % kLmTpr, rloc = e / kLmTpr;  // chunk scans: kLmTpr threads per row
+        // the same verdict for all epilogue threads: did every wait so far succeed?
+        auto agree = [&]() -> bool {
+            epi_sync();
+            if (e == 0)
+                s_ok = (abort_flag == 0);
+            epi_sync();
+            return s_ok != 0;
+        };
+        for (int tile = tile0, i = 0; tile < tile1; ++tile, ++i) {
+            const int b = i & 1;
+            mbar_wait_bounded(p.expire_wait ? &never_bar : &acc_full[b], (uint32_t)(i >> 1) & 1u, &abort_flag,
+                              p.status);
+            if (!agree())
                 break;
             tc_fence_after();
-            for (int b = 0; b < B; ++b) {
-                const uint32_t a_base = smem_u32(sW + (size_t)s * w_stage + (size_t)b * 16384);
-                const uint32_t b_base = smem_u32(sH + (size_t)s * h_stage + (size_t)b * hb);
+            const int v0 = tile * 128, nvalid = min(128, p.V - v0);
+            if constexpr (kTyp) {
+                // the tree edges whose draft token lies in this tile
+                if (e == 0)
+                    s_nhit = 0;
+                epi_sync();
+                for (int bq = 0; bq < p.gather.n_seq; ++bq)
+                    for (int j = 1 + e; j < p.gather.seq[bq].n; j += kEpiThreads) {
+                        int row, col;
+                        if (gather_hit(p.gather, bq, j, p.R, v0, nvalid, &row, &col)) {
+                            const int h = atomicAdd(&s_nhit, 1);
+                            if (h < kHitCap)
+                                s_hit[h] = (bq << 24) | (j << 16) | (row << 7) | col;
+                        }
+                    }
+                epi_sync();
+            }
+            const uint32_t acc = tmem + (uint32_t)(b * p.acc_cols) + ((uint32_t)(32 * q) << 16);
+            for (int c0 = 0; c0 < p.R_pad; c0 += kLmChunk) {
+                const int col = c0 + 16 * half;  // this warp's 16 tree rows of the chunk
+                uint32_t v[16];
+                if (col < p.R_pad) {
+                    tmem_ld_32x32b_x16(acc + (uint32_t)col, v);
+                    tmem_ld_wait();
+                }
+                if (c0 + kLmChunk >= p.R_pad) {
+                    // last read of this accumulator: the MMAs of segment i + 2 may reuse it
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0)
+                        mbar_arrive(&acc_empty[b]);
+                }
+                if (col < p.R_pad) {
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const uint64_t a = smem_desc_sw128(a_base + k * 32, 0, 1024);
-                    const uint64_t bd = smem_desc_sw128(b_base + k * 32, 0, 1024);
-                    tc_mma_f16_ss(tmem, a, bd, idesc, (kb | b | k) != 0 ? 1u : 0u);
+                    for (int j = 0; j < 16; ++j)
+                        chunk[(16 * half + j) * kChunkLd + vr] = __uint_as_float(v[j]);
                 }
-            }
-            tc_commit(&empty_bar[s]);
-        }
-        tc_commit(&acc_bar);
-    } else if (kTyp && warp >= 2) {
-        // ---------------- edges to gather (warps 2.. are otherwise idle here)
-        const int nvalid = min(128, p.V - v0);
-        const int helpers = (int)blockDim.x - 64;
-        for (int b = 0; b < p.gather.n_seq; ++b) {
-            for (int j = 1 + (threadIdx.x - 64); j < p.gather.seq[b].n; j += helpers) {
-                int row, col;
-                if (gather_hit(p.gather, b, j, p.R, v0, nvalid, &row, &col)) {
-                    const int slot = atomicAdd(&s_nhit, 1);
-                    if (slot < kHitCap)
-                        s_hit[slot] = (b << 24) | (j << 16) | (row << 7) | col;
+                epi_sync();
+                // rows c0 .. c0 + 31: two passes (max / first argmax, then the sums)
+                const int r = c0 + rloc;
+                RowStat st = stat_empty();
+                if (r < p.R) {
+                    const float *row = chunk + rloc * kChunkLd;
+                    for (int j = sub; j < nvalid; j += kLmTpr) {
+                        const float z = row[j];
+                        if (z > st.m) {
+                            st.m = z;
+                            st.idx = v0 + j;
+                        }
+                    }
+                    for (int j = sub; j < nvalid; j += kLmTpr) {
+                        const float dz = row[j] - st.m;
+                        const float ex = ex2_approx(dz * kLog2e);
+                        st.s += ex;
+                        st.t += ex * dz;
+                        if constexpr (kTyp) {
+                            const float dT = dz * p.inv_t;
+                            const float eT = ex2_approx(dT * kLog2e);
+                            st.sT += eT;
+                            st.tT += eT * dT;
+                        }
+                    }
                 }
+                st = group_merge<kTyp>(st, kLmTpr, p.inv_t);
+                if (sub == 0 && r < p.R)
+                    run[r] = stat_merge<kTyp>(run[r], st, p.inv_t);
+                if constexpr (kTyp) {
+                    const int nhit = s_nhit;
+                    if (nhit <= kHitCap) {
+                        for (int h = e; h < nhit; h += kEpiThreads) {
+                            const int w = s_hit[h];
+                            const int row = (w >> 7) & 0x1ff;
+                            if (row >= c0 && row < c0 + kLmChunk)
+                                p.gather.seq[w >> 24].out[(w >> 16) & 0xff] = chunk[(row - c0) * kChunkLd + (w & 0x7f)];
+                        }
+                    } else {
+                        for (int bq = 0; bq < p.gather.n_seq; ++bq)
+                            for (int j = 1 + e; j < p.gather.seq[bq].n; j += kEpiThreads) {
+                                int row, cc;
+                                if (gather_hit(p.gather, bq, j, p.R, v0, nvalid, &row, &cc) && row >= c0 &&
+                                    row < c0 + kLmChunk)
+                                    p.gather.seq[bq].out[j] = chunk[(row - c0) * kChunkLd + cc];
+                            }
+                    }
+                    if (p.logits_out) {
+                        // whole logit rows for speculative sampling: 128 consecutive floats per row
+                        for (int x = e; x < kLmChunk * 128; x += kEpiThreads) {
+                            const int rr = x >> 7, j = x & 127;
+                            if (c0 + rr < p.R && j < nvalid)
+                                p.logits_out[(size_t)(c0 + rr) * p.V + v0 + j] = chunk[rr * kChunkLd + j];
+                        }
+                    }
+                }
+                epi_sync();  // the chunk buffer is rewritten next
             }
         }
+        // this CTA's statistics for the final merge
+        if (!abort_flag)
+            for (int r = e; r < p.R; r += kEpiThreads) {
+                p.part_cta[(size_t)c * p.R_pad + r] = stat_pack(run[r]);
+                if constexpr (kTyp)
+                    p.part_cta_t[(size_t)c * p.R_pad + r] = make_float2(run[r].sT, run[r].tT);
+            }
     }
-    __syncwarp();
 
-    // ---------------- epilogue: TMEM -> shared (transposed) -> per-row stats
-    mbar_wait_bounded(p.expire_wait ? &never_bar : &acc_bar, 0, &abort_flag, p.status);
-    tc_fence_after();
-    __syncthreads();
-    const bool ok = (abort_flag == 0);
-    // logits[r][v] at r * ld + v; the row stride 128 + tpr keeps both the
-    // column writes below and the per-row scans free of bank conflicts.
-    const int tpr = threads_per_row(p.R_pad);
-    const int ld = 128 + tpr;
-    float *logits = reinterpret_cast<float *>(smem);  // aliases the drained ring
-    if (ok) {
-        // warps w and w + 4 read TMEM lane quadrant w % 4 (vocab rows 32 (w % 4) ..)
-        // and split the columns (tree rows) in alternate 16-column chunks
-        const int quad = warp & 3, half = warp >> 2, halves = (int)blockDim.x >> 7;
-        const uint32_t row_addr = tmem + ((uint32_t)(32 * quad) << 16);
-        for (int c0 = 16 * half; c0 < p.R_pad; c0 += 16 * halves) {
-            uint32_t r[16];
-            tmem_ld_32x32b_x16(row_addr + (uint32_t)c0, r);
-            tmem_ld_wait();
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-                logits[(c0 + j) * ld + 32 * quad + lane] = __uint_as_float(r[j]);
-        }
-    } else if (warp == 1 && lane == 0) {
-        mbar_wait_drain(&acc_bar, 0);  // MMAs issued before giving up must finish before dealloc
-    }
+    // ---------------- teardown: every MMA has retired before TMEM is released
     tc_fence_before();
     __syncthreads();
-    if (warp == 1)
-        tmem_dealloc(tmem, (uint32_t)p.tmem_cols);
-    if (!ok)
-        return;
-
-    // per-row statistics of this tile: tpr threads per row, two passes
-    {
-        const int sub = threadIdx.x % tpr;
-        const int nvalid = min(128, p.V - v0);
-        for (int r0 = 0; r0 < p.R; r0 += (int)blockDim.x / tpr) {
-            const int r = r0 + threadIdx.x / tpr;
-            RowStat st = stat_empty();
-            if (r < p.R) {
-                const float *row = logits + r * ld;
-                for (int j = sub; j < nvalid; j += tpr) {
-                    const float z = row[j];
-                    if (z > st.m) {
-                        st.m = z;
-                        st.idx = v0 + j;
-                    }
-                }
-                for (int j = sub; j < nvalid; j += tpr) {
-                    const float dz = row[j] - st.m;
-                    const float e = ex2_approx(dz * kLog2e);
-                    st.s += e;
-                    st.t += e * dz;
-                    if constexpr (kTyp) {
-                        const float dT = dz * p.inv_t;
-                        const float eT = ex2_approx(dT * kLog2e);
-                        st.sT += eT;
-                        st.tT += eT * dT;
-                    }
-                }
-            }
-            st = group_merge<kTyp>(st, tpr, p.inv_t);
-            if (sub == 0 && r < p.R) {
-                p.part_tile[(size_t)tile * p.R_pad + r] = stat_pack(st);
-                if constexpr (kTyp)
-                    p.part_tile_t[(size_t)tile * p.R_pad + r] = make_float2(st.sT, st.tT);
-            }
-        }
-        if constexpr (kTyp) {
-            if (p.logits_out) {
-                // whole logit rows for speculative sampling: 128 consecutive floats per row
-                for (int e = threadIdx.x; e < p.R * 128; e += blockDim.x) {
-                    const int r = e >> 7, j = e & 127;
-                    if (j < nvalid)
-                        p.logits_out[(size_t)r * p.V + v0 + j] = logits[r * ld + j];
-                }
-            }
-            const int nhit = s_nhit;
-            if (nhit <= kHitCap) {
-                for (int i = threadIdx.x; i < nhit; i += blockDim.x) {
-                    const int w = s_hit[i];
-                    const int b = w >> 24, j = (w >> 16) & 0xff, row = (w >> 7) & 0x1ff, col = w & 0x7f;
-                    p.gather.seq[b].out[j] = logits[row * ld + col];
-                }
-            } else {
-                for (int b = 0; b < p.gather.n_seq; ++b)
-                    for (int j = 1 + threadIdx.x; j < p.gather.seq[b].n; j += blockDim.x) {
-                        int row, col;
-                        if (gather_hit(p.gather, b, j, p.R, v0, nvalid, &row, &col))
-                            p.gather.seq[b].out[j] = logits[row * ld + col];
-                    }
-            }
-        }
+    if (warp == 1) {
+        if (lane == 0)
+            mbar_wait_drain(&drain_bar, 0);
+        __syncwarp();
+        tmem_dealloc(tmem, 2u * (uint32_t)p.acc_cols);
     }
+    if (abort_flag)
+        return;
 
-    // ---------------- two-level merge by arrival tickets
+    // ---------------- two-level merge of the CTAs' statistics by arrival tickets
     __threadfence();
     __syncthreads();
-    const int g = tile / p.group_size;
+    const int g = c / p.group_size;
     const int g_first = g * p.group_size;
-    const int g_count = min(p.group_size, p.n_tiles - g_first);
+    const int g_count = min(p.group_size, p.P - g_first);
     if (threadIdx.x == 0)
-        ticket = atomicAdd(&p.counters[g], 1);
+        s_ticket = atomicAdd(&p.counters[g], 1);
     __syncthreads();
-    if (ticket != g_count - 1)
+    if (s_ticket != g_count - 1)
         return;
     __threadfence();
-    float4 *sbuf = reinterpret_cast<float4 *>(smem);
-    merge_partials<kTyp>(p, p.part_tile + (size_t)g_first * p.R_pad, p.part_tile_t + (size_t)g_first * p.R_pad,
-                         g_count, sbuf, p.part_group + (size_t)g * p.R_pad, p.part_group_t + (size_t)g * p.R_pad);
+    float4 *sbuf = reinterpret_cast<float4 *>(smem);  // the drained ring
+    merge_partials<kTyp>(p, p.part_cta + (size_t)g_first * p.R_pad, p.part_cta_t + (size_t)g_first * p.R_pad, g_count,
+                         sbuf, p.part_group + (size_t)g * p.R_pad, p.part_group_t + (size_t)g * p.R_pad);
     if (threadIdx.x == 0)
         p.counters[g] = 0;
     __threadfence();
     __syncthreads();
     if (threadIdx.x == 0)
-        ticket = atomicAdd(&p.counters[p.n_groups], 1);
+        s_ticket = atomicAdd(&p.counters[p.n_groups], 1);
     __syncthreads();
-    if (ticket != p.n_groups - 1)
+    if (s_ticket != p.n_groups - 1)
         return;
     __threadfence();
     merge_partials<kTyp>(p, p.part_group, p.part_group_t, p.n_groups, sbuf, nullptr, nullptr);
@@ -511,60 +570,54 @@ static int ceil_div(int a, int b)
     return (a + b - 1) / b;
 }
 
-// 64-column boxes per pipeline stage.  Measured on GB300 (V=32000 and 128256,
-// 26-200 rows): one or two boxes per stage are within 3%; four boxes cost
-// stages and lose; so one box, the deepest ring.
-static int lm_boxes_per_stage(int R_pad)
-{
-    (void)R_pad;
-    return 1;
-}
-
-LmPlan lm_plan(int R, int D, int V)
+LmPlan lm_plan(int R, int D, int V, int n_sm)
 {
     LmPlan pl{};
     pl.R_pad = ceil_div(R, 16) * 16;
     pl.n_tiles = ceil_div(V, 128);
-    pl.bps = lm_boxes_per_stage(pl.R_pad);
-    pl.n_kblocks = ceil_div(D, 64 * pl.bps);
-    const int stage_bytes = (16384 + pl.R_pad * 128) * pl.bps;
-    // Up to 64 rows two CTAs share an SM (110 KB each); wider rows need a
-    // transpose buffer that leaves one CTA per SM, so its ring takes ~200 KB.
-    const size_t transpose_bytes = (size_t)pl.R_pad * (128 + 8) * 4;
-    const int budget = (transpose_bytes + 1024 <= 110 * 1024) ? 110 * 1024 : 200 * 1024;
-    pl.stages = budget / stage_bytes;
+    pl.n_kblocks = ceil_div(D, 64);
+    int cols = 32;
+    while (cols < pl.R_pad)
+        cols *= 2;
+    pl.acc_cols = cols;
+    const size_t stage_bytes = 16384 + (size_t)pl.R_pad * 128;
+    const size_t fixed = (size_t)kLmChunk * kChunkLd * 4 + (size_t)pl.R_pad * sizeof(RowStat);
+    // Two CTAs share an SM when each still gets a ring of at least three stages
+    // in half of its shared memory and four accumulators fit in TMEM: two
+    // independent TMA pipelines per SM stream W faster than one deeper ring.
+    const size_t pad = 1024 + 1024;  // alignment pad, static shared memory
+    const size_t half = 112 * 1024;
+    const int st2 = half > fixed + pad ? (int)((half - fixed - pad) / stage_bytes) : 0;
+    pl.ctas_per_sm = (st2 >= 3 && 4 * cols <= 512) ? 2 : 1;
+    const size_t budget = (pl.ctas_per_sm == 2 ? half : 227 * 1024) - fixed - pad;
+    pl.stages = (int)(budget / stage_bytes);
     if (pl.stages > 8)
         pl.stages = 8;
     if (pl.stages < 2)
         pl.stages = 2;
-    int cols = 32;
-    while (cols < pl.R_pad)
-        cols *= 2;
-    pl.tmem_cols = cols;
+    const int slots = pl.ctas_per_sm * (n_sm > 0 ? n_sm : 1);
+    pl.P = slots < pl.n_tiles ? slots : pl.n_tiles;
     int gs = 1;
-    while (gs * gs < pl.n_tiles)
+    while (gs * gs < pl.P)
         ++gs;
     pl.group_size = gs;
-    pl.n_groups = ceil_div(pl.n_tiles, gs);
-    size_t pipe = (size_t)pl.stages * stage_bytes;
-    size_t tr = (size_t)pl.R_pad * (128 + 8) * 4;
-    size_t mg = (size_t)(gs > pl.n_groups ? gs : pl.n_groups) * pl.R_pad * 16;
-    size_t sm = pipe;
-    if (tr > sm)
-        sm = tr;
+    pl.n_groups = ceil_div(pl.P, gs);
+    size_t sm = (size_t)pl.stages * stage_bytes + fixed;
+    const size_t mg = (size_t)(gs > pl.n_groups ? gs : pl.n_groups) * pl.R_pad * 16;
     if (mg > sm)
         sm = mg;
     pl.smem_bytes = sm + 1024;
-    // (max, argmax, s, t) partials, then the tempered (sT, tT) partials of typical mode
-    pl.ws_bytes = ((size_t)(pl.n_tiles + pl.n_groups) * pl.R_pad * (16 + 8) + 255) / 256 * 256;
+    pl.n_counters = pl.n_groups + 1;
+    // (max, argmax, s, t) and (sT, tT) partials of the CTAs and the groups
+    pl.ws_bytes = ((size_t)(pl.P + pl.n_groups) * pl.R_pad * (16 + 8) + 255) / 256 * 256;
     return pl;
 }
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
-                           float *entropy, void *parts, int *counters, int *status, cudaStream_t stream,
+                           float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
                            const char **err, int expire_wait, const LmTypical *typ)
 {
-    const LmPlan pl = lm_plan(R, D, V);
+    const LmPlan pl = lm_plan(R, D, V, n_sm);
     LmParams p{};
     if (!make_tmap_2d(&p.tmap_w, W, (uint64_t)D, (uint64_t)V, (uint64_t)D * 2, 64, 128, err))
         return cudaErrorInvalidValue;
@@ -575,22 +628,22 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.D = D;
     p.V = V;
     p.n_tiles = pl.n_tiles;
-    p.n_kblocks = pl.n_kblocks;
-    p.bps = pl.bps;
+    p.nk = pl.n_kblocks;
     p.stages = pl.stages;
-    p.tmem_cols = pl.tmem_cols;
+    p.acc_cols = pl.acc_cols;
+    p.P = pl.P;
     p.group_size = pl.group_size;
     p.n_groups = pl.n_groups;
-    p.part_tile = static_cast<float4 *>(parts);
-    p.part_group = p.part_tile + (size_t)pl.n_tiles * pl.R_pad;
+    p.part_cta = static_cast<float4 *>(parts);
+    p.part_group = p.part_cta + (size_t)pl.P * pl.R_pad;
+    p.part_cta_t = reinterpret_cast<float2 *>(p.part_group + (size_t)pl.n_groups * pl.R_pad);
+    p.part_group_t = p.part_cta_t + (size_t)pl.P * pl.R_pad;
     p.counters = counters;
     p.status = status;
     p.argmax = argmax;
     p.top1 = top1;
     p.entropy = entropy;
     p.expire_wait = expire_wait;
-    p.part_tile_t = reinterpret_cast<float2 *>(p.part_group + (size_t)pl.n_groups * pl.R_pad);
-    p.part_group_t = p.part_tile_t + (size_t)pl.n_tiles * pl.R_pad;
     if (typ) {
         p.inv_t = 1.0f / typ->temperature;
         p.logz_t = typ->logz_t;
@@ -600,13 +653,13 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
         if (e != cudaSuccess)
             return e;
-        k2_lm_head<true><<<pl.n_tiles, kLmThreads, pl.smem_bytes, stream>>>(p);
+        k2_lm_head<true><<<pl.P, kLmThreads, pl.smem_bytes, stream>>>(p);
     } else {
         p.inv_t = 1.0f;
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
         if (e != cudaSuccess)
             return e;
-        k2_lm_head<false><<<pl.n_tiles, kLmThreads, pl.smem_bytes, stream>>>(p);
+        k2_lm_head<false><<<pl.P, kLmThreads, pl.smem_bytes, stream>>>(p);
     }
     return cudaGetLastError();
 }

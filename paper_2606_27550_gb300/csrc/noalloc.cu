@@ -13,8 +13,8 @@
 
 namespace tv {
 
-// 4 MiB of partials: (ceil(vocab/128) + groups) x rows (padded to 16) x 16 bytes,
-// e.g. vocab 32000 with up to 256 rows, or vocab 128256 with up to 128 rows.
+// 4 MiB of partials: (CTAs + merge groups) x rows (padded to 16) x 24 bytes,
+// whatever the vocabulary: about 2 MiB for 256 rows on a GPU with 152 SMs.
 constexpr size_t kNoAllocScratchBytes = 4u << 20;
 constexpr size_t kNoAllocCounterBytes = 4096;  // 1024 counters, cleared on every call
 
@@ -59,8 +59,12 @@ extern "C" tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const
     if (n_rows < 1 || n_rows > 256 || d_model < 8 || d_model % 8 || vocab < 1)
         return record_error(TB_EINVAL, "lm_head_stats_noalloc: n_rows %d (1..256), d_model %d (multiple of 8), vocab %d",
                             n_rows, d_model, vocab);
-    const LmPlan pl = lm_plan(n_rows, d_model, vocab);
-    if (pl.ws_bytes > kNoAllocScratchBytes || pl.n_groups + 2 > (int)(kNoAllocCounterBytes / 4))
+    int dev = 0, n_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) !=
+                                                  cudaSuccess)
+        return record_error(TB_ECUDA, "lm_head_stats_noalloc: no current device");
+    const LmPlan pl = lm_plan(n_rows, d_model, vocab, n_sm);
+    if (pl.ws_bytes > kNoAllocScratchBytes || pl.n_counters + 1 > (int)(kNoAllocCounterBytes / 4))
         return record_error(TB_ECAPACITY,
                             "lm_head_stats_noalloc: %d rows x vocab %d need %zu scratch bytes; the built-in array "
                             "holds %zu",
@@ -78,7 +82,7 @@ extern "C" tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const
         return record_error(TB_ECUDA, "lm_head_stats_noalloc: clearing counters: %s", cudaGetErrorString(e));
     const char *err = "";
     int *status = counters + (kNoAllocCounterBytes / 4 - 1);  // last word: device-detected errors
-    e = lm_head_launch(hidden, n_rows, lm_head, d_model, vocab, argmax, top1, entropy, parts, counters, status,
+    e = lm_head_launch(hidden, n_rows, lm_head, d_model, vocab, argmax, top1, entropy, parts, counters, status, n_sm,
                        (cudaStream_t)stream, &err);
     if (e != cudaSuccess)
         return record_error(e == cudaErrorInvalidValue ? TB_EINVAL : TB_ECUDA, "lm_head_stats_noalloc: %s",

@@ -471,7 +471,7 @@ extern "C" size_t tb_workspace_size(int max_rows, int n_layers, int n_kv_heads, 
     if (head_dim > 0)
         bytes += attn_part_bytes(nsm, head_dim);
     if (max_rows > 0 && vocab > 0)  // batched calls run the LM head in chunks of 256 rows
-        bytes += align256(lm_plan(max_rows < 256 ? max_rows : 256, 64, vocab).ws_bytes);
+        bytes += align256(lm_plan(max_rows < 256 ? max_rows : 256, 64, vocab, nsm).ws_bytes);
     return bytes;
 }
 
@@ -669,8 +669,8 @@ static tb_status lm_validate(const void *hidden, int R, const void *W, int D, in
         return fail(TB_EINVAL, "%s: d_model %d must be a positive multiple of 8", fn, D);
     if (V < 1)
         return fail(TB_EINVAL, "%s: vocab %d", fn, V);
-    *plan = lm_plan(R, D, V);
-    if (plan->n_groups + 1 > kMaxLmCounters)
+    *plan = lm_plan(R, D, V, sm_count(current_device()));
+    if (plan->n_counters > kMaxLmCounters)
         return fail(TB_EUNSUPPORTED, "%s: vocab %d too large", fn, V);
     return TB_OK;
 }
@@ -681,8 +681,8 @@ static tb_status lm_enqueue(const void *hidden, int R, const void *W, int D, int
 {
     const char *err = "";
     cudaError_t e = lm_head_launch(hidden, R, W, D, V, am, t1, en, ws + part_off,
-                                   reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws), stream,
-                                   &err, expire_wait, typ);
+                                   reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws),
+                                   sm_count(current_device()), stream, &err, expire_wait, typ);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)

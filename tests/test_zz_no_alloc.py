@@ -32,8 +32,11 @@ def built():
     torch.cuda.set_device(0)
 
 
-@pytest.mark.parametrize("R,D,V", [(64, 4096, 32000), (7, 256, 1000)])
+@pytest.mark.parametrize("R,D,V", [(64, 4096, 32000), (7, 256, 1000), (256, 64, 200000)])
 def test_noalloc_matches_workspace_entry_point(built, R, D, V):
+    """The same kernel and plan run in both: the outputs are identical.  The
+    scratch is one partial per CTA and per merge group, whatever the vocabulary,
+    so the widest rows with a 200000-entry vocabulary fit the built-in array."""
     W = _dev(synth.gen_lm_head(31 + V, V, D))
     outs = []
     for call in range(3):  # call 0: reference entry point; calls 1, 2: no-alloc variant, back to back
@@ -49,20 +52,8 @@ def test_noalloc_matches_workspace_entry_point(built, R, D, V):
         torch.cuda.synchronize()
         outs.append((am.cpu().numpy(), t1.cpu().numpy(), en.cpu().numpy()))
     ref = outs[0]
+    assert np.all(ref[0] >= 0) and np.all(ref[0] < V)
+    assert np.all(ref[1] > 0) and np.all(ref[1] <= 1) and np.all(ref[2] >= -STAT_TOL)
     for got in outs[1:]:
-        assert np.array_equal(got[0], ref[0])
-        assert np.abs(got[1] - ref[1]).max() <= STAT_TOL
-        assert np.abs(got[2] - ref[2]).max() <= STAT_TOL
-        assert np.all(got[0] >= 0) and np.all(got[0] < V)
-
-
-def test_noalloc_rejects_oversized_scratch(built):
-    R, D, V = 256, 64, 200000  # needs more partial scratch than the built-in array holds
-    h = torch.zeros((R, D), dtype=torch.bfloat16, device="cuda")
-    W = torch.zeros((V, D), dtype=torch.bfloat16, device="cuda")
-    o = torch.empty(R, dtype=torch.int32, device="cuda")
-    f = torch.empty(R, dtype=torch.float32, device="cuda")
-    with pytest.raises(tv.TreeVerifyError) as e:
-        tv.lm_head_stats_noalloc(h, W, o, f, f)
-    assert e.value.status == tv.TB_ECAPACITY
-    assert "built-in array" in str(e.value)
+        for x, y in zip(got, ref):
+            assert np.array_equal(x, y)
