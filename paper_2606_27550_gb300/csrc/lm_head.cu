@@ -13,8 +13,9 @@
 // ([128][64] bf16 per k-block, 128-byte swizzled by TMA) is the MMA's M=128 A
 // operand, the tree rows ([R_pad][64], same swizzle) the N = R_pad B operand;
 // tcgen05.mma (kind::f16, f32 accumulate) builds the 128 x R_pad logit tile in
-// TMEM.  Warp 0 lane 0 issues TMA into a ring that runs across tiles, warp 1
-// lane 0 the MMAs into one of two TMEM accumulators, and warps 2-9 drain the
+// TMEM.  Lane 0 of warps 0 and 10 issue TMA (alternate stages) into a ring
+// that runs across tiles, warp 1 lane 0 the MMAs into one of two TMEM
+// accumulators, and warps 2-9 drain the
 // other accumulator meanwhile (32 tree rows at a time: TMEM -> shared memory
 // transposed -> eight threads per row reduce its 128 logits), folding each
 // tile into per-row running statistics of the CTA.  The CTAs' statistics are
@@ -65,10 +66,12 @@ struct RowStat {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// Threads per CTA: warp 0 lane 0 issues TMA, warp 1 lane 0 the MMAs, warps
-// 2-9 form the epilogue (warps w and w + 4 read the same TMEM lane quadrant
-// w % 4 and split each 32-row chunk's columns); all ten merge at the end.
-constexpr int kLmThreads = 320;
+// Threads per CTA: lane 0 of warps 0 and 10 issue TMA, warp 1 lane 0 the
+// MMAs, warps 2-9 form the epilogue (warps w and w + 4 read the same TMEM
+// lane quadrant w % 4 and split each 32-row chunk's columns); all eleven merge
+// at the end.
+constexpr int kLmThreads = 352;
+constexpr int kLmProducer2 = 10;
 constexpr int kEpiThreads = 256;
 constexpr int kLmChunk = 32;             // tree rows per epilogue chunk
 constexpr int kLmTpr = kEpiThreads / kLmChunk;  // threads per row in the chunk scans
@@ -335,14 +338,19 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    if (warp == 0) {
-        // ---------------- TMA producer: one stage = one 64-column box of W
-        // (128 rows) and of the tree rows; the ring runs across the range's tiles
+    if (warp == 0 || warp == kLmProducer2) {
+        // ---------------- TMA producers: one stage = one 64-column box of W
+        // (128 rows) and of the tree rows; the ring runs across the run's tiles.
+        // Warp 0 fills the even stages of the sequence, the last warp the odd
+        // ones: one issuing thread alone streams W measurably slower.
         if (lane == 0) {
-            long long g = 0;
+            const long long mine = warp == 0 ? 0 : 1;
+            long long g = 0, g_end = 0;
             bool ok = true;
             for (int tile = tile0; tile < tile1 && ok; ++tile) {
                 for (int j = 0; j < p.nk; ++j, ++g) {
+                    if ((g & 1) != mine)
+                        continue;
                     const int kb = lm_kb(p, tile, j);
                     const int s = (int)(g % S);
                     if (!mbar_wait_bounded(&empty_bar[s], ((uint32_t)(g / S) & 1u) ^ 1u, &abort_flag, p.status)) {
@@ -352,11 +360,13 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                     mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
                     tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
                     tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                    g_end = g + 1;
                 }
             }
-            if (!ok)  // gave up: the copies in flight land before the CTA exits
-                for (long long it = (g > S ? g - S : 0); it < g; ++it)
-                    mbar_wait_drain(&full_bar[it % S], (uint32_t)(it / S) & 1u);
+            if (!ok)  // gave up: this thread's copies in flight land before the CTA exits
+                for (long long it = (g_end > S ? g_end - S : 0); it < g_end; ++it)
+                    if ((it & 1) == mine)
+                        mbar_wait_drain(&full_bar[it % S], (uint32_t)(it / S) & 1u);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer: the CTA's i-th tile accumulates into TMEM buffer i & 1
@@ -394,7 +404,7 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
             tc_commit(&drain_bar);
         }
-    } else {
+    } else if (warp < kLmProducer2) {
         // ---------------- epilogue (warps 2-9)
         const int e = threadIdx.x - 64;
         const int q = warp & 3, half = (warp - 2) >> 2;
