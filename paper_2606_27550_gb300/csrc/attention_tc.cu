@@ -17,12 +17,14 @@
 //                 is the TMEM A operand, the V tile an MN-major shared-memory
 //                 operand; O accumulates in TMEM.
 //
-// One CTA per SM, 6 warps:
+// One CTA per SM, 7 warps:
 //   warp 0       TMA producer: 128-key K and V tiles (4 boxes of 64 x 128)
 //                through a 3-stage mbarrier ring.
-//   warp 1       TMEM allocation (512 columns) and the single MMA-issuing
-//                thread; S of tile i+1 is issued before O += P V of tile i so
-//                that the softmax of tile i overlaps the next QK^T.
+//   warp 1       TMEM allocation (512 columns) and the QK^T-issuing thread;
+//                S is double-buffered, so the softmax of tile i overlaps
+//                QK^T of tile i+1.
+//   warp 6       the P V-issuing thread (O += P V of tile i as soon as P is
+//                written; it releases the tile's stage).
 //   warps 2-5    one thread per query row (TMEM lane): row max, exp2 with a
 //                lazily rescaled reference maximum (O and l are rescaled only
 //                when the maximum grows by more than 2^8), P written back to
@@ -46,6 +48,7 @@ constexpr int kStages = 3;
 constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
 constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
 constexpr int kStage = 2 * kTile;  // K + V
+constexpr int kTcThreads = 224;    // 7 warps: TMA, QK^T issuer, 4 softmax, P V issuer
 constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
 // TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
 // softmax has read S_b into registers; Q (bf16 pairs) is the A operand of QK^T.
@@ -140,7 +143,7 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t l
 }  // namespace
 
 template <bool kBatched>
-__global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
+__global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
@@ -181,7 +184,7 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
         }
         mbar_init(&q_full, 4);
         mbar_init(&o_free, 4);
-        mbar_init(&drain_bar, 1);
+        mbar_init(&drain_bar, 2);  // one commit from each MMA issuer
         abort_flag = 0;
         fence_mbar_init();
         for (int b = 0; b < (kBatched ? p.n_seq : 1); ++b) {
@@ -231,37 +234,11 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                     mbar_wait_drain(&full_bar[it % kStages], (uint32_t)(it / kStages) & 1u);
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+        // ------------------------------------------------------------ QK^T issuer
         if (lane == 0) {
             const uint32_t idesc_s = idesc_bf16_f32(128, kBN);
-            const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
-            int sg = -1;
-            // the pending O += P V (tile it - 1)
-            bool pend = false, pend_first = false;
-            int pend_sg = 0;
-            long long pend_it = 0;
-            bool ok = true;
-            auto issue_pv = [&](long long j, bool first, int seg) -> bool {
-                const int bj = (int)(j & 1);
-                if (!mbar_wait_bounded(&p_full[bj], (uint32_t)(j >> 1) & 1u, &abort_flag, p.status))
-                    return false;
-                if (first && seg > 0 &&
-                    !mbar_wait_bounded(&o_free, (uint32_t)(seg - 1) & 1u, &abort_flag, p.status))
-                    return false;
-                tc_fence_after();
-                const uint32_t v_base = smem_u32(sKV + (size_t)(j % kStages) * kStage + kTile);
-                const uint32_t p_col = bj ? kColP1 : kColP0;
-#pragma unroll
-                for (int ks = 0; ks < kBN / 16; ++ks) {
-                    const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
-                    tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
-                }
-                tc_commit(&empty_bar[j % kStages]);
-                tc_commit(&pv_done[bj]);
-                return true;
-            };
-            int sb = 0;
-            for (long long it = 0; it < n_tiles && ok; ++it) {
+            int sg = -1, sb = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
                 const long long t = t0 + it;
                 sb = seq_at<kBatched>(p, t, sb);
                 const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
@@ -269,20 +246,14 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                     ++sg;
                 const int s = (int)(it % kStages);
                 const int b = (int)(it & 1);
-                if (first && pend) {
-                    // finish the previous unit first: its epilogue frees O for this one
-                    if (!issue_pv(pend_it, pend_first, pend_sg)) {
-                        ok = false;
-                        break;
-                    }
-                    pend = false;
-                }
+                // K landed; the softmax has read S_b (tile it - 2) and P V(it - 2) has read
+                // the P that shares its columns; at a segment's first tile, its Q is staged
                 if (!mbar_wait_bounded(&full_bar[s], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status) ||
                     !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
-                    (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status))) {
-                    ok = false;
+                    (it >= 2 &&
+                     !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) ||
+                    (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status)))
                     break;
-                }
                 tc_fence_after();
                 const uint32_t k_base = smem_u32(sKV + (size_t)s * kStage);
                 const uint32_t s_col = b ? kColS1 : kColS0;
@@ -293,18 +264,42 @@ __global__ void __launch_bounds__(192, 1) k1_tree_attention_tc(const __grid_cons
                     tc_mma_f16_ts(tmem + s_col, tmem + kColQ + kk * 8, bdesc, idesc_s, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[b]);
-                if (pend && !issue_pv(pend_it, pend_first, pend_sg)) {
-                    ok = false;
-                    break;
-                }
-                pend = true;
-                pend_it = it;
-                pend_first = first;
-                pend_sg = sg;
             }
-            if (ok && pend)
-                issue_pv(pend_it, pend_first, pend_sg);
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
+            tc_commit(&drain_bar);
+        }
+    } else if (warp == 6) {
+        // ------------------------------------------------------------ P V issuer
+        // A second issuing thread: each tcgen05.mma holds its issuer for about
+        // 100 cycles at these shapes, so P V(i) issued here runs alongside
+        // QK^T(i + 1) instead of queueing behind it, and the stage is released
+        // that much sooner.
+        if (lane == 0) {
+            const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
+            int sg = -1, sb = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
+                const long long t = t0 + it;
+                sb = seq_at<kBatched>(p, t, sb);
+                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
+                if (first)
+                    ++sg;
+                const int b = (int)(it & 1);
+                // P written; at a segment's first tile, the previous epilogue has read O
+                if (!mbar_wait_bounded(&p_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status) ||
+                    (first && sg > 0 &&
+                     !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)))
+                    break;
+                tc_fence_after();
+                const uint32_t v_base = smem_u32(sKV + (size_t)(it % kStages) * kStage + kTile);
+                const uint32_t p_col = b ? kColP1 : kColP0;
+#pragma unroll
+                for (int ks = 0; ks < kBN / 16; ++ks) {
+                    const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
+                    tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
+                }
+                tc_commit(&empty_bar[it % kStages]);
+                tc_commit(&pv_done[b]);
+            }
             tc_commit(&drain_bar);
         }
     } else {
@@ -784,7 +779,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     if (n_seq == 1) {
         if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
             return e;
-        k1_tree_attention_tc<false><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+        k1_tree_attention_tc<false><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return e;
         if (p.P > 1)
@@ -792,7 +787,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     } else {
         if ((e = allow_max_smem((const void *)k1_tree_attention_tc<true>)) != cudaSuccess)
             return e;
-        k1_tree_attention_tc<true><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+        k1_tree_attention_tc<true><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
         if ((e = cudaGetLastError()) != cudaSuccess)
             return e;
         if (p.P > 1)
@@ -844,7 +839,7 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
     cudaError_t e;
     if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
         return e;
-    k1_tree_attention_tc<false><<<p.P, 192, tc_smem_bytes(), stream>>>(p);
+    k1_tree_attention_tc<false><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
     if ((e = cudaGetLastError()) != cudaSuccess)
         return e;
     if (p.P > 1)
