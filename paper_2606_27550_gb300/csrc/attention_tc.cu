@@ -48,7 +48,7 @@ constexpr int kStages = 3;
 constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
 constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
 constexpr int kStage = 2 * kTile;  // K + V
-constexpr int kTcThreads = 224;    // 7 warps: TMA, QK^T issuer, 4 softmax, P V issuer
+constexpr int kTcThreads = 256;    // 8 warps: K loads, QK^T issuer, 4 softmax, P V issuer, V loads
 constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
 // TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
 // softmax has read S_b into registers; Q (bf16 pairs) is the A operand of QK^T.
@@ -146,7 +146,7 @@ template <bool kBatched>
 __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
     __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
     __shared__ __align__(8) uint64_t q_full, o_free, drain_bar;
     __shared__ uint32_t tmem_slot;
@@ -173,8 +173,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full_bar[s], 1);
-            mbar_init(&empty_bar[s], 1);
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
@@ -201,15 +203,20 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
+    if (warp == 0 || warp == 7) {
+        // ------------------------------------------------------------ TMA producers
+        // warp 0 streams the K tiles, warp 7 the V tiles, each through its own
+        // half of the 3-stage ring: QK^T releases a K slot, P V a V slot.
         if (lane == 0) {
+            const bool is_v = (warp == 7);
+            uint64_t *full = is_v ? v_full : k_full;
+            uint64_t *empty = is_v ? v_empty : k_empty;
             long long issued = 0;
             int sb = 0;
             for (long long it = 0; it < n_tiles; ++it) {
                 const int s = (int)(it % kStages);
                 const uint32_t ph = (uint32_t)(it / kStages) & 1u;
-                if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status))
+                if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
                     break;
                 const long long t = t0 + it;
                 sb = seq_at<kBatched>(p, t, sb);
@@ -219,19 +226,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 const int j = (int)(tl % sq.T);
                 const int head = (u / sq.row_blocks) % p.Hkv;
                 const int layer = p.layer_begin + u / (sq.row_blocks * p.Hkv);
-                const CUtensorMap *mk = &p.tmap[2 * sb], *mv = &p.tmap[2 * sb + 1];
-                uint8_t *sk = sKV + (size_t)s * kStage;
-                uint8_t *sv = sk + kTile;
-                mbar_arrive_expect_tx(&full_bar[s], kStage);
-                tma_load_4d(sk, mk, &full_bar[s], 0, j * kBN, head, layer);
-                tma_load_4d(sk + kAtom, mk, &full_bar[s], 64, j * kBN, head, layer);
-                tma_load_4d(sv, mv, &full_bar[s], 0, j * kBN, head, layer);
-                tma_load_4d(sv + kAtom, mv, &full_bar[s], 64, j * kBN, head, layer);
+                const CUtensorMap *m = &p.tmap[2 * sb + (is_v ? 1 : 0)];
+                uint8_t *dst = sKV + (size_t)s * kStage + (is_v ? kTile : 0);
+                mbar_arrive_expect_tx(&full[s], kTile);
+                tma_load_4d(dst, m, &full[s], 0, j * kBN, head, layer);
+                tma_load_4d(dst + kAtom, m, &full[s], 64, j * kBN, head, layer);
                 issued = it + 1;
             }
             if (issued < n_tiles)
                 for (long long it = (issued > kStages ? issued - kStages : 0); it < issued; ++it)
-                    mbar_wait_drain(&full_bar[it % kStages], (uint32_t)(it / kStages) & 1u);
+                    mbar_wait_drain(&full[it % kStages], (uint32_t)(it / kStages) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ QK^T issuer
@@ -248,7 +252,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 const int b = (int)(it & 1);
                 // K landed; the softmax has read S_b (tile it - 2) and P V(it - 2) has read
                 // the P that shares its columns; at a segment's first tile, its Q is staged
-                if (!mbar_wait_bounded(&full_bar[s], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status) ||
+                if (!mbar_wait_bounded(&k_full[s], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status) ||
                     !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
                     (it >= 2 &&
                      !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) ||
@@ -264,6 +268,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     tc_mma_f16_ts(tmem + s_col, tmem + kColQ + kk * 8, bdesc, idesc_s, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[b]);
+                tc_commit(&k_empty[s]);
             }
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
             tc_commit(&drain_bar);
@@ -287,7 +292,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 // P written; at a segment's first tile, the previous epilogue has read O
                 if (!mbar_wait_bounded(&p_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status) ||
                     (first && sg > 0 &&
-                     !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)))
+                     !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)) ||
+                    !mbar_wait_bounded(&v_full[it % kStages], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status))
                     break;
                 tc_fence_after();
                 const uint32_t v_base = smem_u32(sKV + (size_t)(it % kStages) * kStage + kTile);
@@ -297,12 +303,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
                     tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
                 }
-                tc_commit(&empty_bar[it % kStages]);
+                tc_commit(&v_empty[it % kStages]);
                 tc_commit(&pv_done[b]);
             }
             tc_commit(&drain_bar);
         }
-    } else {
+    } else if (warp < 6) {
         // ------------------------------------------------------------ softmax / epilogue (warps 2-5)
         const int q4 = warp & 3;  // TMEM lane quadrant of this warp
         const uint32_t lane_addr = tmem + ((uint32_t)(32 * q4) << 16);
