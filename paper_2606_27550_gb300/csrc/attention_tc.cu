@@ -17,9 +17,11 @@
 //                 is the TMEM A operand, the V tile an MN-major shared-memory
 //                 operand; O accumulates in TMEM.
 //
-// One CTA per SM, 7 warps:
-//   warp 0       TMA producer: 128-key K and V tiles (4 boxes of 64 x 128)
-//                through a 3-stage mbarrier ring.
+// One CTA per SM, 8 warps:
+//   warps 0, 7   TMA producers: 128-key K tiles (warp 0) and V tiles (warp 7),
+//                two boxes of 64 x 128 each, through separate 3-stage rings:
+//                QK^T releases a K slot, P V a V slot, so the next K tiles
+//                never wait for a P V.
 //   warp 1       TMEM allocation (512 columns) and the QK^T-issuing thread;
 //                S is double-buffered, so the softmax of tile i overlaps
 //                QK^T of tile i+1.
@@ -44,10 +46,11 @@ namespace {
 
 constexpr int kD = 128;            // head_dim
 constexpr int kBN = 128;           // keys per tile
-constexpr int kStages = 3;
+constexpr int kKStages = 3;        // K ring depth
+constexpr int kVStages = 3;        // V ring depth
+constexpr int kMaxStages = kKStages > kVStages ? kKStages : kVStages;
 constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
 constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
-constexpr int kStage = 2 * kTile;  // K + V
 constexpr int kTcThreads = 256;    // 8 warps: K loads, QK^T issuer, 4 softmax, P V issuer, V loads
 constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
 // TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
@@ -146,7 +149,7 @@ template <bool kBatched>
 __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t k_full[kStages], k_empty[kStages], v_full[kStages], v_empty[kStages];
+    __shared__ __align__(8) uint64_t k_full[kMaxStages], k_empty[kMaxStages], v_full[kMaxStages], v_empty[kMaxStages];
     __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
     __shared__ __align__(8) uint64_t q_full, o_free, drain_bar;
     __shared__ uint32_t tmem_slot;
@@ -155,7 +158,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
     __shared__ long long s_total;
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sKV = smem;
+    uint8_t *sK = smem;                                // K ring: kKStages tiles
+    uint8_t *sV = smem + (size_t)kKStages * kTile;     // V ring: kVStages tiles
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
@@ -172,7 +176,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
     const long long n_tiles = t1 - t0;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < kMaxStages; ++s) {
             mbar_init(&k_full[s], 1);
             mbar_init(&k_empty[s], 1);
             mbar_init(&v_full[s], 1);
@@ -211,11 +215,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             const bool is_v = (warp == 7);
             uint64_t *full = is_v ? v_full : k_full;
             uint64_t *empty = is_v ? v_empty : k_empty;
+            const int S = is_v ? kVStages : kKStages;
+            uint8_t *ring = is_v ? sV : sK;
             long long issued = 0;
             int sb = 0;
             for (long long it = 0; it < n_tiles; ++it) {
-                const int s = (int)(it % kStages);
-                const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+                const int s = (int)(it % S);
+                const uint32_t ph = (uint32_t)(it / S) & 1u;
                 if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
                     break;
                 const long long t = t0 + it;
@@ -227,15 +233,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 const int head = (u / sq.row_blocks) % p.Hkv;
                 const int layer = p.layer_begin + u / (sq.row_blocks * p.Hkv);
                 const CUtensorMap *m = &p.tmap[2 * sb + (is_v ? 1 : 0)];
-                uint8_t *dst = sKV + (size_t)s * kStage + (is_v ? kTile : 0);
+                uint8_t *dst = ring + (size_t)s * kTile;
                 mbar_arrive_expect_tx(&full[s], kTile);
                 tma_load_4d(dst, m, &full[s], 0, j * kBN, head, layer);
                 tma_load_4d(dst + kAtom, m, &full[s], 64, j * kBN, head, layer);
                 issued = it + 1;
             }
             if (issued < n_tiles)
-                for (long long it = (issued > kStages ? issued - kStages : 0); it < issued; ++it)
-                    mbar_wait_drain(&full[it % kStages], (uint32_t)(it / kStages) & 1u);
+                for (long long it = (issued > S ? issued - S : 0); it < issued; ++it)
+                    mbar_wait_drain(&full[it % S], (uint32_t)(it / S) & 1u);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ QK^T issuer
@@ -248,18 +254,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
                 if (first)
                     ++sg;
-                const int s = (int)(it % kStages);
+                const int s = (int)(it % kKStages);
                 const int b = (int)(it & 1);
                 // K landed; the softmax has read S_b (tile it - 2) and P V(it - 2) has read
                 // the P that shares its columns; at a segment's first tile, its Q is staged
-                if (!mbar_wait_bounded(&k_full[s], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status) ||
+                if (!mbar_wait_bounded(&k_full[s], (uint32_t)(it / kKStages) & 1u, &abort_flag, p.status) ||
                     !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
                     (it >= 2 &&
                      !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) ||
                     (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status)))
                     break;
                 tc_fence_after();
-                const uint32_t k_base = smem_u32(sKV + (size_t)s * kStage);
+                const uint32_t k_base = smem_u32(sK + (size_t)s * kTile);
                 const uint32_t s_col = b ? kColS1 : kColS0;
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
@@ -293,17 +299,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 if (!mbar_wait_bounded(&p_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status) ||
                     (first && sg > 0 &&
                      !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)) ||
-                    !mbar_wait_bounded(&v_full[it % kStages], (uint32_t)(it / kStages) & 1u, &abort_flag, p.status))
+                    !mbar_wait_bounded(&v_full[it % kVStages], (uint32_t)(it / kVStages) & 1u, &abort_flag, p.status))
                     break;
                 tc_fence_after();
-                const uint32_t v_base = smem_u32(sKV + (size_t)(it % kStages) * kStage + kTile);
+                const uint32_t v_base = smem_u32(sV + (size_t)(it % kVStages) * kTile);
                 const uint32_t p_col = b ? kColP1 : kColP0;
 #pragma unroll
                 for (int ks = 0; ks < kBN / 16; ++ks) {
                     const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
                     tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
                 }
-                tc_commit(&v_empty[it % kStages]);
+                tc_commit(&v_empty[it % kVStages]);
                 tc_commit(&pv_done[b]);
             }
             tc_commit(&drain_bar);
@@ -695,7 +701,7 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
 
 static size_t tc_smem_bytes()
 {
-    return (size_t)kStages * kStage + 1024;
+    return (size_t)(kKStages + kVStages) * kTile + 1024;
 }
 
 bool attn_tc_supported(int d, int rows)
