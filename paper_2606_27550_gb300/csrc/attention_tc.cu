@@ -56,6 +56,7 @@ constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], 
 // TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
 // softmax has read S_b into registers; Q (bf16 pairs) is the A operand of QK^T.
 constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 0, kColP1 = 128, kColO = 256, kColQ = 384;
+constexpr int kQPrefetchTiles = 3;  // tiles before a segment's end at which the next unit's q rows are prefetched
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
 
 // One sequence of a (possibly batched) launch: its own KV cache (tensor maps),
@@ -419,6 +420,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             float m_ref = -INFINITY, l = 0.f;
             for (long long t = g.start; t < g.end; ++t, ++it) {
                 const int b = (int)(it & 1);
+                if (t + kQPrefetchTiles == g.end && g.end < t1) {
+                    // the next unit's query rows are read from HBM when this segment ends
+                    // (write_q below): ask for them in L2 a few tiles ahead
+                    const Seg nx = describe(g.end);
+                    if (nx.valid) {
+                        const char *row = reinterpret_cast<const char *>(
+                            nx.q + (((size_t)nx.layer_rel * nx.ns + nx.node) * p.Hq + nx.qh) * kD);
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(row));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(row + 128));
+                    }
+                }
                 if (!mbar_wait_bounded(&s_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status)) {
                     aborted = true;
                     break;
