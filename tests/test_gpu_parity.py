@@ -106,7 +106,10 @@ def test_tree_attention_large_L_multilayer(dev, bank):
 
 
 LM_CASES = [(1, 256, 1000), (7, 256, 1000), (26, 4096, 4099), (64, 4096, 32000), (200, 512, 3000), (256, 256, 129),
-            (232, 256, 4099)]
+            (232, 256, 4099),
+            # several vocab tiles per persistent CTA (both TMEM accumulators reused), two CTAs
+            # per SM for narrow rows and one for wide rows, ragged last tiles
+            (26, 256, 128256), (232, 64, 60001), (100, 128, 50001)]
 
 
 @pytest.mark.parametrize("R,D,V", LM_CASES)

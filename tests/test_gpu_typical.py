@@ -57,6 +57,7 @@ LM_CASES = [
     (synth.bank_trees()[-1], 512, 4099, 1.3),   # 64 rows, ragged last vocab tile
     ([-1], 128, 129, 0.7),                      # single node: no edges to gather
     (synth.chain(17), 320, 2000, 0.25),
+    (synth.bank_trees()[-1], 128, 100003, 0.7),  # several vocab tiles per persistent CTA
 ]
 
 
