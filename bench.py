@@ -211,16 +211,17 @@ def run_gpu(args):
         lgs = torch.empty((N + 1, V), dtype=torch.float32, device=dev)
         del zf
 
-    def step(qq=q, hh=hidden, dd=drafts, st=None):
+    def step(qq=q, hh=hidden, dd=drafts, st=None, outs=None):
         st = stream if st is None else st
+        oam, ot1, oen, ores = (am, t1, en, res) if outs is None else outs
         if sampled:
-            tv.verify_step_sampled(bank, bid, kv, qq, hh, W, dd, qd, unif, 0.7, out, am, t1, en, lgs, res, ws,
+            tv.verify_step_sampled(bank, bid, kv, qq, hh, W, dd, qd, unif, 0.7, out, oam, ot1, oen, lgs, ores, ws,
                                    0, st)
         elif typical:
-            tv.verify_step_typical(bank, bid, kv, qq, hh, W, dd, out, am, t1, en, res, ws, *tv.PAPER_TYPICAL,
+            tv.verify_step_typical(bank, bid, kv, qq, hh, W, dd, out, oam, ot1, oen, ores, ws, *tv.PAPER_TYPICAL,
                                    0, st)
         else:
-            tv.verify_step(bank, bid, kv, qq, hh, W, dd, out, am, t1, en, res, ws, 0, st)
+            tv.verify_step(bank, bid, kv, qq, hh, W, dd, out, oam, ot1, oen, ores, ws, 0, st)
 
     visible = os.environ.get("CUDA_VISIBLE_DEVICES")
     sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
@@ -275,15 +276,20 @@ def run_gpu(args):
     # end to end: every step copies its inputs from pinned host memory and reads its result
     # back with a host synchronisation.  Inputs are double-buffered: step i + 1's copy runs on
     # a copy stream while step i computes (events keep a buffer from being overwritten while
-    # a step still reads it); each buffer's verify_step call is captured once into a CUDA
-    # graph, so the host enqueues one replay per step.
+    # a step still reads it).  The step's outputs (result, argmax, top-1, entropy) sit in one
+    # device block, read back by one copy; each buffer's verify_step call and that copy are
+    # captured once into a CUDA graph, so the host enqueues one replay per step, before it
+    # queues the next step's upload.
     q_h = torch.empty(q.shape, dtype=bf, pin_memory=True).copy_(q)
     h_h = torch.empty(hidden.shape, dtype=bf, pin_memory=True).copy_(hidden)
     d_h = torch.empty(drafts.shape, dtype=torch.int32, pin_memory=True).copy_(drafts)
-    res_h = torch.empty(res.shape, dtype=torch.int32, pin_memory=True)
-    stats_h = torch.empty((3, N), dtype=torch.float32, pin_memory=True)
+    RI = tv.RESULT_INTS
+    blk = torch.zeros(RI + 3 * N, dtype=torch.int32, device=dev)
+    outs_e = (blk[RI:RI + N], blk[RI + N:RI + 2 * N].view(torch.float32), blk[RI + 2 * N:].view(torch.float32),
+              blk[:RI])
+    blk_h = [torch.empty(blk.shape, dtype=torch.int32, pin_memory=True) for _ in range(2)]
     h2d = q_h.numel() * 2 + h_h.numel() * 2 + d_h.numel() * 4
-    d2h = res_h.numel() * 4 + stats_h.numel() * 4
+    d2h = blk.numel() * 4
     bufs = [(q, hidden, drafts), (torch.empty_like(q), torch.empty_like(hidden), torch.empty_like(drafts))]
     copy_stream = torch.cuda.Stream()
     ev_copied = [torch.cuda.Event(), torch.cuda.Event()]
@@ -304,7 +310,8 @@ def run_gpu(args):
     for b in range(2):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=cap):
-            step(*bufs[b], st=cap)
+            step(*bufs[b], st=cap, outs=outs_e)
+            blk_h[b].copy_(blk, non_blocking=True)
         graphs.append(g)
     torch.cuda.synchronize()
     for b in range(2):
@@ -316,17 +323,13 @@ def run_gpu(args):
     upload(0)
     for i in range(n_e2e):
         b = i % 2
-        if i + 1 < n_e2e:
-            upload(1 - b)
         stream.wait_event(ev_copied[b])
         graphs[b].replay()
         ev_used[b].record(stream)
-        res_h.copy_(res, non_blocking=True)
-        stats_h[0].copy_(am.view(torch.float32), non_blocking=True)
-        stats_h[1].copy_(t1, non_blocking=True)
-        stats_h[2].copy_(en, non_blocking=True)
+        if i + 1 < n_e2e:
+            upload(1 - b)
         stream.synchronize()
-        _ = int(res_h[0])  # the per-step host read of the accepted length
+        _ = int(blk_h[b][0])  # the per-step host read of the accepted length
     e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
     clocks = sampler.stop()
 
