@@ -131,9 +131,9 @@ __device__ __forceinline__ RowStat stat_unpack(float4 v)
     return RowStat{v.x, __float_as_int(v.y), v.z, v.w, 0.f, 0.f};
 }
 
-// Threads per row for per-row scans by the CTA's threads: the largest power
-// of two with tpr x R_pad <= blockDim.x, at most 8 (the transposed tile's row
-// stride 128 + tpr is sized for 8).
+// Threads per row for the merges of partial statistics by all of the CTA's
+// threads: the largest power of two with tpr x R_pad <= blockDim.x, at most 8
+// (a row's partials are few, so more threads per row would mostly idle).
 __device__ __forceinline__ int threads_per_row(int R_pad)
 {
     int tpr = 1;
