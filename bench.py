@@ -855,9 +855,11 @@ def cpu_baseline(cfg: str, budget_s: float = 20.0):
 
     oracle.build()
     _, _, probe = cpu_sample_step(cfg, 1, 1)
-    n = int(max(1, min(64, budget_s / max(probe, 1e-6))))
     sh, _, _, _ = workload(cfg)
-    full, sample, _ = cpu_sample_step(cfg, min(n, sh.n_layers * sh.n_kv_heads), min(n, 32), seed=1)
+    # as many attention units as about budget_s of work allows (the probe times one unit and one
+    # vocab slice), at most the whole step
+    n = int(max(1, min(sh.n_layers * sh.n_kv_heads, budget_s / max(probe, 1e-6))))
+    full, sample, _ = cpu_sample_step(cfg, n, min(n, 32), seed=1)
     cores = oracle.num_threads()
     prev = oracle.set_num_threads(1)
     try:
