@@ -383,7 +383,9 @@ TB_API tb_status verify_step_batched_typical(const tb_bank *bank, int batch, con
  *   c, uniforms[N + u] draws the token at the final node u; scratch float
  *   [vocab].  All device memory.  *result: accept_len, path, bonus_token = the
  *   drawn token, new_L = L + accept_len, status (a draft token outside
- *   [0, vocab) is never accepted and sets TB_EINVAL).  One CTA. */
+ *   [0, vocab) is never accepted and sets TB_EINVAL).  One cluster of 8 CTAs
+ *   for vocab <= 131072 (scratch unused), else one CTA (scratch holds the
+ *   residual). */
 TB_API tb_status spec_sample_accept(const tb_bank *bank, int bank_id, const int32_t *draft_tokens, const float *logits,
                                     const float *logz_t, const float *draft_probs, const float *uniforms, int vocab,
                                     int L, float temperature, float *scratch, tb_result *result, tb_stream stream);

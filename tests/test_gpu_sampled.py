@@ -95,6 +95,42 @@ def test_walk_random_trees_vs_oracle(dev):
     b.close()
 
 
+def _spiky_rows(g, n, V, spikes, temp):
+    """Logits: N(0, 1) plus +U(8, 12) on `spikes` tokens of each row, so most of
+    p's mass sits on a few tokens anywhere in the vocabulary (the draw stays
+    decidable at any V).  Draft distribution: two of p's spikes and two of its
+    own, plus the background, so the residual keeps peaks after a rejection."""
+    z = g.standard_normal((n, V))
+    q = g.standard_normal((n, V)) * 0.5
+    for u in range(n):
+        hot = g.choice(V, size=spikes + 2, replace=False)
+        z[u, hot[:spikes]] += g.uniform(8.0, 12.0, size=spikes)
+        q[u, np.concatenate([hot[:2], hot[spikes:]])] += g.uniform(11.0, 14.0, size=4)
+    z = z.astype(np.float32).astype(np.float64)
+    q = _softmax_rows(q, 1.0)
+    return z, (q / q.sum(axis=1, keepdims=True)).astype(np.float32).astype(np.float64)
+
+
+@pytest.mark.parametrize("V", [32767, 32768, 32772, 50001, 131072, 131073, 150004])
+def test_walk_vocab_paths(dev, V):
+    """Vocabularies on both sides of the register-slice limits of the cluster
+    walk (8 CTAs x 1024 threads x 4 or 16 entries: 32768 and 131072) and past
+    them (the one-CTA walk), with 16-byte and unaligned rows; the spikes fall
+    in the slices of every CTA."""
+    b = tv.Bank(16, 0)
+    g = synth.rng(34 + V % 97)
+    trees = [synth.bank_trees()[-1], synth.chain(9), np.sort(synth.random_tree(g, 40)), synth.bank_trees()[5]]
+    for trial, parent in enumerate(trees):
+        parent = np.asarray(parent, np.int32)
+        parent[0] = -1
+        z, q = _spiky_rows(g, len(parent), V, 4, T)
+        draft, unif, want = _draw_case(g, parent, z, q, T)
+        r = _walk_on_gpu(dev, b, parent, draft, z, q, unif, T, L=trial)
+        assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (
+            want[0], want[1], want[2], trial + want[0], 0), (V, trial)
+    b.close()
+
+
 def test_walk_is_lossless_on_the_gpu(dev):
     """Root with three children drawn from q: the first emitted token follows p."""
     b = tv.Bank(4, 0)
