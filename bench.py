@@ -387,8 +387,8 @@ def run_gpu(args):
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         # per step: LM head, attention, split-unit merge (head_dim 128), acceptance + compaction
-        # (+ the rotary table and tree-key rotation with --rope; sampled: the walk, then compaction)
-        "gpu_launches": ((4 if d == 128 else 3) + (2 if args.rope else 0) + (1 if args.accept == "sampled" else 0))
+        # (+ the tree-key rotation, which also writes the rotary table, with --rope; sampled: the walk, then compaction)
+        "gpu_launches": ((4 if d == 128 else 3) + (1 if args.rope else 0) + (1 if args.accept == "sampled" else 0))
                         * args.steps,
         "clocks": clocks,
     }

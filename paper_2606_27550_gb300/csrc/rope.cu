@@ -6,16 +6,18 @@
 // element i + d/2) the step's queries and tree keys are rotated at those
 // positions; the prefix keys were rotated when they entered the cache.
 //
-//   k0_rope_table   one CTA per sequence: cos / sin of (L + depth) * theta_i
-//                   for every depth of the tree and i < d/2, into the
-//                   workspace.  The angle is formed and reduced to [-pi, pi]
-//                   in double (positions reach 10^4-10^5 rad), then sin and
-//                   cos are taken in float.  At most 64 x 64 entries, so the
-//                   few double operations stay cheap on a part whose FP64
-//                   rate is low.
-//   k0_rope_tree_k  one warp per tree key row (layer, kv head, node): the
-//                   row's pairs are rotated with the table and written back
-//                   to the bf16 cache in place.
+//   k0_rope_tree_k  one launch: a CTA per (tree node, 64 (layer, kv head)
+//                   rows of it).  Every thread first loads its 8 pairs of
+//                   two rows (16 bytes from each half: the long-context
+//                   step's 1024 CTAs are about one wave), then 64 threads form the
+//                   (cos, sin) of (L + depth) * theta_i for the node's depth
+//                   while the loads are in flight: the angle is formed and
+//                   reduced to [-pi, pi] in double (positions reach 10^4-10^5
+//                   rad), sin and cos are taken in float.  The rotated pairs
+//                   are written back to the bf16 cache in place.  The first
+//                   node of each depth (canonical order: depths do not
+//                   decrease with the id) also writes its table row to the
+//                   workspace for the query rotation.  head_dim 128.
 // The queries are rotated inside the attention kernel as they are staged
 // into tensor memory (attention_tc.cu), with the same table.
 #include <cuda_bf16.h>
@@ -24,35 +26,13 @@
 
 namespace tv {
 
-__global__ void __launch_bounds__(256) k0_rope_table(const __grid_constant__ RopeParams p)
-{
-    const RopeSeq &sq = p.seq[blockIdx.x];
-    const TreeDesc *tree = sq.tree;
-    int L = sq.L;
-    if (p.sched) {
-        const int rung = p.sched[0];
-        if (rung < 0 || rung >= p.n_rungs || p.sched[1] < 0)
-            return;
-        tree = p.rung_tree[rung];
-        L = p.sched[1];
-    }
-    const int h = p.d / 2;
-    const int n = (tree->max_depth + 1) * h;
-    float2 *tab = p.table + (size_t)blockIdx.x * kRopeTableEntries;
-    constexpr double kTwoPi = 6.283185307179586476925286766559;
-    for (int e = threadIdx.x; e < n; e += blockDim.x) {
-        const int dep = e / h, i = e - dep * h;
-        const double a = (double)(L + dep) * p.inv_freq[i];
-        const double r = a - kTwoPi * rint(a * (1.0 / kTwoPi));
-        float s, c;
-        sincosf((float)r, &s, &c);
-        tab[dep * kRopeMaxHalf + i] = make_float2(c, s);
-    }
-}
+constexpr int kRopeThreads = 256;                        // 8 threads per 128-wide row
+constexpr int kRopeRowsPerThread = 2;                    // rows r and r + 32, four 16-byte loads in flight
+constexpr int kRopeRowsPerCta = kRopeThreads / 8 * kRopeRowsPerThread;
 
-__global__ void __launch_bounds__(256) k0_rope_tree_k(const __grid_constant__ RopeParams p)
+__global__ void __launch_bounds__(kRopeThreads) k0_rope_tree_k(const __grid_constant__ RopeParams p, int n_rows)
 {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __shared__ float2 cs[kRopeMaxHalf];
     const RopeSeq &sq = p.seq[blockIdx.z];
     const TreeDesc *tree = sq.tree;
     int L = sq.L;
@@ -63,18 +43,53 @@ __global__ void __launch_bounds__(256) k0_rope_tree_k(const __grid_constant__ Ro
         tree = p.rung_tree[rung];
         L = Ls;
     }
-    const int j = blockIdx.x * 8 + warp;
+    const int j = blockIdx.x;
     if (j >= tree->n)
         return;
-    const int head = blockIdx.y % p.Hkv, layer = p.layer_begin + blockIdx.y / p.Hkv;
-    __nv_bfloat16 *row = sq.k + (size_t)layer * sq.layer_stride + (size_t)head * sq.head_stride + (size_t)(L + j) * p.d;
-    const float2 *tab = p.table + (size_t)blockIdx.z * kRopeTableEntries + tree->depth[j] * kRopeMaxHalf;
-    const int h = p.d / 2;
-    for (int i = lane; i < h; i += 32) {
-        const float2 cs = tab[i];
-        const float x1 = __bfloat162float(row[i]), x2 = __bfloat162float(row[i + h]);
-        row[i] = __float2bfloat16_rn(x1 * cs.x - x2 * cs.y);
-        row[i + h] = __float2bfloat16_rn(x2 * cs.x + x1 * cs.y);
+    const int dep = tree->depth[j];
+    constexpr int kHalf = 64;  // pairs of a 128-wide row
+    const int ch = (threadIdx.x & 7) * 8;
+    __nv_bfloat16 *row[kRopeRowsPerThread];
+    uint4 lo[kRopeRowsPerThread], hi[kRopeRowsPerThread];  // elements [ch, ch + 8) and [64 + ch, 64 + ch + 8)
+#pragma unroll
+    for (int k = 0; k < kRopeRowsPerThread; ++k) {
+        const int r = blockIdx.y * kRopeRowsPerCta + k * (kRopeThreads / 8) + (threadIdx.x >> 3);
+        row[k] = nullptr;
+        lo[k] = hi[k] = make_uint4(0, 0, 0, 0);
+        if (r < n_rows) {
+            const int head = r % p.Hkv, layer = p.layer_begin + r / p.Hkv;
+            row[k] = sq.k + (size_t)layer * sq.layer_stride + (size_t)head * sq.head_stride +
+                     (size_t)(L + j) * (2 * kHalf);
+            lo[k] = *reinterpret_cast<const uint4 *>(row[k] + ch);
+            hi[k] = *reinterpret_cast<const uint4 *>(row[k] + kHalf + ch);
+        }
+    }
+    if (threadIdx.x < kHalf) {
+        const int i = threadIdx.x;
+        constexpr double kTwoPi = 6.283185307179586476925286766559;
+        const double a = (double)(L + dep) * p.inv_freq[i];
+        const double red = a - kTwoPi * rint(a * (1.0 / kTwoPi));
+        float sn, cn;
+        sincosf((float)red, &sn, &cn);
+        cs[i] = make_float2(cn, sn);
+        if (blockIdx.y == 0 && (j == 0 || tree->depth[j - 1] != dep))
+            p.table[(size_t)blockIdx.z * kRopeTableEntries + dep * kRopeMaxHalf + i] = make_float2(cn, sn);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kRopeRowsPerThread; ++k) {
+        if (!row[k])
+            continue;
+        __nv_bfloat16 *x = reinterpret_cast<__nv_bfloat16 *>(&lo[k]), *y = reinterpret_cast<__nv_bfloat16 *>(&hi[k]);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float2 c = cs[ch + e];
+            const float x1 = __bfloat162float(x[e]), x2 = __bfloat162float(y[e]);
+            x[e] = __float2bfloat16_rn(x1 * c.x - x2 * c.y);
+            y[e] = __float2bfloat16_rn(x2 * c.x + x1 * c.y);
+        }
+        *reinterpret_cast<uint4 *>(row[k] + ch) = lo[k];
+        *reinterpret_cast<uint4 *>(row[k] + kHalf + ch) = hi[k];
     }
 }
 
@@ -86,13 +101,11 @@ void rope_inv_freq(double theta, int d, double *inv_freq)
 
 cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_layers, cudaStream_t stream)
 {
-    if (n_seq < 1 || n_seq > TB_MAX_BATCH || p.d > 2 * kRopeMaxHalf)
+    if (n_seq < 1 || n_seq > TB_MAX_BATCH || p.d != 2 * kRopeMaxHalf || max_nodes < 1 || max_nodes > kMaxNodes)
         return cudaErrorInvalidValue;
-    k0_rope_table<<<n_seq, 256, 0, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess)
-        return e;
-    k0_rope_tree_k<<<dim3((max_nodes + 7) / 8, p.Hkv * n_layers, n_seq), 256, 0, stream>>>(p);
+    const int n_rows = n_layers * p.Hkv;
+    k0_rope_tree_k<<<dim3(max_nodes, (n_rows + kRopeRowsPerCta - 1) / kRopeRowsPerCta, n_seq), kRopeThreads, 0,
+                     stream>>>(p, n_rows);
     return cudaGetLastError();
 }
 
