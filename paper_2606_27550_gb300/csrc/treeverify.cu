@@ -555,6 +555,7 @@ struct AttnArgs {
     const void *q;
     int Hq;
     void *out;
+    int max_ctas;  // > 0: the tcgen05 attention grid takes at most this many SMs
 };
 
 static tb_status check_rope(const tb_kv *kv, const char *fn);
@@ -626,7 +627,12 @@ static RopeSeq rope_seq(const tb_kv *kv, const TreeDesc *tree)
                    tree, kv->L};
 }
 
-static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn)
+// The rotary embedding (if any), then the attention.  hf: the step's helper
+// stream is forked after the rotary launch, so that the LM head it carries
+// cannot occupy the SMs before the attention CTAs are placed (an attention
+// CTA needs a whole SM).
+static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn,
+                              HelperFork *hf = nullptr)
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
@@ -639,16 +645,22 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
         if (st != TB_OK)
             return st;
     }
+    if (hf) {
+        tb_status st = hf->fork(fn);
+        if (st != TB_OK)
+            return st;
+    }
+    const int nsm = sm_count(a.bank->device);
     cudaError_t e;
     if (use_tc_attention(a.kv->head_dim, rows))
         e = attn_tc_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
                            reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                           reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err,
-                           rope ? rope_table(ws) : nullptr);
+                           reinterpret_cast<int *>(ws), a.max_ctas > 0 && a.max_ctas < nsm ? a.max_ctas : nsm, stream,
+                           &err, rope ? rope_table(ws) : nullptr);
     else
         e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
                         reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                        reinterpret_cast<int *>(ws), sm_count(a.bank->device), stream, &err);
+                        reinterpret_cast<int *>(ws), nsm, stream, &err);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -861,6 +873,26 @@ extern "C" tb_status typical_accept(const tb_bank *bank, int bank_id, const int3
     return ok();
 }
 
+// The attention grid beside the LM head of the same step.  The attention's
+// persistent grid normally takes one CTA per SM, each holding the whole
+// register file, so the LM head on the helper stream starts on the SMs that
+// attention CTAs release.  When the LM head is the longer of the two (a
+// single layer against a large vocabulary), the attention instead gets only
+// the SMs the LM head's CTAs leave free, and both run from the start.  That
+// pays when the attention on those SMs still ends well before the LM head:
+// about 3 us per 128-key tile a CTA walks plus 6 us, against the weight
+// bytes at 5 TB/s plus 8 us (measured on GB300 at 7B shapes).  0: no cap.
+static int attn_ctas_beside_lm(const AttnPlan &ap, const LmPlan &lp, int d_model, int vocab, int n_sm)
+{
+    const int lm_sms = (lp.P + lp.ctas_per_sm - 1) / lp.ctas_per_sm;
+    const int free_sms = n_sm - lm_sms;
+    if (free_sms < 1 || ap.total < 1)
+        return 0;
+    const double t_attn = 3.0 * (double)((ap.total + free_sms - 1) / free_sms) + 6.0;
+    const double t_lm = 2.0 * (double)vocab * (double)d_model / 5.0e6 + 8.0;
+    return t_attn < 0.75 * t_lm ? free_sms : 0;
+}
+
 static tb_status sample_enqueue(const tb_bank *bank, int bank_id, const int32_t *draft, const float *logits,
                                 const float *logz_t, const float *q, const float *unif, int vocab, int L,
                                 float temperature, float *scratch, tb_result *result, const int *ws_status,
@@ -940,10 +972,9 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
     lt.logz_t = tr.logz_t;
     lt.ent_t = tr.ent_t;
     lt.logits_out = logits;
+    a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
     HelperFork hf(bank, s);
-    if ((st = hf.fork(fn)) != TB_OK)
-        return st;
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &hf)) != TB_OK)
         return st;
     if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
                          hf.aux(), fn, 0, &lt)) != TB_OK)
@@ -1019,11 +1050,12 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, tr.draft_logit, 0, N};
     }
     // attention on the caller's stream; the LM head forked onto the bank's
-    // helper stream fills the SMs that attention CTAs release; join before acceptance
+    // helper stream fills the SMs that attention CTAs release (or, when it is
+    // the longer of the two, the SMs the attention is kept off); join before
+    // acceptance
+    a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
     HelperFork hf(bank, s);
-    if ((st = hf.fork(fn)) != TB_OK)
-        return st;
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &hf)) != TB_OK)
         return st;
     if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
                          hf.aux(), fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr)) != TB_OK)
@@ -1130,9 +1162,8 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
 
     // attention on the caller's stream, the LM head forked onto the helper
     // stream (it fills the SMs the attention CTAs release), joined before acceptance
+    // (forked after the rotary launch, so that the LM head cannot take the SMs first)
     HelperFork hf(bank, s);
-    if ((st = hf.fork(fn)) != TB_OK)
-        return st;
     cudaError_t e = cudaSuccess;
     // tree attention of every sequence (after the rotary embedding of their tree keys)
     if (tc) {
@@ -1147,6 +1178,8 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             if ((st = rope_enqueue(rp, &kv0, batch, 0, kv0.n_layers, max_nodes, ws, s, fn)) != TB_OK)
                 return st;
         }
+        if ((st = hf.fork(fn)) != TB_OK)
+            return st;
         AttnSeq as[TB_MAX_BATCH];
         for (int b = 0; b < batch; ++b)
             as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
@@ -1164,7 +1197,7 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             AttnPlan plan;
             if ((st = attn_validate(a, fn, &plan)) != TB_OK)
                 return st;
-            if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+            if ((st = attn_enqueue(a, ws, kPartBase, s, fn, b == 0 ? &hf : nullptr)) != TB_OK)
                 return st;
         }
     }
@@ -1332,8 +1365,6 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
         sc.rung_tree[r] = bank->d_desc + policy->bank_ids[r];
     {
         HelperFork hf(bank, s);
-        if ((st = hf.fork(fn)) != TB_OK)
-            return st;
         if (kv->rope_theta != 0.f) {
             RopeParams rp{};
             rp.seq[0] = rope_seq(kv, sc.rung_tree[0]);
@@ -1346,6 +1377,8 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
                 return st;
             sc.rope_tab = rope_table(ws);
         }
+        if ((st = hf.fork(fn)) != TB_OK)  // after the rotary launch: the attention CTAs are placed first
+            return st;
         const char *err = "";
         cudaError_t e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
