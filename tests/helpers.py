@@ -137,3 +137,33 @@ def typical_drafts(seed: int, parent, logits, T, eps, alpha, p_likely: float = 0
         if not close and not tie:
             return drafts
     raise RuntimeError("could not draw unambiguous drafts")
+
+
+# ---------------------------------------------------------------- speculative sampling
+
+WALK_MARGIN = 1e-4  # every decision of the oracle's walk at least this far from its boundary
+
+
+def softmax_rows(z, temp):
+    w = np.exp((z - z.max(axis=1, keepdims=True)) / temp)
+    return w / w.sum(axis=1, keepdims=True)
+
+
+def draw_decidable_walk(g, parent, z, q, temp, p_from_q=0.8):
+    """Drafts (children of u drawn from q_u, else uniform) and uniforms that keep
+    every decision of the oracle's walk -- a uniform against a probability ratio,
+    or against a CDF -- at least WALK_MARGIN from its boundary, so float32 and
+    float64 decide alike.  Returns (draft, unif, (accept_len, path, token))."""
+    n, V = z.shape
+    draft = np.zeros(n, np.int32)
+    for c in range(1, n):
+        u = parent[c]
+        draft[c] = g.choice(V, p=q[u] / q[u].sum()) if g.random() < p_from_q else g.integers(0, V)
+    for _ in range(200):
+        unif = g.random(2 * n).astype(np.float32).astype(np.float64)
+        k, path, tok, det = oracle.spec_sample(parent, draft, z, q, temp, unif, detail=True)
+        rm = det["ratio_margin"]
+        tried = rm[~np.isnan(rm)]
+        if (np.abs(tried[np.isfinite(tried)]) > WALK_MARGIN).all() and det["cdf_margin"] > WALK_MARGIN:
+            return draft, unif, (k, path, tok)
+    raise RuntimeError("no unambiguous uniforms")

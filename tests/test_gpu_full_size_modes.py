@@ -1,6 +1,7 @@
 """The long-context step at full size (32 layers x 32 heads x 128, L = 16384,
 64-node tree, V = 32000; the benchmark's launch configuration) with typical
-acceptance and with the rotary embedding applied by the library.
+acceptance, with the rotary embedding applied by the library, and with
+speculative sampling and the rotary embedding together.
 
 Attention is compared with the fp64 oracle on sampled (layer, head) pairs;
 the LM-head statistics, the acceptance and the compacted tree region of every
@@ -10,7 +11,8 @@ import numpy as np
 import pytest
 
 import oracle
-from helpers import STAT_TOL, TYPICAL, bits, check_attention, gap_filtered_hidden, to_dev, typical_drafts
+from helpers import (STAT_TOL, TYPICAL, bits, check_attention, draw_decidable_walk, gap_filtered_hidden,
+                     softmax_rows, to_dev, typical_drafts)
 from paper_2606_27550_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -119,6 +121,52 @@ def test_full_size_rope(dev, full):
         want = oracle.kv_compact(k_rot[0][None], 0, path)[0]
         gk = bits(k[layer, head, :L + N])
         diff = np.abs(_ordered(gk[L:L + N]) - _ordered(want))
+        assert diff.max() <= 1 and (diff > 0).mean() < 0.01
+        assert np.array_equal(gk[:L], kk[:L])
+    assert np.array_equal(bits(v[:, :, L:L + N]), oracle.kv_compact(tree_v, 0, path))
+    b.close()
+
+
+def test_full_size_sampled_rope(dev, full):
+    """The walk of speculative sampling (8-CTA cluster kernel) after attention with
+    the rotary embedding and the LM head writing every logit row: the launch of
+    `bench.py --accept sampled --rope`.  Drafts from a draft distribution that
+    mostly agrees with the target, uniforms that keep every decision decidable."""
+    f = full
+    parent = np.asarray(f["sh"].parent, np.int32)
+    N, L, V = f["N"], f["L"], f["V"]
+    T = 0.7
+    g = synth.rng(82)
+    qd = softmax_rows(f["logits"] / T * 1.3 + g.standard_normal((N, V)) * 0.5, 1.0)
+    qd = (qd / qd.sum(axis=1, keepdims=True)).astype(np.float32).astype(np.float64)
+    draft, unif, want = draw_decidable_walk(g, parent, f["logits"], qd, T)
+    b = tv.Bank(4, 0)
+    bid, _ = b.add(parent)
+    k, v, q = _cache(dev, f, 81)
+    pre = {s: (bits(k[s[0], s[1], :L + N]), bits(v[s[0], s[1], :L + N])) for s in SAMPLES}
+    tree_v = bits(v[:, :, L:L + N])
+    q_h = bits(q)
+    out, g_am, g_t1, g_en, res, ws = _outs(dev, f)
+    lg = torch.full((N + 1, V), float("nan"), dtype=torch.float32, device=dev)
+    tv.verify_step_sampled(b, bid, tv.KvCache(k, v, L, rope_theta=10000.0), q, to_dev(f["hidden"], dev),
+                           to_dev(f["W"], dev), to_dev(draft, dev), to_dev(qd.astype(np.float32), dev),
+                           to_dev(unif.astype(np.float32), dev), T, out, g_am, g_t1, g_en, lg, res, ws)
+    torch.cuda.synchronize()
+    r = tv.parse_result(res)
+    assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (
+        want[0], want[1], want[2], L + want[0], 0)
+    assert np.array_equal(g_am.cpu().numpy(), f["am"])
+    assert np.abs(g_en.cpu().numpy() - f["en"]).max() <= STAT_TOL
+    assert np.abs(lg[:N].cpu().numpy() - f["logits"]).max() <= 1e-3
+    got = out.float().cpu().numpy()
+    path = want[1]
+    for layer, head in SAMPLES:
+        kk, vv = pre[(layer, head)]
+        ref, k_rot = oracle.tree_attention_rope(q_h[layer][:, head:head + 1], kk[None], vv[None], L, parent)
+        check_attention(got[layer][:, head:head + 1], ref, f"layer {layer} head {head}")
+        want_k = oracle.kv_compact(k_rot[0][None], 0, path)[0]
+        gk = bits(k[layer, head, :L + N])
+        diff = np.abs(_ordered(gk[L:L + N]) - _ordered(want_k))
         assert diff.max() <= 1 and (diff > 0).mean() < 0.01
         assert np.array_equal(gk[:L], kk[:L])
     assert np.array_equal(bits(v[:, :, L:L + N]), oracle.kv_compact(tree_v, 0, path))

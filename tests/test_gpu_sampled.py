@@ -13,7 +13,8 @@ import numpy as np
 import pytest
 
 import oracle
-from helpers import STAT_TOL, bits, check_attention, gap_filtered_hidden, to_dev
+from helpers import STAT_TOL, bits, check_attention, draw_decidable_walk as _draw_case, gap_filtered_hidden, \
+    softmax_rows as _softmax_rows, to_dev
 from paper_2606_27550_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -22,7 +23,6 @@ tv = pytest.importorskip("paper_2606_27550_gb300")
 pytestmark = pytest.mark.gpu
 
 T = 0.7
-MARGIN = 1e-4
 
 
 @pytest.fixture(scope="module")
@@ -32,29 +32,6 @@ def dev():
     build.build()
     torch.cuda.set_device(0)
     return torch.device("cuda:0")
-
-
-def _softmax_rows(z, temp):
-    w = np.exp((z - z.max(axis=1, keepdims=True)) / temp)
-    return w / w.sum(axis=1, keepdims=True)
-
-
-def _draw_case(g, parent, z, q, temp, p_from_q=0.8):
-    """Drafts (children of u drawn from q_u, else uniform) and uniforms that keep every
-    decision of the oracle's walk clear of its boundary."""
-    n, V = z.shape
-    draft = np.zeros(n, np.int32)
-    for c in range(1, n):
-        u = parent[c]
-        draft[c] = g.choice(V, p=q[u] / q[u].sum()) if g.random() < p_from_q else g.integers(0, V)
-    for _ in range(200):
-        unif = g.random(2 * n).astype(np.float32).astype(np.float64)
-        k, path, tok, det = oracle.spec_sample(parent, draft, z, q, temp, unif, detail=True)
-        rm = det["ratio_margin"]
-        tried = rm[~np.isnan(rm)]
-        if (np.abs(tried[np.isfinite(tried)]) > MARGIN).all() and det["cdf_margin"] > MARGIN:
-            return draft, unif, (k, path, tok)
-    raise RuntimeError("no unambiguous uniforms")
 
 
 def _walk_on_gpu(dev, bank, parent, draft, z, q, unif, temp, L=0):

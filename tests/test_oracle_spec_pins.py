@@ -115,3 +115,43 @@ def test_second_token_given_acceptance_follows_the_child_target():
             counts[draft[2] if k == 3 else tok] += 1
     assert hits > 5000
     assert np.abs(counts / hits - p1).max() < 0.02
+
+
+def test_closed_form_residual_matches_the_sequential_update():
+    """After k rejected siblings the residual is max(0, p - c_k q) / S_k, with
+    c_0 = 0, S_0 = 1 and, after each rejection, c <- c + S, S <- sum_v max(0,
+    p - c q) -- the form the GPU walk evaluates.  The oracle applies the rule's
+    sequential update norm(max(0, r - q)); its ratio margins give r(t_c) / q(t_c)
+    - unif[c] for every child it tries, so r at each tried token is compared
+    with the closed form."""
+    g = synth.rng(41)
+    n = 7
+    parent = [-1] + [0] * (n - 1)  # a root with six children: up to six rejections in a row
+    compared = deepest = 0
+    for trial in range(60):
+        V = int(g.choice([5, 50, 500]))
+        z = g.standard_normal((n, V)) * float(g.uniform(0.5, 3.0))
+        qs = np.stack([_softmax(g.standard_normal(V) * float(g.uniform(0.5, 3.0)), 1.0) for _ in range(n)])
+        draft = np.concatenate([[0], g.integers(0, V, n - 1)]).astype(np.int32)
+        unif = g.random(2 * n) * float(g.choice([1.0, 0.2]))  # small uniforms: more acceptances, fewer residuals
+        unif = np.where(g.random(2 * n) < 0.5, 1.0 - 1e-12, unif)  # and near-1 ones: long runs of rejections
+        _, _, _, det = oracle.spec_sample(parent, draft, z, qs, T, unif, detail=True)
+        p = _softmax(z[0], T)
+        q = qs[0]
+        c, S = 0.0, 1.0
+        k = 0
+        for child in range(1, n):
+            margin = det["ratio_margin"][child]
+            if np.isnan(margin):
+                break  # not tried: a sibling before it was accepted
+            t = draft[child]
+            r_oracle = (margin + unif[child]) * q[t]
+            r_closed = p[t] if k == 0 else (max(0.0, p[t] - c * q[t]) / S if S > 0 else 0.0)
+            assert r_oracle == pytest.approx(r_closed, rel=1e-9, abs=1e-15), (trial, child)
+            compared += 1
+            if margin > 0:
+                break  # accepted
+            c, S = c + S, float(np.maximum(p - (c + S) * q, 0.0).sum())
+            k += 1
+        deepest = max(deepest, k)
+    assert compared > 150 and deepest >= 5
