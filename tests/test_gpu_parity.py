@@ -249,6 +249,37 @@ def test_verify_step_full_parity(dev, bank, cfg):
     assert np.array_equal(bits(vd), oracle.kv_compact(case.v, case.L, path))
 
 
+# Steps whose LM head is longer than their attention: the attention grid is then
+# capped at the SMs the LM head's CTAs leave free, so that both start at once.
+# On a 152-SM GB300 these shapes get: 73 attention CTAs over 136 tiles (units
+# of 17 tiles spread over several CTAs); 27 over 160 (units of 40 tiles); 27
+# over 64 (units of 2 tiles); 54 over 128 across two layers with GQA group 4.
+BESIDE_LM = [
+    # parent, L, layers, Hq, Hkv, D, V
+    (synth.shape_c2().parent, 2048, 1, 8, 8, 4096, 20000),
+    (synth.bank_trees()[6], 5000, 1, 8, 4, 4096, 32000),
+    (synth.bank_trees()[-1], 100, 1, 32, 32, 4096, 32000),
+    (synth.chain(17), 1000, 2, 32, 8, 2048, 25000),
+]
+
+
+@pytest.mark.parametrize("parent,L,layers,Hq,Hkv,D,V", BESIDE_LM)
+def test_verify_step_beside_lm_head(dev, bank, parent, L, layers, Hq, Hkv, D, V):
+    case = make_case(11, parent, L, layers, Hq, Hkv, 128, D, V, 0.7)
+    out, g_am, g_t1, g_en, r, kd, vd = _full_step(dev, bank, case, Hq, Hkv, 128)
+    got = out.float().cpu().numpy()
+    for layer in range(layers):
+        check_attention(got[layer], oracle.tree_attention(case.q[layer], case.k[layer], case.v[layer], L, case.parent),
+                        f"layer {layer}")
+    assert np.array_equal(g_am.cpu().numpy(), case.argmax)
+    assert np.abs(g_t1.cpu().numpy() - case.top1).max() <= STAT_TOL
+    assert np.abs(g_en.cpu().numpy() - case.entropy).max() <= STAT_TOL
+    k, path, bonus = oracle.accept(case.parent, case.drafts, case.argmax)
+    assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (k, path, bonus, L + k, 0)
+    assert np.array_equal(bits(kd), oracle.kv_compact(case.k, L, path))
+    assert np.array_equal(bits(vd), oracle.kv_compact(case.v, L, path))
+
+
 def test_verify_step_no_compact_flag(dev, bank):
     sh = synth.shape_c1()
     case = make_case(9, sh.parent, sh.L, 1, 4, 4, 64, 256, 1000, 1.0)  # every draft matches
