@@ -143,6 +143,14 @@ def kernel_source_hash(files: str) -> str:
     return h.hexdigest()[:16]
 
 
+def launches_per_step(head_dim: int, rope: bool, accept: str) -> int:
+    """Kernels the library launches for one verify step of a multi-tile problem: the LM
+    head, the attention, the split-unit merge (head_dim 128), acceptance + compaction;
+    + the tree-key rotation (which also writes the rotary table) with rope; sampled
+    acceptance launches the walk, then the compaction."""
+    return (4 if head_dim == 128 else 3) + (1 if rope else 0) + (1 if accept == "sampled" else 0)
+
+
 def acceptance_label(args) -> str:
     if getattr(args, "accept", "greedy") == "typical":
         return "typical (T=0.7, eps=0.09, alpha=0.3)"
@@ -386,10 +394,7 @@ def run_gpu(args):
         "accept_len_last": r["accept_len"],
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        # per step: LM head, attention, split-unit merge (head_dim 128), acceptance + compaction
-        # (+ the tree-key rotation, which also writes the rotary table, with --rope; sampled: the walk, then compaction)
-        "gpu_launches": ((4 if d == 128 else 3) + (1 if args.rope else 0) + (1 if args.accept == "sampled" else 0))
-                        * args.steps,
+        "gpu_launches": launches_per_step(d, args.rope, args.accept) * args.steps,
         "clocks": clocks,
     }
     if args.layers:
