@@ -230,9 +230,10 @@ struct tb_bank {
 };
 
 // The helper stream of a step.  The LM head runs on the bank's helper stream,
-// forked from the caller's stream when the step starts and joined back before
-// acceptance; the bank's fork and join events are shared, so the bank's mutex
-// is held from the fork to the end of the step's enqueueing.
+// forked from the caller's stream just before the attention launch (after the
+// rotary embedding's, if any) and joined back before acceptance; the bank's
+// fork and join events are shared, so the bank's mutex is held from the
+// object's construction to the end of the step's enqueueing.
 class HelperFork {
   public:
     HelperFork(const tb_bank *bank, cudaStream_t s) : bank_(const_cast<tb_bank *>(bank)), s_(s), lk_(bank_->fork_mu)
