@@ -289,20 +289,34 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
  * same kernel, but keeps its scratch in a 4 MiB array compiled into the
  * library (every GPU that loads the library holds it until the process
  * exits); it calls no cudaMalloc, cudaFree or allocating library routine.
- *  - The first call on a device looks up that array's device address
- *    (cudaGetSymbolAddress) with the device current; make that first call
- *    before capturing the stream into a graph.
- *  - Every call clears the array's arrival counters on `stream` and reuses the
- *    array, which keeps the previous call's partial results: calls that can
- *    overlap on the GPU (different streams without ordering) race.
- *  - The scratch is one partial per persistent CTA and per merge group for
- *    every row (about 2 MiB at 256 rows with 152 SMs, for any vocabulary);
- *    a device whose SM count needs more than 4 MiB is rejected with
- *    TB_ECAPACITY before anything is enqueued.
- * Arguments, layouts and tolerances are those of lm_head_stats.  The paper has
- * no counterpart: this is an integration convenience of this library. */
+ *  - Outside stream capture every call looks up that array's device address
+ *    (cudaGetSymbolAddress) on the current device; while `stream` is being
+ *    captured the address found by the last call on this device is used, so
+ *    make one call outside capture first (and again after a cudaDeviceReset).
+ *  - Every call clears the array's arrival counters and status word on
+ *    `stream` and reuses the array, which keeps the previous call's partial
+ *    results: calls that can overlap on the GPU (different streams without
+ *    ordering) race.
+ *  - The scratch is one partial per persistent CTA for every row (at most
+ *    about 1.8 MiB: 256 rows, two CTAs on each of 152 SMs, for any
+ *    vocabulary); a device whose SM count needs more than 4 MiB is rejected
+ *    with TB_ECAPACITY before anything is enqueued.
+ *  - A bounded device wait that runs out (TB_ETIMEOUT) leaves argmax / top1 /
+ *    entropy unwritten and is visible only through
+ *    lm_head_stats_noalloc_status.
+ * flags: 0, or TB_DEBUG_EXPIRE_WAIT (test hook, as for verify_step).
+ * Arguments, layouts, argument checks and tolerances are those of
+ * lm_head_stats.  The paper has no counterpart: this is an integration
+ * convenience of this library. */
 TB_API tb_status lm_head_stats_noalloc(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
-                                       int32_t *argmax, float *top1, float *entropy, tb_stream stream);
+                                       int32_t *argmax, float *top1, float *entropy, int flags, tb_stream stream);
+
+/* Device-detected status of the last lm_head_stats_noalloc call enqueued on
+ * `stream`: waits for `stream`, then reads the built-in array's status word
+ * into *status (TB_OK, or TB_ETIMEOUT when a bounded wait of that call ran
+ * out).  Synchronous; allocates nothing.  The next lm_head_stats_noalloc call
+ * clears the word. */
+TB_API tb_status lm_head_stats_noalloc_status(int32_t *status, tb_stream stream);
 
 /* ------------------------------------------------------------------------
  * Typical acceptance: the Medusa/Hydra verification rule that the paper keeps

@@ -29,7 +29,8 @@ RESULT_INTS = 4 + TB_MAX_NODES  # sizeof(tb_result) / 4
 
 API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb_destroy", "tb_workspace_size",
        "tb_workspace_init", "tb_workspace_status", "tree_attention", "lm_head_stats", "greedy_accept",
-       "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "tb_last_error",
+       "kv_compact", "verify_step", "verify_step_batched", "lm_head_stats_noalloc", "lm_head_stats_noalloc_status",
+       "tb_last_error",
        "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
        "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical",
        "verify_step_scheduled", "spec_sample_accept", "verify_step_sampled")
@@ -101,7 +102,8 @@ def load(path: str = LIB_PATH):
         "greedy_accept": [P, i32, P, P, i32, i32, P, P],
         "kv_compact": [P, P, P],
         "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
-        "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, P],
+        "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, i32, P],
+        "lm_head_stats_noalloc_status": [P, P],
         "verify_step_batched": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, sz, i32, P],
         "tb_last_error": [],
         "lm_head_stats_typical": [P, i32, P, P, i32, i32, ctypes.c_float, P, P, P, P, P, P, P, P, sz, P],
@@ -304,12 +306,20 @@ def verify_step(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft
                               _stream(stream)), "verify_step")
 
 
-def lm_head_stats_noalloc(hidden, lm_head, argmax, top1, entropy, stream=None):
+def lm_head_stats_noalloc(hidden, lm_head, argmax, top1, entropy, flags: int = 0, stream=None):
     """lm_head_stats with the library's built-in scratch array instead of a
     caller workspace, for callers that cannot allocate device memory."""
     R, D = hidden.shape
     _check(load().lm_head_stats_noalloc(_ptr(hidden), R, _ptr(lm_head), D, lm_head.shape[0], _ptr(argmax),
-                                        _ptr(top1), _ptr(entropy), _stream(stream)), "lm_head_stats_noalloc")
+                                        _ptr(top1), _ptr(entropy), flags, _stream(stream)), "lm_head_stats_noalloc")
+
+
+def lm_head_stats_noalloc_status(stream=None) -> int:
+    """Device-detected status (TB_OK or TB_ETIMEOUT) of the last
+    lm_head_stats_noalloc call on `stream`; waits for the stream."""
+    st = ctypes.c_int32(0)
+    _check(load().lm_head_stats_noalloc_status(ctypes.byref(st), _stream(stream)), "lm_head_stats_noalloc_status")
+    return st.value
 
 
 @dataclass

@@ -15,7 +15,8 @@
 // unit's ticket counter (log-sum-exp merge of (m, l, O) partials); no CTA
 // ever waits for another.
 //
-// Per CTA: warp 4 streams 64-key K and V tiles with TMA (4-D tensor maps over
+// This kernel serves head_dim 64 (head_dim 128 runs on the tcgen05 kernel of
+// attention_tc.cu).  Per CTA: warp 4 streams 64-key K and V tiles with TMA (4-D tensor maps over
 // the caller's cache, 128-byte swizzle, zero fill past L + N) through a
 // 3-stage mbarrier ring; warps 0-3 own 16 query rows each and run the
 // online-softmax flash loop on the tensor cores (mma.sync m16n8k16 bf16,
@@ -463,17 +464,15 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
     p.part = part;
     p.counters = counters;
     p.status = status;
-    const size_t smem = attn_smem_bytes(d);
-    cudaError_t e;
-    if (d == 128) {
-        if ((e = allow_max_smem((const void *)k1_tree_attention<128>)) != cudaSuccess)
-            return e;
-        k1_tree_attention<128><<<pl.P, 160, smem, stream>>>(p);
-    } else {
-        if ((e = allow_max_smem((const void *)k1_tree_attention<64>)) != cudaSuccess)
-            return e;
-        k1_tree_attention<64><<<pl.P, 160, smem, stream>>>(p);
+    // head_dim 128 runs on the tcgen05 kernel (attention_tc.cu); this one serves head_dim 64
+    if (d != 64) {
+        *err = "the mma.sync attention kernel serves head_dim 64 only";
+        return cudaErrorInvalidValue;
     }
+    cudaError_t e;
+    if ((e = allow_max_smem((const void *)k1_tree_attention<64>)) != cudaSuccess)
+        return e;
+    k1_tree_attention<64><<<pl.P, 160, attn_smem_bytes(d), stream>>>(p);
     return cudaGetLastError();
 }
 

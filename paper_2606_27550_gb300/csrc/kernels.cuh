@@ -169,6 +169,12 @@ cudaError_t allow_max_smem(const void *kernel);
 // sets the message returned by tb_last_error() on this thread (treeverify.cu)
 tb_status record_error(tb_status st, const char *fmt, ...);
 
+// Argument checks of every LM-head entry point (pointers, alignment, 1..256
+// rows, d_model a multiple of 8, vocab, counter capacity); fills *plan for the
+// current device (treeverify.cu).
+tb_status lm_validate(const void *hidden, int R, const void *W, int D, int V, const void *am, const void *t1,
+                      const void *en, const char *fn, LmPlan *plan);
+
 // tensor maps (treeverify.cu)
 bool make_tmap_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                   uint32_t box_inner, uint32_t box_outer, const char **err);

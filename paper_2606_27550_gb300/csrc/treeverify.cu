@@ -161,13 +161,13 @@ static size_t align256(size_t x)
     return (x + 255) / 256 * 256;
 }
 
-// Partial slots of the split-L merge: two per CTA of whichever attention
-// kernel runs (the tcgen05 one for head_dim 128, else the mma.sync one).
+// Partial slots of the split-L merge: two per CTA of the attention kernel
+// that runs (the tcgen05 one for head_dim 128, the mma.sync one for head_dim 64).
 static size_t attn_part_bytes(int n_sm, int d)
 {
-    const size_t mma = (size_t)2 * n_sm * 2 * attn_slot_floats(d) * 4;
-    const size_t tc = attn_tc_supported(d, 0) ? (size_t)n_sm * 2 * attn_tc_slot_floats() * 4 : 0;
-    return align256(mma > tc ? mma : tc);
+    if (attn_tc_supported(d, 0))
+        return align256((size_t)n_sm * 2 * attn_tc_slot_floats() * 4);
+    return align256((size_t)2 * n_sm * 2 * attn_slot_floats(d) * 4);
 }
 
 // head_dim 128 runs on the tcgen05 kernel; head_dim 64 on the mma.sync one.
@@ -669,8 +669,8 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
     return TB_OK;
 }
 
-static tb_status lm_validate(const void *hidden, int R, const void *W, int D, int V, const void *am, const void *t1,
-                             const void *en, const char *fn, LmPlan *plan)
+tb_status tv::lm_validate(const void *hidden, int R, const void *W, int D, int V, const void *am, const void *t1,
+                          const void *en, const char *fn, LmPlan *plan)
 {
     if (!hidden || !W || !am || !t1 || !en)
         return fail(TB_EINVAL, "%s: NULL LM-head argument", fn);

@@ -76,6 +76,7 @@ def test_every_wrapper_marshals_its_declared_arguments(fake):
     tv.kv_compact(kv, res, stream=s)
     tv.verify_step(bank, 0, kv, q, h, W, i32(3), q, i32(3), f32(3), f32(3), res, ws, stream=s)
     tv.lm_head_stats_noalloc(h, W, i32(3), f32(3), f32(3), stream=s)
+    tv.lm_head_stats_noalloc_status(stream=s)
     seq = tv.Seq(0, kv, q, i32(3), q, res)
     tv.verify_step_batched(bank, [seq, seq], t(6, 64), W, i32(6), f32(6), f32(6), ws, stream=s)
     tv.lm_head_stats_typical(bank, 0, h, W, 0.7, i32(3), i32(3), f32(3), f32(3), f32(3), f32(3), f32(3), ws, stream=s)
@@ -90,7 +91,7 @@ def test_every_wrapper_marshals_its_declared_arguments(fake):
                            f32(4, 10), res, ws, stream=s)
     called = {n for n in tv.API if getattr(fake, n, None) is not None and getattr(getattr(fake, n), "calls", [])}
     wrapped = {"tree_attention", "lm_head_stats", "greedy_accept", "kv_compact", "verify_step",
-               "lm_head_stats_noalloc", "verify_step_batched", "lm_head_stats_typical", "typical_accept",
+               "lm_head_stats_noalloc", "lm_head_stats_noalloc_status", "verify_step_batched", "lm_head_stats_typical", "typical_accept",
                "verify_step_typical", "verify_step_batched_typical", "verify_step_scheduled", "spec_sample_accept",
                "verify_step_sampled"}
     assert wrapped <= called

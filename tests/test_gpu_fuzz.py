@@ -3,12 +3,17 @@ and out of breadth-first order), prefix lengths (including 0), head_dim 64
 and 128, GQA groups, d_model not a multiple of 64, vocabularies from 1 token
 up, single and batched steps.
 
-Same bars as the other parity tests, with one addition for attention: short or
-empty prefixes give rows that average a handful of values, whose outputs reach
-|x| ~ 4; there the bf16 probabilities of the P V product and the bf16 output
-alone account for about two bf16 ulps (2^-7 |x|), so an element may differ by
-max(1e-2, 2^-7 |ref|); the mean-abs bar stays 1e-3.  The workload-shaped tests
-keep the plain 1e-2 bar."""
+Same bars as the other parity tests (attention max-abs 1e-2, mean-abs 1e-3),
+except where the arithmetic of the kernels cannot reach 1e-2.  Short or empty
+prefixes give rows that average a handful of values, with outputs up to
+|x| ~ 4.  Two roundings are part of the kernels' design: the softmax weights
+enter the P V product as bf16 (relative error <= 2^-8 each), and the output is
+stored as bf16 (<= 2^-8 |O|).  With A = sum_s p_s |v_s| / sum_s p_s (the
+attention of the same row over |V|, computed by the oracle), the error of an
+element is bounded by 2^-8 |O| + 2^-8 A, plus 2^-12 A for every fp32 step
+(scores, exponentials, accumulation, split merge), which are orders of
+magnitude smaller.  An element may exceed 1e-2 only where that bound does;
+the test reports how many elements need it."""
 import numpy as np
 import pytest
 
@@ -31,14 +36,30 @@ def dev():
     return torch.device("cuda:0")
 
 
-def check_attention_fuzz(got, ref, what):
+def attention_bound(ref, ref_abs_v):
+    """Per-element error bound of the kernels' attention: bf16 output and bf16
+    probabilities in P V (2^-8 each), and 2^-12 A for the fp32 steps."""
+    return 2.0 ** -8 * np.abs(ref) + (2.0 ** -8 + 2.0 ** -12) * ref_abs_v
+
+
+def check_attention_fuzz(got, ref, ref_abs_v, what):
+    """got vs the oracle's ref, with ref_abs_v the oracle's attention over |V|."""
     got = got.astype(np.float64)
     assert np.all(np.isfinite(got)), f"{what}: non-finite output"
     err = np.abs(got - ref)
-    bound = np.maximum(1e-2, np.abs(ref) * 2.0 ** -7)
+    bound = np.maximum(1e-2, attention_bound(ref, ref_abs_v))
     worst = np.argmax(err - bound)
-    assert (err <= bound).all(), f"{what}: |err| {err.flat[worst]:.3e} at |ref| {abs(ref.flat[worst]):.3f}"
+    n_over = int((err > 1e-2).sum())
+    if n_over:
+        print(f"{what}: {n_over} of {err.size} elements beyond 1e-2, within the derived bound")
+    assert (err <= bound).all(), (f"{what}: |err| {err.flat[worst]:.3e} at |ref| {abs(ref.flat[worst]):.3f}, "
+                                  f"bound {bound.flat[worst]:.3e}")
     assert err.mean() <= 1e-3, f"{what}: mean |err| {err.mean():.3e}"
+
+
+def abs_bits(a):
+    """|x| of bf16 bit patterns (sign bit cleared)."""
+    return (a & np.uint16(0x7FFF)).astype(np.uint16)
 
 
 def _hidden(g, n, W, gap_min=1e-2):
@@ -101,6 +122,7 @@ def test_random_verify_step(dev, seed):
     got = out.float().cpu().numpy()
     for layer in range(layers):
         check_attention_fuzz(got[layer], oracle.tree_attention(q[layer], k[layer], v[layer], L, canon),
+                             oracle.tree_attention(q[layer], k[layer], abs_bits(v[layer]), L, canon),
                              f"seed {seed} layer {layer} (N={N} L={L} d={d} Hq={Hq} Hkv={Hkv})")
     assert np.array_equal(g_am.cpu().numpy(), am), seed
     assert np.abs(g_t1.cpu().numpy() - t1).max() <= STAT_TOL
@@ -159,7 +181,7 @@ def test_random_batched_step(dev, seed):
     for s, (parent, L, k, v, q, drafts, r0) in zip(tseqs, host):
         n = len(parent)
         check_attention_fuzz(s.attn_out[0].float().cpu().numpy(), oracle.tree_attention(q[0], k[0], v[0], L, parent),
-                             f"seed {seed} L={L} n={n}")
+                             oracle.tree_attention(q[0], k[0], abs_bits(v[0]), L, parent), f"seed {seed} L={L} n={n}")
         ka, path, bonus = oracle.accept(parent, drafts, am[r0:r0 + n])
         r = tv.parse_result(s.result)
         assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (ka, path, bonus, L + ka, 0)
