@@ -118,6 +118,12 @@ __device__ void policy_step(const AcceptParams &p, int rung, int L, int len, int
 // blockIdx.y selects the sequence; every CTA of a sequence recomputes its acceptance.
 __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__ AcceptBatch pb)
 {
+    // launched as a programmatic dependent of the step's LM head: its launch
+    // overlaps the LM head's tail, and it reads the LM head's outputs (and the
+    // cache the attention has finished reading) after this wait; the split-unit
+    // merge that follows may then start beside it
+    pdl_wait();
+    pdl_trigger();
     const AcceptParams &p = pb.seq[blockIdx.y];
     __shared__ int s_path[kMaxNodes];
     __shared__ float s_lp[kMaxNodes];
@@ -315,7 +321,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
     }
 }
 
-cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream)
+cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream, bool pdl)
 {
     if (n < 1 || n > TB_MAX_BATCH)
         return cudaErrorInvalidValue;
@@ -333,13 +339,12 @@ cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStr
                 grid = gx;
         }
     }
-    k3_accept_compact<<<dim3(grid, n), 256, 0, stream>>>(pb);
-    return cudaGetLastError();
+    return launch_kernel(k3_accept_compact, dim3(grid, n), dim3(256), 0, stream, pdl, pb);
 }
 
-cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream)
+cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream, bool pdl)
 {
-    return accept_launch_batch(&p, 1, n_sm, stream);
+    return accept_launch_batch(&p, 1, n_sm, stream, pdl);
 }
 
 }  // namespace tv

@@ -7,7 +7,9 @@
 // on tcgen05.  A CTA that covers a whole unit writes its output; a unit split
 // between CTAs leaves one (O, m, l) partial per CTA, and a second small kernel
 // (k1_merge_split, one warp per query row) combines them by log-sum-exp after
-// the first one has finished:
+// the first one has finished (in a verification step, beside the acceptance
+// kernel at the end of the step: nothing in the step reads the attention
+// output):
 //
 //   S   = Q K^T   tcgen05.mma kind::f16, M = 128 query rows, N = 128 keys,
 //                 K = 128 = head_dim; Q (bf16) is the TMEM A operand, the K
@@ -38,6 +40,8 @@
 // Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that the rows
 // are spread over the four lane quadrants (all four SM sub-partitions share
 // the softmax).
+#include <string.h>
+
 #include "kernels.cuh"
 
 namespace tv {
@@ -87,6 +91,7 @@ struct TcParams {
     const int32_t *sched;
     const TreeDesc *rung_tree[8];
     int n_rungs, n_layers, L_cap;
+    int max_rows;  // query rows of the largest row block (the split merge's grid)
     // rotary embedding (null: the queries are already rotated): per sequence a
     // table of (cos, sin) at position L + depth for every pair of head elements
     const float2 *rope_tab;
@@ -164,6 +169,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
+    // Launched as a programmatic dependent (a grid that leaves SMs free), the
+    // kernel waits here for the stream's previous work (the previous step's
+    // compaction writes the cache).  The step's LM head may then be launched:
+    // it fills the SMs that attention CTAs leave free or release.
+    pdl_wait();
+    pdl_trigger();
     const TcSeq *seqs = p.seq;
     long long total = p.total;
     if (p.sched) {
@@ -613,9 +624,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 // first boundary inside a unit handles it.  One warp per query row, each lane
 // 4 of the 128 output columns, four slots' loads issued together; 32 registers
 // per thread keep every row's warp resident at once.
-template <bool kBatched>
+//
+// kAfterStep: launched as a programmatic dependent of a verification step's
+// acceptance kernel.  The attention it merges has completed by then (the
+// acceptance kernel proceeds only once the LM head has, and the LM head
+// completes only after the attention), so it does not wait at entry and runs
+// beside the acceptance kernel; at exit it waits for the acceptance kernel,
+// so that the stream's next kernel also runs after the compaction.
+// Otherwise it waits at entry for the stream's previous kernel.
+struct PdlWaitOnExit {
+    __device__ ~PdlWaitOnExit() { pdl_wait(); }
+};
+
+template <bool kBatched, bool kAfterStep>
 __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__ TcParams p)
 {
+    if constexpr (!kAfterStep)
+        pdl_wait();
+    pdl_trigger();
+    PdlWaitOnExit pdl_exit;
     __shared__ TcSeq s_seq;
     __shared__ long long s_total;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -711,6 +738,29 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
 // ----------------------------------------------------------------------------
 // host side
 
+// The split-unit merge of an attention launch with parameters p (nothing to
+// do when the grid is one CTA).  after_step: see k1_merge_split.
+static cudaError_t merge_launch(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
+{
+    if (p.P <= 1)
+        return cudaSuccess;
+    const dim3 grid(p.P - 1, (p.max_rows + 7) / 8);
+    if (batched)
+        return after_step ? launch_kernel(k1_merge_split<true, true>, grid, dim3(256), 0, stream, pdl, p)
+                          : launch_kernel(k1_merge_split<true, false>, grid, dim3(256), 0, stream, pdl, p);
+    return after_step ? launch_kernel(k1_merge_split<false, true>, grid, dim3(256), 0, stream, pdl, p)
+                      : launch_kernel(k1_merge_split<false, false>, grid, dim3(256), 0, stream, pdl, p);
+}
+
+// The attention launch's parameters, kept for a split-unit merge enqueued later.
+static void stash_merge(const TcParams &p, bool batched, AttnMerge *m)
+{
+    static_assert(sizeof(TcParams) <= sizeof(m->params), "AttnMerge holds the attention launch's parameters");
+    memcpy(m->params, &p, sizeof p);
+    m->batched = batched;
+    m->pending = p.P > 1;
+}
+
 static size_t tc_smem_bytes()
 {
     return (size_t)(kKStages + kVStages) * kTile + 1024;
@@ -753,7 +803,7 @@ int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers)
 
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
                                  int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
-                                 const float2 *rope_tab)
+                                 const float2 *rope_tab, AttnMerge *merge_later)
 {
     if (n_seq < 1 || n_seq > kMaxSeqPerLaunch) {
         *err = "too many sequences for one attention launch";
@@ -799,29 +849,34 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     p.counters = counters;
     p.status = status;
     p.rope_tab = rope_tab;
+    p.max_rows = max_rows;
+    const bool batched = n_seq > 1;
     cudaError_t e;
-    if (n_seq == 1) {
-        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
-            return e;
-        k1_tree_attention_tc<false><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
-        if ((e = cudaGetLastError()) != cudaSuccess)
-            return e;
-        if (p.P > 1)
-            k1_merge_split<false><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
-    } else {
+    // A grid that takes every SM starts when the stream's previous work is done,
+    // so that all its CTAs start together (its work split is static); a grid
+    // capped beside a longer LM head (merge_later->pdl_launch) is launched as a
+    // programmatic dependent and its CTAs wait on SMs that are free already.
+    const bool pdl = merge_later && merge_later->pdl_launch;
+    if (batched) {
         if ((e = allow_max_smem((const void *)k1_tree_attention_tc<true>)) != cudaSuccess)
             return e;
-        k1_tree_attention_tc<true><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
-        if ((e = cudaGetLastError()) != cudaSuccess)
+        e = launch_kernel(k1_tree_attention_tc<true>, dim3(p.P), dim3(kTcThreads), tc_smem_bytes(), stream, pdl, p);
+    } else {
+        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
             return e;
-        if (p.P > 1)
-            k1_merge_split<true><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
+        e = launch_kernel(k1_tree_attention_tc<false>, dim3(p.P), dim3(kTcThreads), tc_smem_bytes(), stream, pdl, p);
     }
-    return cudaGetLastError();
+    if (e != cudaSuccess)
+        return e;
+    if (merge_later) {
+        stash_merge(p, batched, merge_later);
+        return cudaSuccess;
+    }
+    return merge_launch(p, batched, stream, false, false);
 }
 
 cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
-                                 cudaStream_t stream, const char **err)
+                                 cudaStream_t stream, const char **err, AttnMerge *merge_later)
 {
     if (sc.n_rungs < 1 || sc.n_rungs > 8) {
         *err = "scheduled attention: 1..8 rungs";
@@ -859,25 +914,36 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
     p.n_rungs = sc.n_rungs;
     for (int r = 0; r < sc.n_rungs; ++r)
         p.rung_tree[r] = sc.rung_tree[r];
-    const int max_rows = sc.N_max * p.group < 128 ? sc.N_max * p.group : 128;
+    p.max_rows = sc.N_max * p.group < 128 ? sc.N_max * p.group : 128;
     cudaError_t e;
     if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
         return e;
     k1_tree_attention_tc<false><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
     if ((e = cudaGetLastError()) != cudaSuccess)
         return e;
-    if (p.P > 1)
-        k1_merge_split<false><<<dim3(p.P - 1, (max_rows + 7) / 8), 256, 0, stream>>>(p);
-    return cudaGetLastError();
+    if (merge_later) {
+        stash_merge(p, false, merge_later);
+        return cudaSuccess;
+    }
+    return merge_launch(p, false, stream, false, false);
 }
 
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
                            const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                           cudaStream_t stream, const char **err, const float2 *rope_tab)
+                           cudaStream_t stream, const char **err, const float2 *rope_tab, AttnMerge *merge_later)
 {
     AttnSeq one{kv, d_tree, N, q, out};
     return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, counters, status, n_sm, stream, err,
-                                rope_tab);
+                                rope_tab, merge_later);
+}
+
+cudaError_t attn_merge_launch(const AttnMerge &m, cudaStream_t stream, bool after_step)
+{
+    if (!m.pending)
+        return cudaSuccess;
+    TcParams p;
+    memcpy(&p, m.params, sizeof p);
+    return merge_launch(p, m.batched, stream, true, after_step);
 }
 
 }  // namespace tv

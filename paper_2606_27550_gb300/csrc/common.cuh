@@ -294,6 +294,25 @@ __device__ __forceinline__ void fence_proxy_async_smem()
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// ------------------------------------------------------------------ programmatic dependent launch
+//
+// A kernel launched with the programmatic-serialization attribute may start
+// while the previous kernel of its stream still runs.  pdl_wait() returns once
+// that kernel has completed and its writes are visible; pdl_trigger() lets
+// the next such kernel of the stream be launched as soon as every CTA of this
+// grid has executed it.  Both are no-ops for a kernel launched without the
+// attribute.
+
+__device__ __forceinline__ void pdl_wait()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+__device__ __forceinline__ void pdl_trigger()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ misc
 
 __device__ __forceinline__ float ex2_approx(float x)

@@ -5,6 +5,27 @@
 
 namespace tv {
 
+// Launches `kernel` on `stream`; with pdl, with the programmatic-serialization
+// attribute, so that it may be launched while the previous kernel of the
+// stream still runs (the kernel waits for it with pdl_wait before touching
+// memory it writes).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                          Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = pdl ? attr : nullptr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // LM head (lm_head.cu)
 struct LmPlan {
     int R_pad, n_tiles, n_kblocks, stages, acc_cols, group_size, n_groups;
@@ -35,9 +56,12 @@ struct LmTypical {
     LmGather gather;
     float *logits_out;  // null, or [R][V] fp32: the logits themselves (speculative sampling needs whole rows)
 };
+// pdl: launched as a programmatic dependent of the stream's previous kernel (a
+// verification step's attention); the LM head does not wait for it, but
+// completes only after it
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
-                           const char **err, int expire_wait = 0, const LmTypical *typ = nullptr);
+                           const char **err, int expire_wait = 0, const LmTypical *typ = nullptr, bool pdl = false);
 
 // tree attention (attention.cu)
 struct AttnPlan {
@@ -85,11 +109,23 @@ struct AttnSeq {
     void *out;
 };
 int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers);
+// The split-unit merge of an attention launch, kept to be enqueued later in a
+// verification step by attn_merge_launch, as a programmatic dependent of the
+// stream's previous kernel: after the LM head, or (after_step) after the
+// acceptance kernel, beside which it runs.
+struct AttnMerge {
+    bool pdl_launch;  // set by the caller: launch the attention itself as a programmatic dependent
+    bool pending;
+    bool batched;
+    alignas(64) unsigned char params[8192];
+};
+cudaError_t attn_merge_launch(const AttnMerge &m, cudaStream_t stream, bool after_step);
 // rope_tab: null, or the (cos, sin) tables of rope.cu: the queries are then
 // pre-rotary and are rotated at L + depth while they are staged
+// merge_later: the split-unit merge is not enqueued but kept there
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
                                  int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
-                                 const float2 *rope_tab = nullptr);
+                                 const float2 *rope_tab = nullptr, AttnMerge *merge_later = nullptr);
 bool attn_tc_supported(int d, int rows);
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
 size_t attn_tc_slot_floats();
@@ -105,10 +141,11 @@ struct AttnSched {
     const float2 *rope_tab;  // null, or the rotary tables (pre-rotary queries)
 };
 cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
-                                 cudaStream_t stream, const char **err);
+                                 cudaStream_t stream, const char **err, AttnMerge *merge_later = nullptr);
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
                            const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                           cudaStream_t stream, const char **err, const float2 *rope_tab = nullptr);
+                           cudaStream_t stream, const char **err, const float2 *rope_tab = nullptr,
+                           AttnMerge *merge_later = nullptr);
 
 // acceptance + compaction (accept.cu)
 struct AcceptParams {
@@ -143,8 +180,10 @@ struct AcceptParams {
     const float *trace;
     const float *top1, *entropy;
 };
-cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream);
-cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream);
+// pdl: launched as a programmatic dependent of the stream's previous kernel
+// (the step's LM head), whose outputs the kernel reads after pdl_wait
+cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream, bool pdl = false);
+cudaError_t accept_launch_batch(const AcceptParams *ps, int n, int n_sm, cudaStream_t stream, bool pdl = false);
 
 // speculative sampling on the tree (sample.cu): one CTA walks the tree
 struct SampleParams {

@@ -261,6 +261,25 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
     __syncthreads();
 }
 
+// Arrival ticket of this CTA on `counter` once its writes are done: the
+// barrier orders every thread's writes before thread 0's fence (fences are
+// cumulative), and the fence orders them before the atomic, so the CTA that
+// draws the last ticket -- after a fence of its own -- reads all of them.
+// Returns true in every thread of that CTA.
+__device__ __forceinline__ bool arrive_last(int *counter, int expected, int *s_ticket)
+{
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const int t = atomicAdd(counter, 1);
+        if (t == expected - 1)
+            __threadfence();
+        *s_ticket = t;
+    }
+    __syncthreads();
+    return *s_ticket == expected - 1;
+}
+
 // Named barrier of the eight epilogue warps.
 __device__ __forceinline__ void epi_sync()
 {
@@ -282,9 +301,21 @@ __device__ __forceinline__ int lm_kb(const LmParams &p, int tile, int j)
     return x >= p.nk ? x - p.nk : x;
 }
 
+// Waits, when it goes out of scope (every exit of the kernel), for the
+// stream's previous kernel to complete.  In a verification step the LM head
+// runs beside the attention without depending on it; this keeps the step's
+// acceptance kernel, which waits for the LM head, ordered after the attention
+// as well.
+struct PdlWaitOnExit {
+    __device__ ~PdlWaitOnExit() { pdl_wait(); }
+};
+
 template <bool kTyp>
 __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constant__ LmParams p)
 {
+    // the acceptance kernel that reads this kernel's outputs may be launched now
+    pdl_trigger();
+    PdlWaitOnExit pdl_exit;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[8];
     __shared__ __align__(8) uint64_t empty_bar[8];
@@ -543,30 +574,18 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         return;
 
     // ---------------- two-level merge of the CTAs' statistics by arrival tickets
-    __threadfence();
-    __syncthreads();
     const int g = c / p.group_size;
     const int g_first = g * p.group_size;
     const int g_count = min(p.group_size, p.P - g_first);
-    if (threadIdx.x == 0)
-        s_ticket = atomicAdd(&p.counters[g], 1);
-    __syncthreads();
-    if (s_ticket != g_count - 1)
+    if (!arrive_last(&p.counters[g], g_count, &s_ticket))
         return;
-    __threadfence();
     float4 *sbuf = reinterpret_cast<float4 *>(smem);  // the drained ring
     merge_partials<kTyp>(p, p.part_cta + (size_t)g_first * p.R_pad, p.part_cta_t + (size_t)g_first * p.R_pad, g_count,
                          sbuf, p.part_group + (size_t)g * p.R_pad, p.part_group_t + (size_t)g * p.R_pad);
     if (threadIdx.x == 0)
         p.counters[g] = 0;
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0)
-        s_ticket = atomicAdd(&p.counters[p.n_groups], 1);
-    __syncthreads();
-    if (s_ticket != p.n_groups - 1)
+    if (!arrive_last(&p.counters[p.n_groups], p.n_groups, &s_ticket))
         return;
-    __threadfence();
     merge_partials<kTyp>(p, p.part_group, p.part_group_t, p.n_groups, sbuf, nullptr, nullptr);
     if (threadIdx.x == 0)
         p.counters[p.n_groups] = 0;
@@ -625,7 +644,7 @@ LmPlan lm_plan(int R, int D, int V, int n_sm)
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
-                           const char **err, int expire_wait, const LmTypical *typ)
+                           const char **err, int expire_wait, const LmTypical *typ, bool pdl)
 {
     const LmPlan pl = lm_plan(R, D, V, n_sm);
     LmParams p{};
@@ -663,15 +682,13 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
         if (e != cudaSuccess)
             return e;
-        k2_lm_head<true><<<pl.P, kLmThreads, pl.smem_bytes, stream>>>(p);
-    } else {
-        p.inv_t = 1.0f;
-        cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
-        if (e != cudaSuccess)
-            return e;
-        k2_lm_head<false><<<pl.P, kLmThreads, pl.smem_bytes, stream>>>(p);
+        return launch_kernel(k2_lm_head<true>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
     }
-    return cudaGetLastError();
+    p.inv_t = 1.0f;
+    cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
+    if (e != cudaSuccess)
+        return e;
+    return launch_kernel(k2_lm_head<false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
 }
 
 }  // namespace tv

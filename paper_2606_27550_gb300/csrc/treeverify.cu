@@ -220,45 +220,6 @@ struct tb_bank {
     TreeDesc *d_desc;
     std::vector<TreeDesc> h_desc;
     std::vector<int32_t> h_parent;  // canonical parents, capacity x 64
-    // A verification step forks the LM head onto `aux` so that it runs in the
-    // tail of the attention kernel (whose CTAs each hold a whole SM), then
-    // joins back before acceptance.  The mutex keeps one step's fork/join
-    // enqueue sequence contiguous when several host threads share the bank.
-    cudaStream_t aux;
-    cudaEvent_t ev_fork, ev_join;
-    std::mutex fork_mu;
-};
-
-// The helper stream of a step.  The LM head runs on the bank's helper stream,
-// forked from the caller's stream just before the attention launch (after the
-// rotary embedding's, if any) and joined back before acceptance; the bank's
-// fork and join events are shared, so the bank's mutex is held from the
-// object's construction to the end of the step's enqueueing.
-class HelperFork {
-  public:
-    HelperFork(const tb_bank *bank, cudaStream_t s) : bank_(const_cast<tb_bank *>(bank)), s_(s), lk_(bank_->fork_mu)
-    {
-    }
-    cudaStream_t aux() const { return bank_->aux; }
-    tb_status fork(const char *fn)
-    {
-        cudaError_t e = cudaEventRecord(bank_->ev_fork, s_);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(bank_->aux, bank_->ev_fork, 0);
-        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: fork: %s", fn, cudaGetErrorString(e));
-    }
-    tb_status join(const char *fn)
-    {
-        cudaError_t e = cudaEventRecord(bank_->ev_join, bank_->aux);
-        if (e == cudaSuccess)
-            e = cudaStreamWaitEvent(s_, bank_->ev_join, 0);
-        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: join: %s", fn, cudaGetErrorString(e));
-    }
-
-  private:
-    tb_bank *bank_;
-    cudaStream_t s_;
-    std::lock_guard<std::mutex> lk_;
 };
 
 extern "C" tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
@@ -349,18 +310,6 @@ extern "C" tb_status tb_create(tb_bank **out, int max_topologies, int device)
     }
     b->h_desc.resize(max_topologies);
     b->h_parent.assign((size_t)max_topologies * TB_MAX_NODES, -1);
-    b->aux = nullptr;
-    b->ev_fork = b->ev_join = nullptr;
-    if ((e = cudaSetDevice(device)) == cudaSuccess &&
-        (e = cudaStreamCreateWithFlags(&b->aux, cudaStreamNonBlocking)) == cudaSuccess &&
-        (e = cudaEventCreateWithFlags(&b->ev_fork, cudaEventDisableTiming)) == cudaSuccess)
-        e = cudaEventCreateWithFlags(&b->ev_join, cudaEventDisableTiming);
-    if (prev >= 0)
-        cudaSetDevice(prev);
-    if (e != cudaSuccess) {
-        tb_destroy(b);
-        return cuda_fail(e, "tb_create: helper stream / events");
-    }
     *out = b;
     return ok();
 }
@@ -436,12 +385,6 @@ extern "C" tb_status tb_destroy(tb_bank *bank)
     cudaError_t e = cudaSetDevice(bank->device);
     if (e == cudaSuccess && bank->d_desc)
         e = cudaFree(bank->d_desc);
-    if (bank->ev_fork)
-        cudaEventDestroy(bank->ev_fork);
-    if (bank->ev_join)
-        cudaEventDestroy(bank->ev_join);
-    if (bank->aux)
-        cudaStreamDestroy(bank->aux);
     if (prev >= 0)
         cudaSetDevice(prev);
     delete bank;
@@ -628,12 +571,11 @@ static RopeSeq rope_seq(const tb_kv *kv, const TreeDesc *tree)
                    tree, kv->L};
 }
 
-// The rotary embedding (if any), then the attention.  hf: the step's helper
-// stream is forked after the rotary launch, so that the LM head it carries
-// cannot occupy the SMs before the attention CTAs are placed (an attention
-// CTA needs a whole SM).
+// The rotary embedding (if any), then the attention.  merge_later: the
+// tcgen05 attention's split-unit merge is kept there, to be enqueued later in
+// the verification step.
 static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn,
-                              HelperFork *hf = nullptr)
+                              AttnMerge *merge_later = nullptr)
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
@@ -646,18 +588,13 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
         if (st != TB_OK)
             return st;
     }
-    if (hf) {
-        tb_status st = hf->fork(fn);
-        if (st != TB_OK)
-            return st;
-    }
     const int nsm = sm_count(a.bank->device);
     cudaError_t e;
     if (use_tc_attention(a.kv->head_dim, rows))
         e = attn_tc_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
                            reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
                            reinterpret_cast<int *>(ws), a.max_ctas > 0 && a.max_ctas < nsm ? a.max_ctas : nsm, stream,
-                           &err, rope ? rope_table(ws) : nullptr);
+                           &err, rope ? rope_table(ws) : nullptr, merge_later);
     else
         e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
                         reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
@@ -690,12 +627,12 @@ tb_status tv::lm_validate(const void *hidden, int R, const void *W, int D, int V
 
 static tb_status lm_enqueue(const void *hidden, int R, const void *W, int D, int V, int32_t *am, float *t1, float *en,
                             uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn, int expire_wait = 0,
-                            const LmTypical *typ = nullptr)
+                            const LmTypical *typ = nullptr, bool pdl = false)
 {
     const char *err = "";
     cudaError_t e = lm_head_launch(hidden, R, W, D, V, am, t1, en, ws + part_off,
                                    reinterpret_cast<int *>(ws + kLmCounterOff), reinterpret_cast<int *>(ws),
-                                   sm_count(current_device()), stream, &err, expire_wait, typ);
+                                   sm_count(current_device()), stream, &err, expire_wait, typ, pdl);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -876,8 +813,8 @@ extern "C" tb_status typical_accept(const tb_bank *bank, int bank_id, const int3
 
 // The attention grid beside the LM head of the same step.  The attention's
 // persistent grid normally takes one CTA per SM, each holding the whole
-// register file, so the LM head on the helper stream starts on the SMs that
-// attention CTAs release.  When the LM head is the longer of the two (a
+// register file, so the LM head (launched once every attention CTA has
+// started) runs on the SMs that attention CTAs release.  When the LM head is the longer of the two (a
 // single layer against a large vocabulary), the attention instead gets only
 // the SMs the LM head's CTAs leave free, and both run from the start.  That
 // pays when the attention on those SMs still ends well before the LM head:
@@ -974,13 +911,13 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
     lt.ent_t = tr.ent_t;
     lt.logits_out = logits;
     a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
-    HelperFork hf(bank, s);
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &hf)) != TB_OK)
+    // the chain of verify_step, with the walk between the LM head and the compaction
+    AttnMerge merge{};
+    merge.pdl_launch = a.max_ctas > 0 && kv->rope_theta == 0.f;
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &merge)) != TB_OK)
         return st;
-    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                         hf.aux(), fn, 0, &lt)) != TB_OK)
-        return st;
-    if ((st = hf.join(fn)) != TB_OK)
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s, fn,
+                         0, &lt, true)) != TB_OK)
         return st;
     if ((st = sample_enqueue(bank, bank_id, draft_tokens, logits, tr.logz_t, draft_probs, uniforms, vocab, kv->L,
                              temperature, logits + (size_t)N * vocab, result, reinterpret_cast<const int *>(ws), s,
@@ -991,10 +928,13 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
         p.result = result;
         p.from_result = 1;
         add_compaction(p, kv);
-        cudaError_t e = accept_launch(p, sm_count(bank->device), s);
+        cudaError_t e = accept_launch(p, sm_count(bank->device), s, true);
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
     }
+    cudaError_t e = attn_merge_launch(merge, s, true);
+    if (e != cudaSuccess)
+        return cuda_fail(e, fn);
     return ok();
 }
 
@@ -1050,18 +990,24 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         lt.gather.n_seq = 1;
         lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, tr.draft_logit, 0, N};
     }
-    // attention on the caller's stream; the LM head forked onto the bank's
-    // helper stream fills the SMs that attention CTAs release (or, when it is
-    // the longer of the two, the SMs the attention is kept off); join before
-    // acceptance
+    // One chain on the caller's stream: [rotary embedding,] attention (launched
+    // once the stream's previous work is done, so that all its CTAs start
+    // together), LM head, acceptance + compaction, split-unit merge; the last
+    // three are programmatic dependents of the kernel before them.  The LM head
+    // does not depend on the attention: it is launched once every attention CTA
+    // has started and fills the SMs that attention CTAs release (or, when it is
+    // the longer of the two, the SMs the attention is kept off); it completes
+    // only after the attention has, so the acceptance kernel, which waits for
+    // it, compacts the cache after the attention read it.  Nothing in the step
+    // reads the attention output, so its split units are merged beside the
+    // acceptance kernel.
     a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
-    HelperFork hf(bank, s);
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &hf)) != TB_OK)
+    AttnMerge merge{};
+    merge.pdl_launch = a.max_ctas > 0 && kv->rope_theta == 0.f;
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &merge)) != TB_OK)
         return st;
-    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
-                         hf.aux(), fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr)) != TB_OK)
-        return st;
-    if ((st = hf.join(fn)) != TB_OK)
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s, fn,
+                         (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr, true)) != TB_OK)
         return st;
     AcceptParams p =
         accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
@@ -1069,7 +1015,9 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         add_typical(p, typ, tr.logz_t, tr.ent_t, tr.draft_logit);
     if (!(flags & TB_NO_COMPACT))
         add_compaction(p, kv);
-    cudaError_t e = accept_launch(p, sm_count(bank->device), s);
+    cudaError_t e = accept_launch(p, sm_count(bank->device), s, true);
+    if (e == cudaSuccess)
+        e = attn_merge_launch(merge, s, true);
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
@@ -1161,11 +1109,10 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = (cudaStream_t)stream;
 
-    // attention on the caller's stream, the LM head forked onto the helper
-    // stream (it fills the SMs the attention CTAs release), joined before acceptance
-    // (forked after the rotary launch, so that the LM head cannot take the SMs first)
-    HelperFork hf(bank, s);
+    // the chain of verify_step: [rotary embedding,] attention, LM head,
+    // acceptance + compaction, split-unit merge
     cudaError_t e = cudaSuccess;
+    AttnMerge merge{};
     // tree attention of every sequence (after the rotary embedding of their tree keys)
     if (tc) {
         const bool rope = kv0.rope_theta != 0.f;
@@ -1179,15 +1126,13 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             if ((st = rope_enqueue(rp, &kv0, batch, 0, kv0.n_layers, max_nodes, ws, s, fn)) != TB_OK)
                 return st;
         }
-        if ((st = hf.fork(fn)) != TB_OK)
-            return st;
         AttnSeq as[TB_MAX_BATCH];
         for (int b = 0; b < batch; ++b)
             as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
         const char *err = "";
         e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err, rope ? rope_table(ws) : nullptr);
+                                 &err, rope ? rope_table(ws) : nullptr, &merge);
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
@@ -1198,7 +1143,7 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             AttnPlan plan;
             if ((st = attn_validate(a, fn, &plan)) != TB_OK)
                 return st;
-            if ((st = attn_enqueue(a, ws, kPartBase, s, fn, b == 0 ? &hf : nullptr)) != TB_OK)
+            if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
                 return st;
         }
     }
@@ -1223,13 +1168,12 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
                 sr += Ns[b];
             }
         }
+        // the chunks share the partials and counters: only the first overlaps the attention
         if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
-                             entropy + r0, ws, kPartBase + attn_bytes, bank->aux, fn, 0, typ ? &lt : nullptr)) !=
+                             entropy + r0, ws, kPartBase + attn_bytes, s, fn, 0, typ ? &lt : nullptr, r0 == 0)) !=
             TB_OK)
             return st;
     }
-    if ((st = hf.join(fn)) != TB_OK)
-        return st;
     // acceptance + compaction, one launch
     AcceptParams ps[TB_MAX_BATCH];
     int r0 = 0;
@@ -1242,7 +1186,9 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             add_compaction(ps[b], &seqs[b].kv);
         r0 += Ns[b];
     }
-    e = accept_launch_batch(ps, batch, nsm, s);
+    e = accept_launch_batch(ps, batch, nsm, s, true);
+    if (e == cudaSuccess)
+        e = attn_merge_launch(merge, s, true);
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
@@ -1342,6 +1288,9 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
         return fail(TB_EINVAL, "%s: n_q_heads %d not a multiple of n_kv_heads %d", fn, n_q_heads, kv->n_kv_heads);
     if (N_max * (n_q_heads / kv->n_kv_heads) > 256)
         return fail(TB_EUNSUPPORTED, "%s: N_max * group = %d > 256", fn, N_max * (n_q_heads / kv->n_kv_heads));
+    if ((long long)kv->n_layers * kv->n_kv_heads * ((N_max * (n_q_heads / kv->n_kv_heads) + 127) / 128) >
+        kMaxAttnUnits)
+        return fail(TB_EUNSUPPORTED, "%s: more than %d attention units", fn, kMaxAttnUnits);
     if (!q || !attn_out || !aligned16(q) || !aligned16(attn_out))
         return fail(TB_EINVAL, "%s: q / attn_out NULL or not 16-byte aligned", fn);
     if (!draft_tokens || !result)
@@ -1364,8 +1313,10 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     sc.out = attn_out;
     for (int r = 0; r < policy->n_rungs; ++r)
         sc.rung_tree[r] = bank->d_desc + policy->bank_ids[r];
+    // the chain of verify_step, with the split-unit merge before the acceptance
+    // kernel, which moves the device state on to the next step
+    AttnMerge merge{};
     {
-        HelperFork hf(bank, s);
         if (kv->rope_theta != 0.f) {
             RopeParams rp{};
             rp.seq[0] = rope_seq(kv, sc.rung_tree[0]);
@@ -1378,21 +1329,19 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
                 return st;
             sc.rope_tab = rope_table(ws);
         }
-        if ((st = hf.fork(fn)) != TB_OK)  // after the rotary launch: the attention CTAs are placed first
-            return st;
         const char *err = "";
         cudaError_t e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err);
+                                 &err, &merge);
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
         if ((st = lm_enqueue(hidden, N_max, lm_head, d_model, vocab, argmax, top1, entropy, ws,
-                             kPartBase + attn_bytes, hf.aux(), fn)) != TB_OK)
+                             kPartBase + attn_bytes, s, fn, 0, nullptr, true)) != TB_OK)
             return st;
-        if ((st = hf.join(fn)) != TB_OK)
-            return st;
+        if ((e = attn_merge_launch(merge, s, false)) != cudaSuccess)
+            return cuda_fail(e, fn);
     }
     AcceptParams p = accept_params(bank, policy->bank_ids[0], draft_tokens, argmax, vocab, 0, result,
                                    reinterpret_cast<const int *>(ws));
@@ -1416,7 +1365,7 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     p.trace = policy->trace;
     p.top1 = top1;
     p.entropy = entropy;
-    cudaError_t e = accept_launch(p, nsm, s);
+    cudaError_t e = accept_launch(p, nsm, s, true);
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
