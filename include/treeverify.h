@@ -164,6 +164,18 @@ TB_API tb_status tb_workspace_init(void *workspace, size_t workspace_bytes, tb_s
  * device-detected error (TB_ETIMEOUT, TB_EINVAL). */
 TB_API tb_status tb_workspace_status(const void *workspace, int32_t *status);
 
+/* Test support for the debug build of the library (compiled with
+ * TB_DEBUG_BOUNDS; the paper has no counterpart).  In that build every kernel
+ * checks its global-memory indices against the extents it was given; a failed
+ * check skips the access, raises an error bit in the workspace status word
+ * (reported as TB_EINVAL by tb_workspace_status and in tb_result.status) and
+ * is counted.  tb_debug_bounds_violations synchronises the device, stores the
+ * number of failed checks since its previous call in *count and resets it
+ * (always 0 in a normal build).  tb_debug_bounds_build returns 1 in the debug
+ * build, 0 otherwise. */
+TB_API tb_status tb_debug_bounds_violations(uint32_t *count);
+TB_API int tb_debug_bounds_build(void);
+
 /* ------------------------------------------------------------------------
  * The verification pass and its stages
  * ---------------------------------------------------------------------- */

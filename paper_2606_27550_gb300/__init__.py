@@ -18,7 +18,10 @@ from dataclasses import dataclass
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libtreeverify.so")
+# TB_DEBUG_BOUNDS=1 in the environment selects the debug build of the library,
+# whose kernels check their global indices (build.build(debug_bounds=True))
+LIB_PATH = os.path.join(_HERE, "libtreeverify_debug.so" if os.environ.get("TB_DEBUG_BOUNDS") == "1"
+                        else "libtreeverify.so")
 
 TB_OK, TB_EINVAL, TB_ENOMEM, TB_ECUDA, TB_ENOTFOUND, TB_ECAPACITY, TB_ETIMEOUT, TB_EUNSUPPORTED = (
     0, -1, -2, -3, -4, -5, -6, -7)
@@ -33,7 +36,8 @@ API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb
        "tb_last_error",
        "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
        "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical",
-       "verify_step_scheduled", "spec_sample_accept", "verify_step_sampled")
+       "verify_step_scheduled", "spec_sample_accept", "verify_step_sampled", "tb_debug_bounds_violations",
+       "tb_debug_bounds_build")
 
 
 class TreeVerifyError(RuntimeError):
@@ -104,6 +108,8 @@ def load(path: str = LIB_PATH):
         "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
         "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, i32, P],
         "lm_head_stats_noalloc_status": [P, P],
+        "tb_debug_bounds_violations": [P],
+        "tb_debug_bounds_build": [],
         "verify_step_batched": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, sz, i32, P],
         "tb_last_error": [],
         "lm_head_stats_typical": [P, i32, P, P, i32, i32, ctypes.c_float, P, P, P, P, P, P, P, P, sz, P],
@@ -312,6 +318,18 @@ def lm_head_stats_noalloc(hidden, lm_head, argmax, top1, entropy, flags: int = 0
     R, D = hidden.shape
     _check(load().lm_head_stats_noalloc(_ptr(hidden), R, _ptr(lm_head), D, lm_head.shape[0], _ptr(argmax),
                                         _ptr(top1), _ptr(entropy), flags, _stream(stream)), "lm_head_stats_noalloc")
+
+
+def tb_debug_bounds_violations() -> int:
+    """Failed index checks of the debug build's kernels since the last call
+    (0 in a normal build); synchronises the device."""
+    n = ctypes.c_uint32(0)
+    _check(load().tb_debug_bounds_violations(ctypes.byref(n)), "tb_debug_bounds_violations")
+    return int(n.value)
+
+
+def tb_debug_bounds_build() -> bool:
+    return bool(load().tb_debug_bounds_build())
 
 
 def lm_head_stats_noalloc_status(stream=None) -> int:

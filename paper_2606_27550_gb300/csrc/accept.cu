@@ -36,7 +36,8 @@ namespace tv {
 // and a chunk's writes land below every source of the later chunks: each chunk
 // loads all of its source rows, then stores them.  A warp covers 512 bytes per
 // pass: 512 / row_bytes rows side by side (row_bytes a multiple of 16, <= 512).
-__device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k, int row_bytes, int room, int lane)
+__device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k, int row_bytes, int room, int lane,
+                                          int *status)
 {
     constexpr int kChunk = 8;
     const int lanes_per_row = row_bytes >> 4;
@@ -60,7 +61,7 @@ __device__ __forceinline__ void copy_rows(uint8_t *base, const int *path, int k,
             const int j = j0 + r_in + m * rows_per_pass;
             if (m * rows_per_pass < kChunk && j < k && j < j0 + kChunk) {
                 const int src = path[j];
-                if (src > j && src < room)
+                if (src > j && src < room && in_bounds(j < room && off + 16 <= row_bytes, status))
                     *reinterpret_cast<uint4 *>(base + (size_t)j * row_bytes + off) = buf[m];
             }
         }
@@ -171,7 +172,8 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
             for (int h = 0; h < 2; ++h) {
                 const int i = lane + 32 * h;
                 bool m = false;
-                if (i >= 1 && i < n) {
+                if (i >= 1 && i < n && in_bounds(n <= kMaxNodes && t->parent[i] >= 0 && t->parent[i] < i,
+                                                 const_cast<int *>(p.ws_status))) {
                     const int tok = draft[i];
                     const bool bad_tok = (tok < 0 || tok >= p.vocab);
                     bad |= bad_tok;
@@ -278,7 +280,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                         st = s_err;
                     else if (ws & kStatusTimeout)
                         st = TB_ETIMEOUT;
-                    else if (any_bad || (ws & kStatusBadToken))
+                    else if (any_bad || (ws & (kStatusBadToken | kStatusBounds)))
                         st = TB_EINVAL;
                     r->new_L = (p.sched && s_err != TB_OK) ? p.sched[1] : L + len;
                     r->status = st;
@@ -303,7 +305,9 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
             const int head = lh % p.n_kv_heads, layer = lh / p.n_kv_heads;
             uint8_t *base = (which ? p.v : p.k) + layer * p.layer_stride_b + head * p.head_stride_b +
                             (size_t)L * p.row_bytes;
-            copy_rows(base, s_path, k, p.row_bytes, p.L_cap - L, lane);
+            if (in_bounds(layer < p.n_layers && head < p.n_kv_heads && k <= kMaxNodes,
+                          const_cast<int *>(p.ws_status)))
+                copy_rows(base, s_path, k, p.row_bytes, p.L_cap - L, lane, const_cast<int *>(p.ws_status));
         }
     }
     if (!p.sched)
@@ -346,5 +350,7 @@ cudaError_t accept_launch(const AcceptParams &p, int n_sm, cudaStream_t stream, 
 {
     return accept_launch_batch(&p, 1, n_sm, stream, pdl);
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_accept)
 
 }  // namespace tv

@@ -170,10 +170,15 @@ __global__ void __launch_bounds__(160, 2) k1_tree_attention(const __grid_constan
 
         // rows owned by this thread: r0 = warp*16 + g, r1 = r0 + 8 (within the block)
         const int lr0 = warp * 16 + g, lr1 = lr0 + 8;
-        const bool v0 = lr0 < rows_here, v1 = lr1 < rows_here;
+        bool v0 = lr0 < rows_here, v1 = lr1 < rows_here;
         const int gr0 = rb * 64 + lr0, gr1 = rb * 64 + lr1;
         const int node0 = v0 ? gr0 / p.group : 0, node1 = v1 ? gr1 / p.group : 0;
         const int qh0 = head * p.group + gr0 % p.group, qh1 = head * p.group + gr1 % p.group;
+        // the rows' query / output rows and tree entries
+        if (!in_bounds(layer_rel < p.n_layers && c < p.P && (!v0 || (node0 < p.N && node0 < kMaxNodes && qh0 < p.Hq)) &&
+                           (!v1 || (node1 < p.N && node1 < kMaxNodes && qh1 < p.Hq)),
+                       p.status))
+            v0 = v1 = false;
         const uint64_t anc0 = v0 ? p.tree->anc[node0] : 0ull;
         const uint64_t anc1 = v1 ? p.tree->anc[node1] : 0ull;
 
@@ -392,9 +397,11 @@ __global__ void __launch_bounds__(160, 2) k1_tree_attention(const __grid_constan
                 const int node = grow / p.group;
                 const int qh = head * p.group + grow % p.group;
                 __nv_bfloat16 *op = p.out + (((size_t)layer_rel * p.N + node) * p.Hq + qh) * D + c0;
+                if (in_bounds(node < p.N && qh < p.Hq && c_lo >= 0 && c_hi < p.P, p.status)) {
 #pragma unroll
-                for (int x = 0; x < D / 2; x += 2)
-                    *reinterpret_cast<uint32_t *>(op + x) = pack_bf16x2(acc[x] * inv, acc[x + 1] * inv);
+                    for (int x = 0; x < D / 2; x += 2)
+                        *reinterpret_cast<uint32_t *>(op + x) = pack_bf16x2(acc[x] * inv, acc[x + 1] * inv);
+                }
             }
             if (threadIdx.x == 0)
                 p.counters[u] = 0;
@@ -475,5 +482,7 @@ cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int laye
     k1_tree_attention<64><<<pl.P, 160, attn_smem_bytes(d), stream>>>(p);
     return cudaGetLastError();
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_attention)
 
 }  // namespace tv

@@ -360,6 +360,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             const int grow = g.rb * 128 + rloc;
             g.node = g.valid ? grow / p.group : 0;
             g.qh = g.head * p.group + grow % p.group;
+            // the row's query / output rows and tree entries
+            if (g.valid)
+                g.valid = in_bounds(g.layer_rel < p.n_layers && g.node < sq.N && g.node < sq.nstride &&
+                                        g.node < kMaxNodes && g.qh < p.Hq,
+                                    p.status);
             g.anc = g.valid ? sq.tree->anc[g.node] : 0ull;
             g.dep = g.valid ? sq.tree->depth[g.node] : 0;
             g.L = sq.L;
@@ -561,6 +566,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             tc_fence_after();
             const bool whole = (g.start == g.u_first && g.end == g.u_last);
             float *slot = p.part + ((size_t)c * 2 + (g.start == t0 ? 0 : 1)) * kSlot;
+            if (!whole && g.valid)
+                g.valid = in_bounds(c < p.P && rloc < 128, p.status);
             {
                 const float inv = 1.f / l;
                 uint4 *dst =
@@ -678,6 +685,13 @@ __global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__
     const int r = blockIdx.y * 8 + warp;
     if (r >= rows_here)
         return;
+    {
+        const int grow = rb * 128 + r;
+        if (!in_bounds(c_lo >= 0 && c_hi < p.P && layer_rel < p.n_layers && grow / p.group < sq.nstride &&
+                           head * p.group + grow % p.group < p.Hq,
+                       p.status))
+            return;
+    }
     // lane j of each 32-slot block owns slot c_lo + j0 + j: its row pointer, max and weight
     float M = -INFINITY;
     for (int j0 = 0; j0 < nseg; j0 += 32) {
@@ -842,6 +856,7 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     p.Hkv = Hkv;
     p.group = Hq / Hkv;
     p.layer_begin = layer_begin;
+    p.n_layers = n_layers;
     p.total = tiles;
     p.P = (int)(tiles < n_sm ? tiles : n_sm);
     p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
@@ -945,5 +960,7 @@ cudaError_t attn_merge_launch(const AttnMerge &m, cudaStream_t stream, bool afte
     memcpy(&p, m.params, sizeof p);
     return merge_launch(p, m.batched, stream, true, after_step);
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_attention_tc)
 
 }  // namespace tv

@@ -27,6 +27,56 @@ struct alignas(64) TreeDesc {
 // Status bits kept in the workspace status word.
 constexpr int kStatusTimeout = 1;
 constexpr int kStatusBadToken = 2;
+constexpr int kStatusBounds = 4;  // a debug build found a global index outside its buffer
+
+// ------------------------------------------------------------------ debug bounds checks
+//
+// A library built with TB_DEBUG_BOUNDS checks the global-memory indices of its
+// kernels against the extents each kernel was given (rows, nodes, heads,
+// layers, cache slots, partial slots, vocabulary).  A failed check skips the
+// access, raises kStatusBounds in the status word (when the kernel has one)
+// and counts the violation in a device counter of its translation unit, which
+// tb_debug_bounds_violations() reads.  Nothing traps.  In a normal build
+// in_bounds() is `true` and the checks compile away.
+#ifdef TB_DEBUG_BOUNDS
+static __device__ unsigned int g_bounds_violations;
+
+__device__ __forceinline__ bool in_bounds(bool ok, int *status)
+{
+    if (!ok) {
+        atomicAdd(&g_bounds_violations, 1u);
+        if (status)
+            atomicOr(status, kStatusBounds);
+    }
+    return ok;
+}
+#else
+__device__ __forceinline__ bool in_bounds(bool, int *)
+{
+    return true;
+}
+#endif
+
+// Host side: this translation unit's violation count since the last call
+// (0 in a normal build).  Each .cu file with kernels defines one, named after
+// the file.
+#ifdef TB_DEBUG_BOUNDS
+#define TB_BOUNDS_COUNTER(name)                                                              \
+    unsigned int name()                                                                      \
+    {                                                                                        \
+        unsigned int n = 0, zero = 0;                                                        \
+        if (cudaMemcpyFromSymbol(&n, g_bounds_violations, sizeof n) != cudaSuccess)          \
+            return 0xffffffffu;                                                              \
+        cudaMemcpyToSymbol(g_bounds_violations, &zero, sizeof zero);                         \
+        return n;                                                                            \
+    }
+#else
+#define TB_BOUNDS_COUNTER(name) \
+    unsigned int name()         \
+    {                           \
+        return 0;               \
+    }
+#endif
 
 // Every bounded wait gives up after this many SM clock cycles (about one
 // second at the 1.4-2.1 GHz SM clock).  The deadline is checked with the

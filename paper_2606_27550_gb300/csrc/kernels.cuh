@@ -201,6 +201,15 @@ struct SampleParams {
 };
 cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream);
 
+// Debug-bounds violation counters of the kernel translation units (0 in a
+// normal build); each call resets the count it returns.
+unsigned int bounds_violations_attention();
+unsigned int bounds_violations_attention_tc();
+unsigned int bounds_violations_lm_head();
+unsigned int bounds_violations_accept();
+unsigned int bounds_violations_rope();
+unsigned int bounds_violations_sample();
+
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once
 // per (kernel, device) (treeverify.cu).
 cudaError_t allow_max_smem(const void *kernel);

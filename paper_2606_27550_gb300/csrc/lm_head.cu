@@ -37,6 +37,7 @@ struct LmParams {
     int n_tiles, nk, stages, acc_cols;
     int P;               // CTAs
     int group_size, n_groups;
+    size_t smem_avail;   // dynamic shared memory after alignment (the merges stage partials there)
     float4 *part_cta;    // [P][R_pad]  (max, argmax bits, s, t)
     float4 *part_group;  // [n_groups][R_pad]
     float2 *part_cta_t;  // [P][R_pad]  (sT, tT), typical mode
@@ -177,6 +178,8 @@ __device__ void merge_partials(const LmParams &p, const float4 *src, const float
     // and a load-then-store loop would pay one round trip per element
     constexpr int kInFlight = 8;
     const int n = count * p.R_pad;
+    if (!in_bounds((size_t)n * sizeof(float4) <= p.smem_avail, p.status))
+        return;
     for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kInFlight) {
         float4 v[kInFlight];
 #pragma unroll
@@ -528,7 +531,9 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                         for (int h = e; h < nhit; h += kEpiThreads) {
                             const int w = s_hit[h];
                             const int row = (w >> 7) & 0x1ff;
-                            if (row >= c0 && row < c0 + kLmChunk)
+                            if (row >= c0 && row < c0 + kLmChunk &&
+                                in_bounds((w >> 24) < p.gather.n_seq && ((w >> 16) & 0xff) < p.gather.seq[w >> 24].n,
+                                          p.status))
                                 p.gather.seq[w >> 24].out[(w >> 16) & 0xff] = chunk[(row - c0) * kChunkLd + (w & 0x7f)];
                         }
                     } else {
@@ -663,6 +668,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.P = pl.P;
     p.group_size = pl.group_size;
     p.n_groups = pl.n_groups;
+    p.smem_avail = pl.smem_bytes - 1024;
     p.part_cta = static_cast<float4 *>(parts);
     p.part_group = p.part_cta + (size_t)pl.P * pl.R_pad;
     p.part_cta_t = reinterpret_cast<float2 *>(p.part_group + (size_t)pl.n_groups * pl.R_pad);
@@ -690,5 +696,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         return e;
     return launch_kernel(k2_lm_head<false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_lm_head)
 
 }  // namespace tv

@@ -56,7 +56,7 @@ __global__ void __launch_bounds__(kRopeThreads) k0_rope_tree_k(const __grid_cons
         const int r = blockIdx.y * kRopeRowsPerCta + k * (kRopeThreads / 8) + (threadIdx.x >> 3);
         row[k] = nullptr;
         lo[k] = hi[k] = make_uint4(0, 0, 0, 0);
-        if (r < n_rows) {
+        if (r < n_rows && in_bounds((long long)(L + j + 1) * (2 * kHalf) <= sq.head_stride && dep < kMaxNodes, nullptr)) {
             const int head = r % p.Hkv, layer = p.layer_begin + r / p.Hkv;
             row[k] = sq.k + (size_t)layer * sq.layer_stride + (size_t)head * sq.head_stride +
                      (size_t)(L + j) * (2 * kHalf);
@@ -108,5 +108,7 @@ cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_lay
                      stream>>>(p, n_rows);
     return cudaGetLastError();
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_rope)
 
 }  // namespace tv

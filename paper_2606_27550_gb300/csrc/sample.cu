@@ -132,6 +132,8 @@ __global__ void __launch_bounds__(kSampleThreads) k4_spec_sample(const __grid_co
     const TreeDesc *t = p.tree;
     const int n = t->n;
     const int tid = threadIdx.x;
+    if (!in_bounds(n >= 1 && n <= kMaxNodes, const_cast<int *>(p.ws_status)))
+        return;
     if (tid < kMaxNodes) {
         s_par[tid] = tid < n ? t->parent[tid] : -2;
         s_draft[tid] = tid < n ? p.draft[tid] : 0;
@@ -235,7 +237,8 @@ __global__ void __launch_bounds__(kSampleThreads) k4_spec_sample(const __grid_co
         res->bonus_token = s_tok == 0x7fffffff ? p.V - 1 : s_tok;  // threshold at the total: the last token
         res->new_L = p.L + len;
         const int ws = p.ws_status ? *p.ws_status : 0;
-        res->status = (ws & kStatusTimeout) ? TB_ETIMEOUT : ((bad || (ws & kStatusBadToken)) ? TB_EINVAL : TB_OK);
+        res->status = (ws & kStatusTimeout) ? TB_ETIMEOUT
+                                            : ((bad || (ws & (kStatusBadToken | kStatusBounds))) ? TB_EINVAL : TB_OK);
     }
 }
 
@@ -366,6 +369,8 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
     const int tid = threadIdx.x, lane = tid & 31;
     const TreeDesc *t = p.tree;
     const int n = t->n;
+    if (!in_bounds(n >= 1 && n <= kMaxNodes, const_cast<int *>(p.ws_status)))
+        return;  // the same tree in every CTA: the whole cluster returns before its first barrier
     if (tid < kMaxNodes)
         s_kids[tid] = 0;
     if (tid == 0)
@@ -502,7 +507,8 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
         res->bonus_token = tok == 0x7fffffff ? p.V - 1 : tok;  // threshold at the total: the last token
         res->new_L = p.L + len;
         const int ws = p.ws_status ? *p.ws_status : 0;
-        res->status = (ws & kStatusTimeout) ? TB_ETIMEOUT : ((bad || (ws & kStatusBadToken)) ? TB_EINVAL : TB_OK);
+        res->status = (ws & kStatusTimeout) ? TB_ETIMEOUT
+                                            : ((bad || (ws & (kStatusBadToken | kStatusBounds))) ? TB_EINVAL : TB_OK);
     }
     cluster_sync();  // no CTA exits while rank 0 reads its shared memory
 }
@@ -517,5 +523,7 @@ cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream)
         k4_spec_sample<<<1, kSampleThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
+
+TB_BOUNDS_COUNTER(bounds_violations_sample)
 
 }  // namespace tv

@@ -437,8 +437,36 @@ extern "C" tb_status tb_workspace_status(const void *workspace, int32_t *status)
     cudaError_t e = cudaMemcpy(&w, workspace, sizeof w, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess)
         return cuda_fail(e, "tb_workspace_status");
-    *status = (w & kStatusTimeout) ? TB_ETIMEOUT : (w & kStatusBadToken) ? TB_EINVAL : TB_OK;
+    *status = (w & kStatusTimeout) ? TB_ETIMEOUT : (w & (kStatusBadToken | kStatusBounds)) ? TB_EINVAL : TB_OK;
     return ok();
+}
+
+extern "C" tb_status tb_debug_bounds_violations(uint32_t *count)
+{
+    if (!count)
+        return fail(TB_EINVAL, "tb_debug_bounds_violations: count is NULL");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess)
+        return cuda_fail(e, "tb_debug_bounds_violations");
+    unsigned int n = 0;
+    for (unsigned int (*f)() : {bounds_violations_attention, bounds_violations_attention_tc, bounds_violations_lm_head,
+                                bounds_violations_accept, bounds_violations_rope, bounds_violations_sample}) {
+        const unsigned int x = f();
+        if (x == 0xffffffffu)
+            return fail(TB_ECUDA, "tb_debug_bounds_violations: reading a device counter failed");
+        n += x;
+    }
+    *count = n;
+    return ok();
+}
+
+extern "C" int tb_debug_bounds_build(void)
+{
+#ifdef TB_DEBUG_BOUNDS
+    return 1;
+#else
+    return 0;
+#endif
 }
 
 // ------------------------------------------------------------------ validation helpers

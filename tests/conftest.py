@@ -138,3 +138,9 @@ def guard_canaries(request):
         guards.uninstall()
     bad = guards.check()
     assert not bad, f"a kernel wrote outside {len(bad)} device buffer(s) of {bad} bytes (guard canaries overwritten)"
+    if os.environ.get("TB_DEBUG_BOUNDS") == "1":
+        # the debug build of the library: no kernel may have failed an index check
+        import paper_2606_27550_gb300 as tv
+
+        n = tv.tb_debug_bounds_violations()
+        assert n == 0, f"{n} global-memory index checks failed in the debug build"
