@@ -39,6 +39,10 @@ import numpy as np  # noqa: E402
 from paper_2606_27550_gb300 import synth  # noqa: E402
 
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_BYTES = 129 << 20  # GB300 L2
+# the bank loop's L2 policy: the cache is compacted in place every step, so it cannot rotate
+C3_L2 = ("inputs larger than L2 every step: the LM head (262 MB) streams through L2 between one step's cache "
+         "reads (34-130 MB as L grows) and the next's")
 NOMINAL_HBM_GBS = 8000.0  # nominal HBM3e bandwidth, for context beside the measured copy peak
 
 
@@ -159,6 +163,32 @@ def acceptance_label(args) -> str:
     return "greedy"
 
 
+def l2_plan(sh, kv_bytes: int, w_bytes: int):
+    """(copies, bytes of one copy, description) of the L2 policy of run_gpu: when a step's
+    cache, queries and hidden rows (and the LM head, when it is small too) fit in L2, the
+    timed steps rotate over enough copies of them that a step's data was last read more
+    than twice the L2 size of traffic earlier."""
+    cache = sh.n_layers * sh.n_kv_heads * sh.L_cap * sh.head_dim * 2 * 2
+    qh = sh.n_layers * sh.N * sh.n_q_heads * sh.head_dim * 2 + sh.N * sh.d_model * 2
+    small = cache + qh + (w_bytes if w_bytes < L2_BYTES else 0)
+    if small >= 2 * L2_BYTES:
+        return 1, small, f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)"
+    n = min(512, -(-2 * L2_BYTES // small))
+    if w_bytes >= L2_BYTES:
+        return n, small, (f"the timed steps rotate over {n} copies of the cache, queries and hidden rows "
+                          f"({small / 1e6:.1f} MB each); the LM head of {w_bytes / 1e6:.0f} MB streams through L2 "
+                          f"every step")
+    return n, small, f"the timed steps rotate over {n} copies of every input ({small / 1e6:.2f} MB each)"
+
+
+def workload_config(args, sh, kv_bytes: int, w_bytes: int) -> dict:
+    """The `config` of the JSON line (both arms)."""
+    return {"workload": sh.name, "layers": sh.n_layers, "q_heads": sh.n_q_heads, "kv_heads": sh.n_kv_heads,
+            "head_dim": sh.head_dim, "L": sh.L, "tree_nodes": sh.N, "tree_depth": int(synth.depth_of(sh.parent).max()),
+            "d_model": sh.d_model, "vocab": sh.vocab, "batch": 1, "l2": l2_plan(sh, kv_bytes, w_bytes)[2],
+            "acceptance": acceptance_label(args), "rope": "in-kernel, theta 10000" if args.rope else "none"}
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -189,6 +219,15 @@ def run_gpu(args):
     # --rope: the queries and tree keys are pre-rotary and every call applies the rotary
     # embedding at L + depth (the tree slots are rotated in place again each step: timing only)
     kv = tv.KvCache(k, v, L, rope_theta=10000.0 if args.rope else 0.0)
+    # L2 policy: when a step's cache, queries and hidden rows (and the LM head, when it is
+    # small too) fit in L2, the timed steps rotate over enough copies of them that a step's
+    # data was last read more than twice the L2 size of traffic earlier
+    n_copies, _, _ = l2_plan(sh, kv_bytes, w_bytes)
+    rot = [(kv, q, hidden, W)]
+    for c in range(1, n_copies):
+        kc, vc = torch.empty_like(k).copy_(k), torch.empty_like(v).copy_(v)
+        rot.append((tv.KvCache(kc, vc, L, rope_theta=kv.rope_theta), q.clone(), hidden.clone(),
+                    W.clone() if W.numel() * 2 < L2_BYTES else W))
     out = torch.empty((nl, N, H, d), dtype=bf, device=dev)
     am = torch.empty(N, dtype=torch.int32, device=dev)
     t1 = torch.empty(N, dtype=torch.float32, device=dev)
@@ -219,31 +258,35 @@ def run_gpu(args):
         lgs = torch.empty((N + 1, V), dtype=torch.float32, device=dev)
         del zf
 
-    def step(qq=q, hh=hidden, dd=drafts, st=None, outs=None):
+    def step(qq=q, hh=hidden, dd=drafts, st=None, outs=None, kvx=kv, Wx=W):
         st = stream if st is None else st
         oam, ot1, oen, ores = (am, t1, en, res) if outs is None else outs
         if sampled:
-            tv.verify_step_sampled(bank, bid, kv, qq, hh, W, dd, qd, unif, 0.7, out, oam, ot1, oen, lgs, ores, ws,
+            tv.verify_step_sampled(bank, bid, kvx, qq, hh, Wx, dd, qd, unif, 0.7, out, oam, ot1, oen, lgs, ores, ws,
                                    0, st)
         elif typical:
-            tv.verify_step_typical(bank, bid, kv, qq, hh, W, dd, out, oam, ot1, oen, ores, ws, *tv.PAPER_TYPICAL,
+            tv.verify_step_typical(bank, bid, kvx, qq, hh, Wx, dd, out, oam, ot1, oen, ores, ws, *tv.PAPER_TYPICAL,
                                    0, st)
         else:
-            tv.verify_step(bank, bid, kv, qq, hh, W, dd, out, oam, ot1, oen, ores, ws, 0, st)
+            tv.verify_step(bank, bid, kvx, qq, hh, Wx, dd, out, oam, ot1, oen, ores, ws, 0, st)
+
+    def rstep(i):
+        kvx, qq, hh, Wx = rot[i % n_copies]
+        step(qq, hh, kvx=kvx, Wx=Wx)
 
     visible = os.environ.get("CUDA_VISIBLE_DEVICES")
     sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
     sampler.start()
-    for _ in range(args.warmup):
-        step()
+    for i in range(args.warmup):
+        rstep(i)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
-        step()
+    for i in range(args.steps):
+        rstep(args.warmup + i)
     e1.record(stream)
     torch.cuda.synchronize()
     elapsed_ms = e0.elapsed_time(e1)
@@ -258,23 +301,31 @@ def run_gpu(args):
     # keep the GPU busy while the host enqueues, so that the events bracket
     # device time only (no host launch gaps between stages)
     torch.cuda._sleep(200_000_000)
+    nvtx = torch.cuda.nvtx
     for i in range(n_k):
+        kvx, qq, hh, Wx = rot[i % n_copies]
         ev[i][0].record(stream)
+        nvtx.range_push("lm_head")
         if typical or sampled:
-            tv.lm_head_stats_typical(bank, bid, hidden, W, tv.PAPER_TYPICAL[0], drafts, am, t1, en, lz, et, dl, ws,
+            tv.lm_head_stats_typical(bank, bid, hh, Wx, tv.PAPER_TYPICAL[0], drafts, am, t1, en, lz, et, dl, ws,
                                      stream)
         else:
-            tv.lm_head_stats(hidden, W, am, t1, en, ws, stream)
+            tv.lm_head_stats(hh, Wx, am, t1, en, ws, stream)
+        nvtx.range_pop()
         ev[i][1].record(stream)
-        tv.tree_attention(bank, bid, kv, q, out, ws, 0, nl, stream)
+        nvtx.range_push("tree_attention")
+        tv.tree_attention(bank, bid, kvx, qq, out, ws, 0, nl, stream)
+        nvtx.range_pop()
         ev[i][2].record(stream)
+        nvtx.range_push("acceptance+compaction")
         if sampled:
             tv.spec_sample_accept(bank, bid, drafts, lgs[:N], lz, qd, unif, L, 0.7, lgs[N], res, stream)
         elif typical:
             tv.typical_accept(bank, bid, drafts, am, lz, et, dl, V, L, res, *tv.PAPER_TYPICAL, stream=stream)
         else:
             tv.greedy_accept(bank, bid, drafts, am, V, L, res, stream)
-        tv.kv_compact(kv, res, stream)
+        tv.kv_compact(kvx, res, stream)
+        nvtx.range_pop()
         ev[i][3].record(stream)
     torch.cuda.synchronize()
     t_lm = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
@@ -367,10 +418,7 @@ def run_gpu(args):
         "dtype": "bf16",
         "data": "synthetic (seeded normal bf16 K/V, queries, hidden rows; LM head N(0, 0.02^2)); "
                 "drafts = parent greedy token with p, else uniform",
-        "config": {"workload": sh.name, "layers": nl, "q_heads": H, "kv_heads": Hkv, "head_dim": d, "L": L,
-                   "tree_nodes": N, "tree_depth": int(synth.depth_of(sh.parent).max()), "d_model": D, "vocab": V,
-                   "batch": 1, "l2": f"inputs larger than L2 ({(kv_bytes + w_bytes) / 1e9:.2f} GB read per step)",
-                   "acceptance": acceptance_label(args), "rope": "in-kernel, theta 10000" if args.rope else "none"},
+        "config": workload_config(args, sh, kv_bytes, w_bytes),
         "tree_tokens_per_s": round(value * N, 1),
         "hbm_roofline": {"bytes_per_step": kv_bytes + w_bytes,
                          "frac": round((kv_bytes + w_bytes) / (ms * 1e-3) / 1e9 / hbm, 4),
@@ -456,10 +504,9 @@ def run_gpu_batched(args):
 
     def step():
         if args.accept == "typical":
-            tv.verify_step_batched_typical(bank, seqs, hidden, W, am, t1, en, ws, *tv.PAPER_TYPICAL,
-                                           tv.TB_NO_COMPACT, stream)
+            tv.verify_step_batched_typical(bank, seqs, hidden, W, am, t1, en, ws, *tv.PAPER_TYPICAL, 0, stream)
         else:
-            tv.verify_step_batched(bank, seqs, hidden, W, am, t1, en, ws, tv.TB_NO_COMPACT, stream)
+            tv.verify_step_batched(bank, seqs, hidden, W, am, t1, en, ws, 0, stream)
 
     sampler = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]
                            if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
@@ -497,8 +544,8 @@ def run_gpu_batched(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded)",
         "config": {"workload": sh.name, "batch": len(sh.parents), "tree_nodes": sh.Ns, "L": sh.Ls, "q_heads": Hq,
                    "kv_heads": Hkv, "head_dim": d, "d_model": D, "vocab": V,
-                   "l2": "256 MB flush before every step (the batch's KV fits in L2)",
-                   "acceptance": acceptance_label(args)},
+                   "l2": "256 MB flush before every step, outside the timed interval (the batch's KV fits in L2)",
+                   "compaction": "included (every step)", "acceptance": acceptance_label(args)},
         "tree_tokens_per_s": round(value * R, 1),
         "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
                      "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
@@ -598,7 +645,7 @@ def run_gpu_bank_loop(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded), AR(1) entropy trace",
         "config": {"workload": sh.name, "bank_sizes": [len(t) for t in trees], "L_start": L, "L_end": L_end,
                    "policy": "hysteretic step ladder: up below 1.5 nats, down above 2.5 nats",
-                   "host_read_per_step": True},
+                   "host_read_per_step": True, "l2": C3_L2},
         "tree_tokens_per_s": round(toks / el, 1),
         "tau_mean_accept_len": round(float(np.mean(accepted)), 4),
         "tree_histogram": hist,
@@ -674,7 +721,8 @@ def bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs,
         "steps": done, "warmup": max(args.warmup, 3), "ms_per_step": round(el / done * 1e3, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded), AR(1) entropy trace",
-        "config": {"workload": sh.name + "-device-driven", "bank_sizes": [len(t) for t in trees], "L_start": L0,
+        "config": {"workload": sh.name + "-device-driven", "l2": C3_L2, "bank_sizes": [len(t) for t in trees],
+                   "L_start": L0,
                    "L_end": st["L"], "policy": "hysteretic step ladder on the device: up below 1.5, down above 2.5",
                    "host_read_per_step": False, "cuda_graph_steps": G},
         "tau_mean_accept_len": round((st["L"] - L0) / done, 4),
@@ -755,14 +803,14 @@ def run_gpu_sweep(args):
             n_steps = max(10, min(args.steps, 100))
             for _ in range(args.warmup):
                 tv.verify_step(bank, ids[j], kv, qn, hid[:n], W, drafts[:n], out, am[:n], t1[:n], en[:n], res, ws,
-                               tv.TB_NO_COMPACT, stream)
+                               0, stream)
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                   for _ in range(n_steps)]
             for i in range(n_steps):
                 flush.zero_()
                 ev[i][0].record(stream)
                 tv.verify_step(bank, ids[j], kv, qn, hid[:n], W, drafts[:n], out, am[:n], t1[:n], en[:n], res, ws,
-                               tv.TB_NO_COMPACT, stream)
+                               0, stream)
                 ev[i][1].record(stream)
             torch.cuda.synchronize()
             ms = statistics.median(a.elapsed_time(b) for a, b in ev)
@@ -789,7 +837,8 @@ def run_gpu_sweep(args):
         "ms_per_step": c4_64["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic (seeded); accept lengths from the independent-match draft model",
         "config": {"workload": "bank sweep: 8 trees x {7B 1 layer L=2048, 7B 32 layers L=16384}",
-                   "l2": "256 MB flush before every timed step"},
+                   "l2": "256 MB flush before every timed step, outside the timed interval",
+                   "compaction": "included (every step)"},
         "sweep": rows,
         "throughput_optimal_tree": best,
         "gpu_launches": 4 * max(10, min(args.steps, 100)) * len(rows),
@@ -833,7 +882,7 @@ def cpu_sample_step(cfg: str, attn_units: int, vocab_slices: int, seed: int = 0)
     sample = (f"{attn_units} of {units_total} (layer, kv head) attention units ({N} nodes x {group} q heads x "
               f"{L + N} keys x d {d}) and {vocab_slices} of 32 vocab slices ({slice_rows} x {D}) of the LM head "
               f"for {N} rows, plus acceptance; time extrapolated to one full step")
-    return full, sample, t_attn + t_lm
+    return full, sample, t_attn + t_lm, t_attn * attn_units + t_lm * vocab_slices + t_acc
 
 
 def cpu_model() -> str:
@@ -853,22 +902,26 @@ def cpu_model() -> str:
     return platform.processor() or platform.machine()
 
 
+def sample_units(cfg: str, budget_s: float) -> int:
+    """Attention units of a CPU sample that takes about budget_s (a probe times one unit
+    and one vocab slice), at most the whole step."""
+    _, _, probe, _ = cpu_sample_step(cfg, 1, 1)
+    sh, _, _, _ = workload(cfg)
+    return int(max(1, min(sh.n_layers * sh.n_kv_heads, budget_s / max(probe, 1e-6))))
+
+
 def cpu_baseline(cfg: str, budget_s: float = 20.0):
     """The oracle timed on this host's cores on a bounded sample of the workload (all
     cores, and one thread on a smaller sample)."""
     import oracle
 
     oracle.build()
-    _, _, probe = cpu_sample_step(cfg, 1, 1)
-    sh, _, _, _ = workload(cfg)
-    # as many attention units as about budget_s of work allows (the probe times one unit and one
-    # vocab slice), at most the whole step
-    n = int(max(1, min(sh.n_layers * sh.n_kv_heads, budget_s / max(probe, 1e-6))))
-    full, sample, _ = cpu_sample_step(cfg, n, min(n, 32), seed=1)
+    n = sample_units(cfg, budget_s)
+    full, sample, _, _ = cpu_sample_step(cfg, n, min(n, 32), seed=1)
     cores = oracle.num_threads()
     prev = oracle.set_num_threads(1)
     try:
-        full1, sample1, _ = cpu_sample_step(cfg, 1, 1, seed=2)
+        full1, sample1, _, _ = cpu_sample_step(cfg, 1, 1, seed=2)
     finally:
         oracle.set_num_threads(prev)
     return {"value": round(1.0 / full, 6), "unit": "verify-steps/s", "cores": cores, "kind": "oracle",
@@ -885,13 +938,17 @@ def run_reference(args):
         return
     oracle.build()
     sh, _, _, _ = workload(args.config)
+    # each step: a sample of as many attention units as the run's time budget allows
+    # (args.cpu_budget x 6 seconds over warm-up and timed steps), extrapolated to a full step
+    n = sample_units(args.config, args.cpu_budget * 6.0 / (args.warmup + args.steps))
     for i in range(args.warmup):
-        cpu_sample_step(args.config, 1, 1, seed=i)
-    times = []
+        cpu_sample_step(args.config, n, min(n, 32), seed=i)
+    times, measured = [], []
     sample = ""
     for i in range(args.steps):
-        full, sample, _ = cpu_sample_step(args.config, 1, 1, seed=100 + i)
+        full, sample, _, took = cpu_sample_step(args.config, n, min(n, 32), seed=100 + i)
         times.append(full)
+        measured.append(took)
     mean = statistics.mean(times)
     value = 1.0 / mean
     line = {
@@ -903,12 +960,14 @@ def run_reference(args):
         "steps": args.steps,
         "warmup": args.warmup,
         "ms_per_step": round(mean * 1e3, 3),
+        "ms_per_step_kind": "extrapolated: each step times a sample of the workload and scales it to one full step",
+        "measured_s_per_step": round(statistics.mean(measured), 3),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic (seeded)",
-        "config": {"workload": sh.name},
+        "config": workload_config(args, sh, *workload(args.config)[1:3]),
         "cpu_baseline": {"value": round(value, 6), "unit": "verify-steps/s", "cores": oracle.num_threads(),
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(value, 6), "unit": "verify-steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -220,6 +220,91 @@ struct tb_bank {
     TreeDesc *d_desc;
     std::vector<TreeDesc> h_desc;
     std::vector<int32_t> h_parent;  // canonical parents, capacity x 64
+    // A step whose attention is the longer pass forks the LM head onto `aux`
+    // so that it runs in the tail of the attention kernel (whose CTAs each hold
+    // a whole SM), then joins back before acceptance.  The mutex keeps one
+    // step's fork/join enqueue sequence contiguous when several host threads
+    // share the bank.
+    cudaStream_t aux;
+    cudaEvent_t ev_fork, ev_join;
+    std::mutex fork_mu;
+};
+
+// The order in which one verification step's kernels are enqueued.  Two
+// structures:
+//  - The attention grid is capped beside a longer LM head (a single layer
+//    against a large vocabulary; attn_ctas_beside_lm): one chain on the
+//    caller's stream, each kernel a programmatic dependent of the one before:
+//    [rotary embedding,] attention, LM head, acceptance + compaction, then the
+//    attention's (small) split-unit merge, beside the acceptance kernel
+//    (nothing in the step reads the attention output).  The LM head does not
+//    depend on the attention: it is launched as soon as every attention CTA has
+//    started and fills the SMs the attention is kept off; it completes only
+//    after the attention has, so the acceptance kernel, which waits for it,
+//    compacts the cache after the attention read it, and its launch overlaps
+//    the LM head's tail.  The capped attention grid is itself a programmatic
+//    dependent of the previous step.
+//  - Otherwise: the LM head is forked onto the bank's helper stream just before
+//    the attention launch (after the rotary embedding's, so that the attention
+//    CTAs are placed first) and runs on the SMs that attention CTAs release,
+//    the split-unit merge follows the attention on the caller's stream beside
+//    the LM head, and the streams join before acceptance.  The bank's fork and
+//    join events are shared, so the bank's mutex is held from construction to
+//    the end of the step's enqueueing.
+// Measured on GB300 against the second structure: the chain saves 1-1.5 us
+// per step at the 7B single-layer shape; with an uncapped grid it cost 4-8 us
+// (ragged batch, device-driven bank loop), the split-unit merge then lying on
+// the critical path behind the acceptance kernel.
+class StepStreams {
+  public:
+    StepStreams(const tb_bank *bank, cudaStream_t s, bool chain)
+        : bank_(const_cast<tb_bank *>(bank)), s_(s), chain_(chain), merge_{}
+    {
+        if (!chain_)
+            lk_ = std::unique_lock<std::mutex>(bank_->fork_mu);
+    }
+    bool chain() const { return chain_; }
+    // the split-unit merge is kept for finish() in the chain, enqueued right
+    // after the attention otherwise
+    AttnMerge *merge_later() { return chain_ ? &merge_ : nullptr; }
+    // an attention grid capped beside a longer LM head is itself a programmatic dependent
+    void attention_pdl(bool pdl) { merge_.pdl_launch = chain_ && pdl; }
+    // called between the rotary launch and the attention launch
+    tb_status before_attention(const char *fn)
+    {
+        if (chain_)
+            return TB_OK;
+        cudaError_t e = cudaEventRecord(bank_->ev_fork, s_);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(bank_->aux, bank_->ev_fork, 0);
+        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: fork: %s", fn, cudaGetErrorString(e));
+    }
+    cudaStream_t lm_stream() const { return chain_ ? s_ : bank_->aux; }
+    bool lm_pdl() const { return chain_; }
+    // called after the LM head, before the kernels that read its outputs
+    tb_status before_accept(const char *fn)
+    {
+        if (chain_)
+            return TB_OK;
+        cudaError_t e = cudaEventRecord(bank_->ev_join, bank_->aux);
+        if (e == cudaSuccess)
+            e = cudaStreamWaitEvent(s_, bank_->ev_join, 0);
+        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: join: %s", fn, cudaGetErrorString(e));
+    }
+    bool accept_pdl() const { return chain_; }
+    // the kept split-unit merge; after_step: behind the acceptance kernel (see k1_merge_split)
+    tb_status merge(const char *fn, bool after_step)
+    {
+        cudaError_t e = chain_ ? attn_merge_launch(merge_, s_, after_step) : cudaSuccess;
+        return e == cudaSuccess ? TB_OK : fail(TB_ECUDA, "%s: split-unit merge: %s", fn, cudaGetErrorString(e));
+    }
+
+  private:
+    tb_bank *bank_;
+    cudaStream_t s_;
+    bool chain_;
+    AttnMerge merge_;
+    std::unique_lock<std::mutex> lk_;
 };
 
 extern "C" tb_status tb_canonicalize(const int32_t *parent, int n, int32_t *order, int32_t *bfs_parent,
@@ -310,6 +395,18 @@ extern "C" tb_status tb_create(tb_bank **out, int max_topologies, int device)
     }
     b->h_desc.resize(max_topologies);
     b->h_parent.assign((size_t)max_topologies * TB_MAX_NODES, -1);
+    b->aux = nullptr;
+    b->ev_fork = b->ev_join = nullptr;
+    if ((e = cudaSetDevice(device)) == cudaSuccess &&
+        (e = cudaStreamCreateWithFlags(&b->aux, cudaStreamNonBlocking)) == cudaSuccess &&
+        (e = cudaEventCreateWithFlags(&b->ev_fork, cudaEventDisableTiming)) == cudaSuccess)
+        e = cudaEventCreateWithFlags(&b->ev_join, cudaEventDisableTiming);
+    if (prev >= 0)
+        cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        tb_destroy(b);
+        return cuda_fail(e, "tb_create: helper stream / events");
+    }
     *out = b;
     return ok();
 }
@@ -385,6 +482,12 @@ extern "C" tb_status tb_destroy(tb_bank *bank)
     cudaError_t e = cudaSetDevice(bank->device);
     if (e == cudaSuccess && bank->d_desc)
         e = cudaFree(bank->d_desc);
+    if (bank->ev_fork)
+        cudaEventDestroy(bank->ev_fork);
+    if (bank->ev_join)
+        cudaEventDestroy(bank->ev_join);
+    if (bank->aux)
+        cudaStreamDestroy(bank->aux);
     if (prev >= 0)
         cudaSetDevice(prev);
     delete bank;
@@ -599,11 +702,11 @@ static RopeSeq rope_seq(const tb_kv *kv, const TreeDesc *tree)
                    tree, kv->L};
 }
 
-// The rotary embedding (if any), then the attention.  merge_later: the
-// tcgen05 attention's split-unit merge is kept there, to be enqueued later in
-// the verification step.
+// The rotary embedding (if any), then the attention; ss: the verification
+// step's structure (the fork comes after the rotary launch; the split-unit
+// merge may be kept for later).
 static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, cudaStream_t stream, const char *fn,
-                              AttnMerge *merge_later = nullptr)
+                              StepStreams *ss = nullptr)
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
@@ -616,6 +719,12 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
         if (st != TB_OK)
             return st;
     }
+    if (ss) {
+        tb_status st = ss->before_attention(fn);
+        if (st != TB_OK)
+            return st;
+    }
+    AttnMerge *merge_later = ss ? ss->merge_later() : nullptr;
     const int nsm = sm_count(a.bank->device);
     cudaError_t e;
     if (use_tc_attention(a.kv->head_dim, rows))
@@ -939,13 +1048,15 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
     lt.ent_t = tr.ent_t;
     lt.logits_out = logits;
     a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
-    // the chain of verify_step, with the walk between the LM head and the compaction
-    AttnMerge merge{};
-    merge.pdl_launch = a.max_ctas > 0 && kv->rope_theta == 0.f;
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &merge)) != TB_OK)
+    // the structure of verify_step, with the walk between the LM head and the compaction
+    StepStreams ss(bank, s, a.max_ctas > 0);
+    ss.attention_pdl(kv->rope_theta == 0.f);
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &ss)) != TB_OK)
         return st;
-    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s, fn,
-                         0, &lt, true)) != TB_OK)
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                         ss.lm_stream(), fn, 0, &lt, ss.lm_pdl())) != TB_OK)
+        return st;
+    if ((st = ss.before_accept(fn)) != TB_OK)
         return st;
     if ((st = sample_enqueue(bank, bank_id, draft_tokens, logits, tr.logz_t, draft_probs, uniforms, vocab, kv->L,
                              temperature, logits + (size_t)N * vocab, result, reinterpret_cast<const int *>(ws), s,
@@ -956,13 +1067,12 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
         p.result = result;
         p.from_result = 1;
         add_compaction(p, kv);
-        cudaError_t e = accept_launch(p, sm_count(bank->device), s, true);
+        cudaError_t e = accept_launch(p, sm_count(bank->device), s, ss.accept_pdl());
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
     }
-    cudaError_t e = attn_merge_launch(merge, s, true);
-    if (e != cudaSuccess)
-        return cuda_fail(e, fn);
+    if ((st = ss.merge(fn, true)) != TB_OK)
+        return st;
     return ok();
 }
 
@@ -1018,24 +1128,17 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         lt.gather.n_seq = 1;
         lt.gather.seq[0] = LmGatherSeq{bank->d_desc + bank_id, draft_tokens, tr.draft_logit, 0, N};
     }
-    // One chain on the caller's stream: [rotary embedding,] attention (launched
-    // once the stream's previous work is done, so that all its CTAs start
-    // together), LM head, acceptance + compaction, split-unit merge; the last
-    // three are programmatic dependents of the kernel before them.  The LM head
-    // does not depend on the attention: it is launched once every attention CTA
-    // has started and fills the SMs that attention CTAs release (or, when it is
-    // the longer of the two, the SMs the attention is kept off); it completes
-    // only after the attention has, so the acceptance kernel, which waits for
-    // it, compacts the cache after the attention read it.  Nothing in the step
-    // reads the attention output, so its split units are merged beside the
-    // acceptance kernel.
+    // the step's structure: see StepStreams
     a.max_ctas = attn_ctas_beside_lm(aplan, lplan, d_model, vocab, sm_count(bank->device));
-    AttnMerge merge{};
-    merge.pdl_launch = a.max_ctas > 0 && kv->rope_theta == 0.f;
-    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &merge)) != TB_OK)
+    StepStreams ss(bank, s, a.max_ctas > 0);
+    ss.attention_pdl(kv->rope_theta == 0.f);
+    if ((st = attn_enqueue(a, ws, kPartBase, s, fn, &ss)) != TB_OK)
         return st;
-    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes, s, fn,
-                         (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr, true)) != TB_OK)
+    if ((st = lm_enqueue(hidden, N, lm_head, d_model, vocab, argmax, top1, entropy, ws, kPartBase + attn_bytes,
+                         ss.lm_stream(), fn, (flags & TB_DEBUG_EXPIRE_WAIT) ? 1 : 0, typ ? &lt : nullptr,
+                         ss.lm_pdl())) != TB_OK)
+        return st;
+    if ((st = ss.before_accept(fn)) != TB_OK)
         return st;
     AcceptParams p =
         accept_params(bank, bank_id, draft_tokens, argmax, vocab, kv->L, result, reinterpret_cast<const int *>(ws));
@@ -1043,11 +1146,11 @@ static tb_status verify_step_impl(const tb_bank *bank, int bank_id, const tb_kv 
         add_typical(p, typ, tr.logz_t, tr.ent_t, tr.draft_logit);
     if (!(flags & TB_NO_COMPACT))
         add_compaction(p, kv);
-    cudaError_t e = accept_launch(p, sm_count(bank->device), s, true);
-    if (e == cudaSuccess)
-        e = attn_merge_launch(merge, s, true);
+    cudaError_t e = accept_launch(p, sm_count(bank->device), s, ss.accept_pdl());
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
+    if ((st = ss.merge(fn, true)) != TB_OK)
+        return st;
     return ok();
 }
 
@@ -1137,10 +1240,9 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     cudaStream_t s = (cudaStream_t)stream;
 
-    // the chain of verify_step: [rotary embedding,] attention, LM head,
-    // acceptance + compaction, split-unit merge
+    // the step's structure: see StepStreams
     cudaError_t e = cudaSuccess;
-    AttnMerge merge{};
+    StepStreams ss(bank, s, false);  // the batch's attention takes every SM
     // tree attention of every sequence (after the rotary embedding of their tree keys)
     if (tc) {
         const bool rope = kv0.rope_theta != 0.f;
@@ -1154,13 +1256,15 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             if ((st = rope_enqueue(rp, &kv0, batch, 0, kv0.n_layers, max_nodes, ws, s, fn)) != TB_OK)
                 return st;
         }
+        if ((st = ss.before_attention(fn)) != TB_OK)
+            return st;
         AttnSeq as[TB_MAX_BATCH];
         for (int b = 0; b < batch; ++b)
             as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
         const char *err = "";
         e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err, rope ? rope_table(ws) : nullptr, &merge);
+                                 &err, rope ? rope_table(ws) : nullptr, ss.merge_later());
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
@@ -1171,7 +1275,8 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             AttnPlan plan;
             if ((st = attn_validate(a, fn, &plan)) != TB_OK)
                 return st;
-            if ((st = attn_enqueue(a, ws, kPartBase, s, fn)) != TB_OK)
+            // the fork before the first launch
+            if ((st = attn_enqueue(a, ws, kPartBase, s, fn, b == 0 ? &ss : nullptr)) != TB_OK)
                 return st;
         }
     }
@@ -1198,10 +1303,12 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
         }
         // the chunks share the partials and counters: only the first overlaps the attention
         if ((st = lm_enqueue(h8 + (size_t)r0 * d_model * 2, rc, lm_head, d_model, vocab, argmax + r0, top1 + r0,
-                             entropy + r0, ws, kPartBase + attn_bytes, s, fn, 0, typ ? &lt : nullptr, r0 == 0)) !=
-            TB_OK)
+                             entropy + r0, ws, kPartBase + attn_bytes, ss.lm_stream(), fn, 0, typ ? &lt : nullptr,
+                             ss.lm_pdl() && r0 == 0)) != TB_OK)
             return st;
     }
+    if ((st = ss.before_accept(fn)) != TB_OK)
+        return st;
     // acceptance + compaction, one launch
     AcceptParams ps[TB_MAX_BATCH];
     int r0 = 0;
@@ -1214,11 +1321,11 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
             add_compaction(ps[b], &seqs[b].kv);
         r0 += Ns[b];
     }
-    e = accept_launch_batch(ps, batch, nsm, s, true);
-    if (e == cudaSuccess)
-        e = attn_merge_launch(merge, s, true);
+    e = accept_launch_batch(ps, batch, nsm, s, ss.accept_pdl());
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
+    if ((st = ss.merge(fn, true)) != TB_OK)
+        return st;
     return ok();
 }
 
@@ -1341,9 +1448,7 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     sc.out = attn_out;
     for (int r = 0; r < policy->n_rungs; ++r)
         sc.rung_tree[r] = bank->d_desc + policy->bank_ids[r];
-    // the chain of verify_step, with the split-unit merge before the acceptance
-    // kernel, which moves the device state on to the next step
-    AttnMerge merge{};
+    StepStreams ss(bank, s, false);  // the scheduled attention takes every SM
     {
         if (kv->rope_theta != 0.f) {
             RopeParams rp{};
@@ -1357,19 +1462,23 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
                 return st;
             sc.rope_tab = rope_table(ws);
         }
+        if ((st = ss.before_attention(fn)) != TB_OK)
+            return st;
         const char *err = "";
         cudaError_t e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
                                  reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err, &merge);
+                                 &err, ss.merge_later());
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
         if ((st = lm_enqueue(hidden, N_max, lm_head, d_model, vocab, argmax, top1, entropy, ws,
-                             kPartBase + attn_bytes, s, fn, 0, nullptr, true)) != TB_OK)
+                             kPartBase + attn_bytes, ss.lm_stream(), fn, 0, nullptr, ss.lm_pdl())) != TB_OK)
             return st;
-        if ((e = attn_merge_launch(merge, s, false)) != cudaSuccess)
-            return cuda_fail(e, fn);
+        if ((st = ss.merge(fn, false)) != TB_OK)
+            return st;
+        if ((st = ss.before_accept(fn)) != TB_OK)
+            return st;
     }
     AcceptParams p = accept_params(bank, policy->bank_ids[0], draft_tokens, argmax, vocab, 0, result,
                                    reinterpret_cast<const int *>(ws));
@@ -1393,7 +1502,7 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     p.trace = policy->trace;
     p.top1 = top1;
     p.entropy = entropy;
-    cudaError_t e = accept_launch(p, nsm, s, true);
+    cudaError_t e = accept_launch(p, nsm, s, ss.accept_pdl());
     if (e != cudaSuccess)
         return cuda_fail(e, fn);
     return ok();
