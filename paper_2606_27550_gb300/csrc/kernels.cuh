@@ -5,37 +5,59 @@
 
 namespace tv {
 
-// Launches `kernel` on `stream`; with pdl, with the programmatic-serialization
-// attribute, so that it may be launched while the previous kernel of the
-// stream still runs (the kernel waits for it with pdl_wait before touching
-// memory it writes).
+// Launches `kernel` on `stream` in clusters of `cluster_x` CTAs (1: none);
+// with pdl, with the programmatic-serialization attribute, so that it may be
+// launched while the previous kernel of the stream still runs (the kernel
+// waits for it with pdl_wait before touching memory it writes).
 template <typename... KArgs, typename... Args>
-cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
-                          Args &&...args)
+cudaError_t launch_kernel_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                                  bool pdl, int cluster_x, Args &&...args)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = pdl ? attr : nullptr;
-    cfg.numAttrs = pdl ? 1 : 0;
+    cudaLaunchAttribute attr[2];
+    int n = 0;
+    if (pdl) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (cluster_x > 1) {
+        attr[n].id = cudaLaunchAttributeClusterDimension;
+        attr[n].val.clusterDim.x = (unsigned)cluster_x;
+        attr[n].val.clusterDim.y = 1;
+        attr[n].val.clusterDim.z = 1;
+        ++n;
+    }
+    cfg.attrs = n ? attr : nullptr;
+    cfg.numAttrs = n;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                          Args &&...args)
+{
+    return launch_kernel_cluster(kernel, grid, block, smem, stream, pdl, 1, static_cast<Args &&>(args)...);
 }
 
 // LM head (lm_head.cu)
 struct LmPlan {
     int R_pad, n_tiles, n_kblocks, stages, acc_cols, group_size, n_groups;
     int ctas_per_sm;  // 2 when two rings fit side by side, else 1
-    int P;            // persistent CTAs: ctas_per_sm per SM, at most one per vocab tile
+    bool pair;        // CTA pairs share each MMA (M = 256); tiles are then 256 vocab entries
+    int units;        // the tile split's units: CTAs, or CTA pairs
+    int P;            // persistent CTAs: ctas_per_sm per SM, at most one per vocab tile (two per pair tile)
     int n_counters;   // workspace counters used (group tickets)
     size_t smem_bytes;
     size_t ws_bytes;  // partials (CTA + group), 256-byte aligned
 };
-LmPlan lm_plan(int R, int D, int V, int n_sm);
+// n_sm: the SMs the launch may use; max_pairs: the clusters of two that can
+// be resident at once (-1: n_sm / 2), which bounds the pairs of a pair plan.
+LmPlan lm_plan(int R, int D, int V, int n_sm, int max_pairs = -1);
 // typical-acceptance inputs produced by the same pass: per-row statistics at
 // temperature T and the draft-token logit of every tree edge j, written to
 // seq[b].out[j] for edges whose parent row row_base + parent[j] is in [0, R)

@@ -23,6 +23,7 @@
 // merges the group; the last group merges everything); no CTA ever waits for
 // another.
 //
+#include <atomic>
 #include <math.h>
 #include <stdlib.h>
 
@@ -32,10 +33,11 @@ namespace tv {
 
 struct LmParams {
     CUtensorMap tmap_w;  // (d_model, vocab), box (64, 128), 128B swizzle
-    CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad), 128B swizzle
+    CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad) (R_pad / 2 for CTA pairs), 128B swizzle
     int R, R_pad, D, V;
-    int n_tiles, nk, stages, acc_cols;
+    int n_tiles, nk, stages, acc_cols;  // tiles of 128 vocab entries (256 for CTA pairs)
     int P;               // CTAs
+    int units;           // the tile split's units: CTAs, or CTA pairs
     int group_size, n_groups;
     size_t smem_avail;   // dynamic shared memory after alignment (the merges stage partials there)
     float4 *part_cta;    // [P][R_pad]  (max, argmax bits, s, t)
@@ -289,10 +291,10 @@ __device__ __forceinline__ void epi_sync()
     asm volatile("bar.sync 1, 256;" ::: "memory");
 }
 
-// First vocab tile of CTA c's run.
+// First vocab tile of unit c's run.
 __device__ __forceinline__ int lm_tile_begin(const LmParams &p, int c)
 {
-    return (int)((long long)c * p.n_tiles / p.P);
+    return (int)((long long)c * p.n_tiles / p.units);
 }
 
 // k-block j of a tile's loop: the order is rotated by the tile index, so the
@@ -313,7 +315,14 @@ struct PdlWaitOnExit {
     __device__ ~PdlWaitOnExit() { pdl_wait(); }
 };
 
-template <bool kTyp>
+// kPair: CTA pairs (clusters of two) share each MMA (tcgen05 cta_group::2, M =
+// 256): a pair tile is 256 vocab entries, 128 per CTA, and each CTA stages only
+// half of the tree rows, so a stage moves 16 KB of W plus half the rows' box
+// through each SM's shared memory instead of the whole box.  The even CTA
+// issues the MMAs; both CTAs' TMA loads complete on its stage barriers, its
+// commits arrive on both CTAs' barriers, and both CTAs' epilogues release its
+// accumulators.  Used for wide rows, where a CTA holds an SM alone.
+template <bool kTyp, bool kPair>
 __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constant__ LmParams p)
 {
     // the acceptance kernel that reads this kernel's outputs may be launched now
@@ -326,6 +335,8 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
     __shared__ __align__(8) uint64_t drain_bar, never_bar;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
+    // CTA pairs: the stage sequences each producer thread issued, this CTA's and the odd CTA's
+    __shared__ long long s_gend[2], s_peer_gend[2];
     __shared__ int s_ticket, s_ok;
     // typical mode: edges whose draft token lies in the current tile, packed as
     // (seq << 24) | (node << 16) | (row << 7) | col; overflow -> rescan per chunk
@@ -335,7 +346,8 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
 
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = p.stages;
-    const uint32_t hb = (uint32_t)p.R_pad * 128u;  // one 64-column box of the tree rows
+    // one 64-column box of this CTA's tree rows (half of them in a pair)
+    const uint32_t hb = (uint32_t)(kPair ? p.R_pad / 2 : p.R_pad) * 128u;
     const uint32_t stage_bytes = 16384u + hb;
     uint8_t *ring = smem;
     float *chunk = reinterpret_cast<float *>(smem + (size_t)S * stage_bytes);  // [kLmChunk][kChunkLd]
@@ -343,7 +355,11 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
-    const int tile0 = lm_tile_begin(p, c), tile1 = lm_tile_begin(p, c + 1);
+    // the unit of the tile split: a CTA, or a pair; tiles are 128 (256 for a pair) vocab entries
+    const uint32_t rank = kPair ? cluster_ctarank() : 0u;
+    const bool leader = rank == 0;
+    const int unit = kPair ? c >> 1 : c;
+    const int tile0 = lm_tile_begin(p, unit), tile1 = lm_tile_begin(p, unit + 1);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -352,23 +368,31 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&acc_full[b], 1);
-            mbar_init(&acc_empty[b], kEpiThreads / 32);
+            mbar_init(&acc_empty[b], (kEpiThreads / 32) * (kPair ? 2 : 1));  // a pair's epilogues release the even CTA's
         }
         mbar_init(&drain_bar, 1);
         mbar_init(&never_bar, 1);
         abort_flag = 0;
+        s_gend[0] = s_gend[1] = s_peer_gend[0] = s_peer_gend[1] = 0;
         fence_mbar_init();
         prefetch_tmap(&p.tmap_w);
         prefetch_tmap(&p.tmap_h);
     }
     if (warp == 1) {
-        tmem_alloc(&tmem_slot, 2u * (uint32_t)p.acc_cols);
-        tmem_relinquish();
+        if constexpr (kPair) {
+            tmem_alloc_pair(&tmem_slot, 2u * (uint32_t)p.acc_cols);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(&tmem_slot, 2u * (uint32_t)p.acc_cols);
+            tmem_relinquish();
+        }
     }
     for (int r = threadIdx.x; r < p.R_pad; r += blockDim.x)
         run[r] = stat_empty();
     tc_fence_before();
     __syncthreads();
+    if constexpr (kPair)
+        cluster_barrier();  // both CTAs' barriers are initialised before either CTA signals the other's
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
@@ -391,21 +415,36 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
-                    tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
-                    tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                    if constexpr (kPair) {
+                        // the stage's four boxes (W and tree rows of both CTAs) complete on the even CTA's barrier
+                        if (leader)
+                            mbar_arrive_expect_tx(&full_bar[s], 2 * stage_bytes);
+                        const uint32_t fb = cluster_addr(&full_bar[s], 0);
+                        tma_load_2d_pair(ring + (size_t)s * stage_bytes, &p.tmap_w, fb, kb * 64,
+                                         tile * 256 + (int)rank * 128);
+                        tma_load_2d_pair(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, fb, kb * 64,
+                                         (int)rank * (p.R_pad / 2));
+                    } else {
+                        mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+                        tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
+                        tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                    }
                     g_end = g + 1;
                 }
             }
-            if (!ok)  // gave up: this thread's copies in flight land before the CTA exits
+            s_gend[mine] = g_end;
+            // Gave up: this thread's copies in flight land before the CTA exits.  (In a
+            // pair, the even CTA drains both CTAs' copies at the teardown.)
+            if (!ok && !kPair)
                 for (long long it = (g_end > S ? g_end - S : 0); it < g_end; ++it)
                     if ((it & 1) == mine)
                         mbar_wait_drain(&full_bar[it % S], (uint32_t)(it / S) & 1u);
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer: the CTA's i-th tile accumulates into TMEM buffer i & 1
-        if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, p.R_pad);
+        // (in a pair, the even CTA issues for both)
+        if (lane == 0 && leader) {
+            const uint32_t idesc = idesc_bf16_f32(kPair ? 256 : 128, p.R_pad);
             long long g = 0;
             bool ok = true;
             for (int tile = tile0, i = 0; tile < tile1 && ok; ++tile, ++i) {
@@ -427,16 +466,28 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                     for (int k = 0; k < 4; ++k) {
                         const uint64_t ad = smem_desc_sw128(a_base + k * 32, 0, 1024);
                         const uint64_t bd = smem_desc_sw128(b_base + k * 32, 0, 1024);
-                        tc_mma_f16_ss(d, ad, bd, idesc, (j != 0 || k != 0) ? 1u : 0u);
+                        if constexpr (kPair)
+                            tc_mma_f16_ss_pair(d, ad, bd, idesc, (j != 0 || k != 0) ? 1u : 0u);
+                        else
+                            tc_mma_f16_ss(d, ad, bd, idesc, (j != 0 || k != 0) ? 1u : 0u);
                     }
-                    tc_commit(&empty_bar[s]);
+                    if constexpr (kPair)
+                        tc_commit_pair(&empty_bar[s]);
+                    else
+                        tc_commit(&empty_bar[s]);
                 }
                 if (!ok)
                     break;
-                tc_commit(&acc_full[b]);
+                if constexpr (kPair)
+                    tc_commit_pair(&acc_full[b]);
+                else
+                    tc_commit(&acc_full[b]);
             }
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
-            tc_commit(&drain_bar);
+            if constexpr (kPair)
+                tc_commit_pair(&drain_bar);
+            else
+                tc_commit(&drain_bar);
         }
     } else if (warp < kLmProducer2) {
         // ---------------- epilogue (warps 2-9)
@@ -459,7 +510,8 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             if (!agree())
                 break;
             tc_fence_after();
-            const int v0 = tile * 128, nvalid = min(128, p.V - v0);
+            // this CTA's 128 vocab entries (the odd CTA of a pair's last tile may have none)
+            const int v0 = kPair ? tile * 256 + (int)rank * 128 : tile * 128, nvalid = min(128, p.V - v0);
             if constexpr (kTyp) {
                 // the tree edges whose draft token lies in this tile
                 if (e == 0)
@@ -488,8 +540,12 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                     // last read of this accumulator: the MMAs of segment i + 2 may reuse it
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0)
-                        mbar_arrive(&acc_empty[b]);
+                    if (lane == 0) {
+                        if constexpr (kPair)
+                            mbar_arrive_cluster(cluster_addr(&acc_empty[b], 0));
+                        else
+                            mbar_arrive(&acc_empty[b]);
+                    }
                 }
                 if (col < p.R_pad) {
 #pragma unroll
@@ -573,7 +629,35 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         if (lane == 0)
             mbar_wait_drain(&drain_bar, 0);
         __syncwarp();
-        tmem_dealloc(tmem, 2u * (uint32_t)p.acc_cols);
+        if constexpr (!kPair)
+            tmem_dealloc(tmem, 2u * (uint32_t)p.acc_cols);
+    }
+    if constexpr (kPair) {
+        // Both CTAs' epilogues are done with TMEM and both have seen the MMAs retire
+        // before the pair frees it.  Every copy either CTA issued lands before either
+        // exits: normally the MMAs consumed them all; after a give-up, the even CTA
+        // arms the stages only the odd CTA filled (at most a ring's worth ahead) and
+        // drains the last ring's worth of stages of each producer thread, waiting
+        // with the usual bound.
+        if (!leader && threadIdx.x < 2)
+            st_cluster_s64(cluster_addr(&s_peer_gend[threadIdx.x], 0), s_gend[threadIdx.x]);
+        cluster_barrier();
+        if (warp == 1) {
+            tc_fence_after();
+            tmem_dealloc_pair(tmem, 2u * (uint32_t)p.acc_cols);
+        }
+        if (leader && threadIdx.x < 2) {
+            const long long mine = threadIdx.x, gl = s_gend[mine], go = s_peer_gend[mine];
+            for (long long it = gl; it < go; ++it)
+                if ((it & 1) == mine)
+                    mbar_arrive_expect_tx(&full_bar[it % S], stage_bytes);
+            const long long ge = gl > go ? gl : go;
+            if (abort_flag || gl != go)
+                for (long long it = (ge > S ? ge - S : 0); it < ge; ++it)
+                    if ((it & 1) == mine)
+                        mbar_wait_drain(&full_bar[it % S], (uint32_t)(it / S) & 1u);
+        }
+        cluster_barrier();
     }
     if (abort_flag)
         return;
@@ -604,33 +688,48 @@ static int ceil_div(int a, int b)
     return (a + b - 1) / b;
 }
 
-LmPlan lm_plan(int R, int D, int V, int n_sm)
+LmPlan lm_plan(int R, int D, int V, int n_sm, int max_pairs)
 {
     LmPlan pl{};
+    if (n_sm < 1)
+        n_sm = 1;
     pl.R_pad = ceil_div(R, 16) * 16;
-    pl.n_tiles = ceil_div(V, 128);
     pl.n_kblocks = ceil_div(D, 64);
     int cols = 32;
     while (cols < pl.R_pad)
         cols *= 2;
     pl.acc_cols = cols;
-    const size_t stage_bytes = 16384 + (size_t)pl.R_pad * 128;
     const size_t fixed = (size_t)kLmChunk * kChunkLd * 4 + (size_t)pl.R_pad * sizeof(RowStat);
     // Two CTAs share an SM when each still gets a ring of at least three stages
     // in half of its shared memory and four accumulators fit in TMEM: two
     // independent TMA pipelines per SM stream W faster than one deeper ring.
     const size_t pad = 1024 + 1024;  // alignment pad, static shared memory
     const size_t half = 112 * 1024;
-    const int st2 = half > fixed + pad ? (int)((half - fixed - pad) / stage_bytes) : 0;
+    const size_t stage1 = 16384 + (size_t)pl.R_pad * 128;
+    const int st2 = half > fixed + pad ? (int)((half - fixed - pad) / stage1) : 0;
     pl.ctas_per_sm = (st2 >= 3 && 4 * cols <= 512) ? 2 : 1;
+    // Otherwise (wide rows, one CTA per SM) CTA pairs share each MMA: each CTA
+    // stages half of the rows, so the rows cross each SM's shared memory once
+    // per 256 vocab entries instead of once per 128.
+    if (max_pairs < 0)
+        max_pairs = n_sm / 2;
+    pl.pair = pl.ctas_per_sm == 1 && max_pairs >= 1;
+    pl.n_tiles = ceil_div(V, pl.pair ? 256 : 128);
+    const size_t stage_bytes = 16384 + (size_t)(pl.pair ? pl.R_pad / 2 : pl.R_pad) * 128;
     const size_t budget = (pl.ctas_per_sm == 2 ? half : 227 * 1024) - fixed - pad;
     pl.stages = (int)(budget / stage_bytes);
     if (pl.stages > 8)
         pl.stages = 8;
     if (pl.stages < 2)
         pl.stages = 2;
-    const int slots = pl.ctas_per_sm * (n_sm > 0 ? n_sm : 1);
-    pl.P = slots < pl.n_tiles ? slots : pl.n_tiles;
+    if (pl.pair) {
+        pl.units = max_pairs < pl.n_tiles ? max_pairs : pl.n_tiles;
+        pl.P = 2 * pl.units;
+    } else {
+        const int slots = pl.ctas_per_sm * n_sm;
+        pl.P = slots < pl.n_tiles ? slots : pl.n_tiles;
+        pl.units = pl.P;
+    }
     int gs = 1;
     while (gs * gs < pl.P)
         ++gs;
@@ -641,21 +740,86 @@ LmPlan lm_plan(int R, int D, int V, int n_sm)
     if (mg > sm)
         sm = mg;
     pl.smem_bytes = sm + 1024;
-    pl.n_counters = pl.n_groups + 1;
-    // (max, argmax, s, t) and (sT, tT) partials of the CTAs and the groups
-    pl.ws_bytes = ((size_t)(pl.P + pl.n_groups) * pl.R_pad * (16 + 8) + 255) / 256 * 256;
+    // (max, argmax, s, t) and (sT, tT) partials of the CTAs and the groups.  The
+    // workspace also covers the plan without pairs, which a launch takes when
+    // no cluster of two can be resident.
+    const int slots = pl.ctas_per_sm * n_sm, n128 = ceil_div(V, 128);
+    const int p1 = slots < n128 ? slots : n128;
+    int gs1 = 1;
+    while (gs1 * gs1 < p1)
+        ++gs1;
+    const int ng1 = ceil_div(p1, gs1);
+    const int parts = pl.P + pl.n_groups > p1 + ng1 ? pl.P + pl.n_groups : p1 + ng1;
+    pl.n_counters = (pl.n_groups > ng1 ? pl.n_groups : ng1) + 1;
+    pl.ws_bytes = ((size_t)parts * pl.R_pad * (16 + 8) + 255) / 256 * 256;
     return pl;
+}
+
+// Clusters of two CTAs of k2_lm_head<kTyp, true> with `smem` bytes each that
+// can be resident at once (cached per shared-memory size; 0 if none).
+template <bool kTyp>
+static int lm_max_pairs(size_t smem, int n_sm)
+{
+    static std::atomic<int> cache[24];  // by smem / 16 KB; 0: not queried yet, else pairs + 1
+    const size_t slot = smem / 16384 < 24 ? smem / 16384 : 23;
+    int v = cache[slot].load(std::memory_order_relaxed);
+    if (v > 0)
+        return v - 1;
+    int pairs = 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (n_sm / 2 > 0 ? n_sm / 2 : 1));
+    cfg.blockDim = dim3(kLmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (allow_max_smem((const void *)k2_lm_head<kTyp, true>) != cudaSuccess ||
+        cudaOccupancyMaxActiveClusters(&pairs, k2_lm_head<kTyp, true>, &cfg) != cudaSuccess) {
+        (void)cudaGetLastError();
+        pairs = 0;
+    }
+    if (pairs > n_sm / 2)
+        pairs = n_sm / 2;
+    cache[slot].store(pairs + 1, std::memory_order_relaxed);
+    return pairs;
+}
+
+template <bool kTyp>
+static cudaError_t lm_launch_as(LmParams &p, const LmPlan &pl, cudaStream_t stream, bool pdl)
+{
+    if (pl.pair) {
+        cudaError_t e = allow_max_smem((const void *)k2_lm_head<kTyp, true>);
+        if (e != cudaSuccess)
+            return e;
+        return launch_kernel_cluster(k2_lm_head<kTyp, true>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl,
+                                     2, p);
+    }
+    cudaError_t e = allow_max_smem((const void *)k2_lm_head<kTyp, false>);
+    if (e != cudaSuccess)
+        return e;
+    return launch_kernel(k2_lm_head<kTyp, false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
 }
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
                            float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
                            const char **err, int expire_wait, const LmTypical *typ, bool pdl)
 {
-    const LmPlan pl = lm_plan(R, D, V, n_sm);
+    LmPlan pl = lm_plan(R, D, V, n_sm);
+    if (pl.pair) {
+        // as many pairs as can be resident at once (the SMs of a cluster share a GPC)
+        const int mp = typ ? lm_max_pairs<true>(pl.smem_bytes, n_sm) : lm_max_pairs<false>(pl.smem_bytes, n_sm);
+        if (mp != pl.units || mp < 1)
+            pl = lm_plan(R, D, V, n_sm, mp);
+    }
     LmParams p{};
     if (!make_tmap_2d(&p.tmap_w, W, (uint64_t)D, (uint64_t)V, (uint64_t)D * 2, 64, 128, err))
         return cudaErrorInvalidValue;
-    if (!make_tmap_2d(&p.tmap_h, hidden, (uint64_t)D, (uint64_t)R, (uint64_t)D * 2, 64, (uint32_t)pl.R_pad, err))
+    if (!make_tmap_2d(&p.tmap_h, hidden, (uint64_t)D, (uint64_t)R, (uint64_t)D * 2, 64,
+                      (uint32_t)(pl.pair ? pl.R_pad / 2 : pl.R_pad), err))
         return cudaErrorInvalidValue;
     p.R = R;
     p.R_pad = pl.R_pad;
@@ -666,6 +830,7 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.stages = pl.stages;
     p.acc_cols = pl.acc_cols;
     p.P = pl.P;
+    p.units = pl.units;
     p.group_size = pl.group_size;
     p.n_groups = pl.n_groups;
     p.smem_avail = pl.smem_bytes - 1024;
@@ -685,16 +850,10 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
         p.ent_t = typ->ent_t;
         p.gather = typ->gather;
         p.logits_out = typ->logits_out;
-        cudaError_t e = allow_max_smem((const void *)k2_lm_head<true>);
-        if (e != cudaSuccess)
-            return e;
-        return launch_kernel(k2_lm_head<true>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
+        return lm_launch_as<true>(p, pl, stream, pdl);
     }
     p.inv_t = 1.0f;
-    cudaError_t e = allow_max_smem((const void *)k2_lm_head<false>);
-    if (e != cudaSuccess)
-        return e;
-    return launch_kernel(k2_lm_head<false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
+    return lm_launch_as<false>(p, pl, stream, pdl);
 }
 
 TB_BOUNDS_COUNTER(bounds_violations_lm_head)
