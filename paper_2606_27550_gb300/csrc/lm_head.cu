@@ -297,14 +297,48 @@ __device__ __forceinline__ int lm_tile_begin(const LmParams &p, int c)
     return (int)((long long)c * p.n_tiles / p.units);
 }
 
-// k-block j of a tile's loop: the order is rotated by the tile index, so the
-// CTAs in flight read their W rows at spread-out column offsets rather than
-// all at the same one.
-__device__ __forceinline__ int lm_kb(const LmParams &p, int tile, int j)
+// Step j of a tile's k-loop reads k-block j + lm_rot (mod nk): the order is
+// rotated by the tile index, so the CTAs in flight read their W rows at
+// spread-out column offsets rather than all at the same one.
+__device__ __forceinline__ int lm_rot(const LmParams &p, int tile)
 {
-    const int x = j + (int)(((long long)tile * 5) % p.nk);
-    return x >= p.nk ? x - p.nk : x;
+    return (int)(((long long)tile * 5) % p.nk);
 }
+
+// A producer thread's position in the ring: the k-block sequence g = g0,
+// g0 + 2, ... of a run, as (tile, k-block) and (ring slot, phase parity),
+// advanced without divisions.
+struct RingCursor {
+    int tile, j, kb, rot, slot;
+    uint32_t phase;
+    __device__ RingCursor(const LmParams &p, int tile0, int g0) : tile(tile0), j(g0), slot(g0), phase(0)
+    {
+        // g0 is 0 or 1; the ring has at least two slots
+        while (j >= p.nk) {
+            j -= p.nk;
+            ++tile;
+        }
+        rot = lm_rot(p, tile);
+        kb = j + rot >= p.nk ? j + rot - p.nk : j + rot;
+    }
+    __device__ __forceinline__ void advance2(const LmParams &p, int S)
+    {
+        slot += 2;
+        if (slot >= S) {
+            slot -= S;
+            phase ^= 1u;
+        }
+        j += 2;
+        if (j >= p.nk) {
+            while (j >= p.nk) {
+                j -= p.nk;
+                ++tile;
+            }
+            rot = lm_rot(p, tile);
+        }
+        kb = j + rot >= p.nk ? j + rot - p.nk : j + rot;
+    }
+};
 
 // Waits, when it goes out of scope (every exit of the kernel), for the
 // stream's previous kernel to complete.  In a verification step the LM head
@@ -402,35 +436,32 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         // Warp 0 fills the even stages of the sequence, the last warp the odd
         // ones: one issuing thread alone streams W measurably slower.
         if (lane == 0) {
-            const long long mine = warp == 0 ? 0 : 1;
-            long long g = 0, g_end = 0;
+            const int mine = warp == 0 ? 0 : 1;
+            const long long G = (long long)(tile1 - tile0) * p.nk;  // the run's k-blocks
+            RingCursor cur(p, tile0, mine);  // this thread's steps g = mine, mine + 2, ...
+            long long g_end = 0;
             bool ok = true;
-            for (int tile = tile0; tile < tile1 && ok; ++tile) {
-                for (int j = 0; j < p.nk; ++j, ++g) {
-                    if ((g & 1) != mine)
-                        continue;
-                    const int kb = lm_kb(p, tile, j);
-                    const int s = (int)(g % S);
-                    if (!mbar_wait_bounded(&empty_bar[s], ((uint32_t)(g / S) & 1u) ^ 1u, &abort_flag, p.status)) {
-                        ok = false;
-                        break;
-                    }
-                    if constexpr (kPair) {
-                        // the stage's four boxes (W and tree rows of both CTAs) complete on the even CTA's barrier
-                        if (leader)
-                            mbar_arrive_expect_tx(&full_bar[s], 2 * stage_bytes);
-                        const uint32_t fb = cluster_addr(&full_bar[s], 0);
-                        tma_load_2d_pair(ring + (size_t)s * stage_bytes, &p.tmap_w, fb, kb * 64,
-                                         tile * 256 + (int)rank * 128);
-                        tma_load_2d_pair(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, fb, kb * 64,
-                                         (int)rank * (p.R_pad / 2));
-                    } else {
-                        mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
-                        tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
-                        tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
-                    }
-                    g_end = g + 1;
+            for (long long g = mine; g < G; g += 2, cur.advance2(p, S)) {
+                const int s = cur.slot, tile = cur.tile, kb = cur.kb;
+                if (!mbar_wait_bounded(&empty_bar[s], cur.phase ^ 1u, &abort_flag, p.status)) {
+                    ok = false;
+                    break;
                 }
+                if constexpr (kPair) {
+                    // the stage's four boxes (W and tree rows of both CTAs) complete on the even CTA's barrier
+                    if (leader)
+                        mbar_arrive_expect_tx(&full_bar[s], 2 * stage_bytes);
+                    const uint32_t fb = cluster_addr(&full_bar[s], 0);
+                    tma_load_2d_pair(ring + (size_t)s * stage_bytes, &p.tmap_w, fb, kb * 64,
+                                     tile * 256 + (int)rank * 128);
+                    tma_load_2d_pair(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, fb, kb * 64,
+                                     (int)rank * (p.R_pad / 2));
+                } else {
+                    mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+                    tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
+                    tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                }
+                g_end = g + 1;
             }
             s_gend[mine] = g_end;
             // Gave up: this thread's copies in flight land before the CTA exits.  (In a
@@ -445,7 +476,8 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         // (in a pair, the even CTA issues for both)
         if (lane == 0 && leader) {
             const uint32_t idesc = idesc_bf16_f32(kPair ? 256 : 128, p.R_pad);
-            long long g = 0;
+            int s = 0;          // ring slot of the next k-block
+            uint32_t ph = 0;    // and its phase parity
             bool ok = true;
             for (int tile = tile0, i = 0; tile < tile1 && ok; ++tile, ++i) {
                 const int b = i & 1;
@@ -453,9 +485,8 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                     break;
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * p.acc_cols);
-                for (int j = 0; j < p.nk; ++j, ++g) {
-                    const int s = (int)(g % S);
-                    if (!mbar_wait_bounded(&full_bar[s], (uint32_t)(g / S) & 1u, &abort_flag, p.status)) {
+                for (int j = 0; j < p.nk; ++j) {
+                    if (!mbar_wait_bounded(&full_bar[s], ph, &abort_flag, p.status)) {
                         ok = false;
                         break;
                     }
@@ -475,6 +506,10 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                         tc_commit_pair(&empty_bar[s]);
                     else
                         tc_commit(&empty_bar[s]);
+                    if (++s == S) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
                 if (!ok)
                     break;
