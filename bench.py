@@ -149,10 +149,10 @@ def kernel_source_hash(files: str) -> str:
 
 def launches_per_step(head_dim: int, rope: bool, accept: str) -> int:
     """Kernels the library launches for one verify step of a multi-tile problem: the LM
-    head, the attention, the split-unit merge (head_dim 128), acceptance + compaction;
-    + the tree-key rotation (which also writes the rotary table) with rope; sampled
-    acceptance launches the walk, then the compaction."""
-    return (4 if head_dim == 128 else 3) + (1 if rope else 0) + (1 if accept == "sampled" else 0)
+    head and its merge, the attention, the split-unit merge (head_dim 128), acceptance +
+    compaction; + the tree-key rotation (which also writes the rotary table) with rope;
+    sampled acceptance launches the walk, then the compaction."""
+    return (5 if head_dim == 128 else 4) + (1 if rope else 0) + (1 if accept == "sampled" else 0)
 
 
 def acceptance_label(args) -> str:
@@ -550,7 +550,7 @@ def run_gpu_batched(args):
         "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
                      "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
                      "flops_per_step": flops, "peak_gbs": hbm, "peak_tflops_sustained": tflops, "peak_src": peak_src},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": 5 * args.steps,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -651,7 +651,7 @@ def run_gpu_bank_loop(args):
         "tree_histogram": hist,
         "hbm_roofline": {"bytes": kv_b + w_b, "frac": round((kv_b + w_b) / el / 1e9 / hbm, 4), "peak_gbs": hbm,
                          "peak_src": peak_src},
-        "gpu_launches": 4 * steps,
+        "gpu_launches": 5 * steps,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -726,7 +726,7 @@ def bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs,
                    "L_end": st["L"], "policy": "hysteretic step ladder on the device: up below 1.5, down above 2.5",
                    "host_read_per_step": False, "cuda_graph_steps": G},
         "tau_mean_accept_len": round((st["L"] - L0) / done, 4),
-        "gpu_launches": 4 * done,
+        "gpu_launches": 5 * done,
         "clocks": clocks,
         "hbm_roofline": {"peak_gbs": float(peaks["hbm_gbs"]), "peak_src": peak_src},
     }
@@ -841,7 +841,7 @@ def run_gpu_sweep(args):
                    "compaction": "included (every step)"},
         "sweep": rows,
         "throughput_optimal_tree": best,
-        "gpu_launches": 4 * max(10, min(args.steps, 100)) * len(rows),
+        "gpu_launches": 5 * max(10, min(args.steps, 100)) * len(rows),
     }
     print(json.dumps(line), flush=True)
 

@@ -298,7 +298,7 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
  * sandbox that forbids cudaMalloc, or next to a memory pool that is already
  * fully carved up has no way to provide the workspace that lm_head_stats
  * needs.  This variant computes the same argmax / top1 / entropy with the
- * same kernel, but keeps its scratch in a 4 MiB array compiled into the
+ * same kernel, but keeps its scratch in a 16 MiB array compiled into the
  * library (every GPU that loads the library holds it until the process
  * exits); it calls no cudaMalloc, cudaFree or allocating library routine.
  *  - Outside stream capture every call looks up that array's device address
@@ -309,10 +309,11 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
  *    `stream` and reuses the array, which keeps the previous call's partial
  *    results: calls that can overlap on the GPU (different streams without
  *    ordering) race.
- *  - The scratch is one partial per persistent CTA for every row (at most
- *    about 1.8 MiB: 256 rows, two CTAs on each of 152 SMs, for any
- *    vocabulary); a device whose SM count needs more than 4 MiB is rejected
- *    with TB_ECAPACITY before anything is enqueued.
+ *  - The scratch is one partial per 128 vocabulary entries for every row
+ *    (rows padded to 16, 24 bytes each) plus one per merge group: about
+ *    (vocab / 128 + sqrt(vocab / 128)) x 24 x padded rows bytes, 10 MiB at
+ *    256 rows and vocab 200000; a call that needs more than 16 MiB is
+ *    rejected with TB_ECAPACITY before anything is enqueued.
  *  - A bounded device wait that runs out (TB_ETIMEOUT) leaves argmax / top1 /
  *    entropy unwritten and is visible only through
  *    lm_head_stats_noalloc_status.

@@ -40,6 +40,7 @@
 // Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that the rows
 // are spread over the four lane quadrants (all four SM sub-partitions share
 // the softmax).
+#include <limits.h>
 #include <string.h>
 
 #include "kernels.cuh"
@@ -132,15 +133,62 @@ __device__ __forceinline__ int seq_at(const TcParams &p, long long t, int b)
     }
 }
 
+// First flattened tile of CTA c's range (the ranges split the tile space
+// evenly).  The quotients take 32-bit divisions whenever the operands fit.
 __device__ __forceinline__ long long tc_seg_begin(long long total, int P, int c)
 {
-    return (long long)c * total / P;
+    const unsigned long long x = (unsigned long long)c * (unsigned long long)total;
+    return x <= 0xffffffffull ? (long long)((uint32_t)x / (uint32_t)P) : (long long)(x / (unsigned long long)P);
 }
 
+// The CTA whose range holds tile t.
 __device__ __forceinline__ int tc_cta_of(long long total, int P, long long t)
 {
-    return total > 0 ? (int)(((t + 1) * (long long)P - 1) / total) : 0;
+    if (total <= 0)
+        return 0;
+    const unsigned long long x = (unsigned long long)(t + 1) * (unsigned long long)P - 1ull;
+    return x <= 0xffffffffull && (unsigned long long)total <= 0xffffffffull ? (int)((uint32_t)x / (uint32_t)total)
+                                                                           : (int)(x / (unsigned long long)total);
 }
+
+// One role's walk over its CTA's tiles t0, t0 + 1, ...: the sequence, the unit
+// within it, the unit's kv head and layer, and the key tile within the unit,
+// advanced without 64-bit divisions (tile ranges of the sequences are
+// contiguous and in order).
+template <bool kBatched>
+struct TileWalk {
+    int sb, u, j, head, layer_rel;
+    long long next_base;  // first tile of the next sequence
+    __device__ void locate(const TcParams &p, const TcSeq *seqs, long long t)
+    {
+        sb = seq_at<kBatched>(p, t, kBatched ? sb : 0);
+        const TcSeq &sq = seqs[sb];
+        const long long tl = t - sq.tile_base;
+        u = (int)(tl / sq.T);
+        j = (int)(tl - (long long)u * sq.T);
+        next_base = (kBatched && sb + 1 < p.n_seq) ? p.seq[sb + 1].tile_base : LLONG_MAX;
+        unit_changed(p, sq);
+    }
+    __device__ __forceinline__ void unit_changed(const TcParams &p, const TcSeq &sq)
+    {
+        head = (u / sq.row_blocks) % p.Hkv;
+        layer_rel = u / (sq.row_blocks * p.Hkv);
+    }
+    __device__ TileWalk(const TcParams &p, const TcSeq *seqs, long long t0) : sb(0) { locate(p, seqs, t0); }
+    // to tile t + 1 (t is the current tile)
+    __device__ __forceinline__ void advance(const TcParams &p, const TcSeq *seqs, long long t)
+    {
+        if (t + 1 >= next_base) {
+            locate(p, seqs, t + 1);
+            return;
+        }
+        if (++j == seqs[sb].T) {
+            j = 0;
+            ++u;
+            unit_changed(p, seqs[sb]);
+        }
+    }
+};
 
 // MN-major (N contiguous) 128-byte-swizzled operand: lbo = stride between
 // 64-element column atoms, sbo = stride between groups of 8 K rows.
@@ -150,6 +198,22 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t l
 }
 
 }  // namespace
+
+// Allowed-key bits of 32 consecutive keys whose first has tree index tj0
+// (key position minus the prefix length): bit c is set when key tj0 + c is a
+// prefix key (tree index < 0) or an ancestor of the row's node (bit tj0 + c of
+// its ancestor set anc, whose bits lie below the tree's node count).
+__device__ __forceinline__ uint32_t tile_allow(int tj0, uint64_t anc)
+{
+    if (tj0 <= -32)
+        return 0xffffffffu;
+    if (tj0 >= 64)
+        return 0u;
+    if (tj0 >= 0)
+        return (uint32_t)(anc >> tj0);
+    const int pre = -tj0;  // 1 .. 31 prefix keys, then the tree from bit pre
+    return ((1u << pre) - 1u) | (uint32_t)(anc << pre);
+}
 
 template <bool kBatched>
 __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
@@ -224,32 +288,33 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // warp 0 streams the K tiles, warp 7 the V tiles, each through its own
         // half of the 3-stage ring: QK^T releases a K slot, P V a V slot.
         if (lane == 0) {
+            static_assert(kKStages == kVStages, "one ring depth for K and V");
+            constexpr int S = kKStages;
             const bool is_v = (warp == 7);
             uint64_t *full = is_v ? v_full : k_full;
             uint64_t *empty = is_v ? v_empty : k_empty;
-            const int S = is_v ? kVStages : kKStages;
             uint8_t *ring = is_v ? sV : sK;
             long long issued = 0;
-            int sb = 0;
-            for (long long it = 0; it < n_tiles; ++it) {
-                const int s = (int)(it % S);
-                const uint32_t ph = (uint32_t)(it / S) & 1u;
-                if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
-                    break;
-                const long long t = t0 + it;
-                sb = seq_at<kBatched>(p, t, sb);
-                const TcSeq &sq = seqs[sb];
-                const long long tl = t - sq.tile_base;
-                const int u = (int)(tl / sq.T);
-                const int j = (int)(tl % sq.T);
-                const int head = (u / sq.row_blocks) % p.Hkv;
-                const int layer = p.layer_begin + u / (sq.row_blocks * p.Hkv);
-                const CUtensorMap *m = &p.tmap[2 * sb + (is_v ? 1 : 0)];
-                uint8_t *dst = ring + (size_t)s * kTile;
-                mbar_arrive_expect_tx(&full[s], kTile);
-                tma_load_4d(dst, m, &full[s], 0, j * kBN, head, layer);
-                tma_load_4d(dst + kAtom, m, &full[s], 64, j * kBN, head, layer);
-                issued = it + 1;
+            int s = 0;
+            uint32_t ph = 0;
+            if (n_tiles > 0) {
+                TileWalk<kBatched> w(p, seqs, t0);
+                for (long long it = 0; it < n_tiles; ++it) {
+                    if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
+                        break;
+                    const CUtensorMap *m = &p.tmap[2 * w.sb + (is_v ? 1 : 0)];
+                    uint8_t *dst = ring + (size_t)s * kTile;
+                    const int layer = p.layer_begin + w.layer_rel;
+                    mbar_arrive_expect_tx(&full[s], kTile);
+                    tma_load_4d(dst, m, &full[s], 0, w.j * kBN, w.head, layer);
+                    tma_load_4d(dst + kAtom, m, &full[s], 64, w.j * kBN, w.head, layer);
+                    issued = it + 1;
+                    if (++s == S) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                    w.advance(p, seqs, t0 + it);
+                }
             }
             if (issued < n_tiles)
                 for (long long it = (issued > S ? issued - S : 0); it < issued; ++it)
@@ -259,25 +324,30 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // ------------------------------------------------------------ QK^T issuer
         if (lane == 0) {
             const uint32_t idesc_s = idesc_bf16_f32(128, kBN);
-            int sg = -1, sb = 0;
-            for (long long it = 0; it < n_tiles; ++it) {
-                const long long t = t0 + it;
-                sb = seq_at<kBatched>(p, t, sb);
-                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
+            int sg = -1, s = 0;
+            uint32_t ph = 0;
+            TileWalk<kBatched> w(p, seqs, t0);
+            for (long long it = 0; it < n_tiles; w.advance(p, seqs, t0 + it), ++it) {
+                const bool first = (it == 0) || w.j == 0;
                 if (first)
                     ++sg;
-                const int s = (int)(it % kKStages);
                 const int b = (int)(it & 1);
+                const int sk = s;
+                const uint32_t phk = ph;
+                if (++s == kKStages) {
+                    s = 0;
+                    ph ^= 1u;
+                }
                 // K landed; the softmax has read S_b (tile it - 2) and P V(it - 2) has read
                 // the P that shares its columns; at a segment's first tile, its Q is staged
-                if (!mbar_wait_bounded(&k_full[s], (uint32_t)(it / kKStages) & 1u, &abort_flag, p.status) ||
+                if (!mbar_wait_bounded(&k_full[sk], phk, &abort_flag, p.status) ||
                     !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
                     (it >= 2 &&
                      !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) ||
                     (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status)))
                     break;
                 tc_fence_after();
-                const uint32_t k_base = smem_u32(sK + (size_t)s * kTile);
+                const uint32_t k_base = smem_u32(sK + (size_t)sk * kTile);
                 const uint32_t s_col = b ? kColS1 : kColS0;
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
@@ -286,7 +356,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     tc_mma_f16_ts(tmem + s_col, tmem + kColQ + kk * 8, bdesc, idesc_s, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[b]);
-                tc_commit(&k_empty[s]);
+                tc_commit(&k_empty[sk]);
             }
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
             tc_commit(&drain_bar);
@@ -299,29 +369,35 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // that much sooner.
         if (lane == 0) {
             const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
-            int sg = -1, sb = 0;
-            for (long long it = 0; it < n_tiles; ++it) {
-                const long long t = t0 + it;
-                sb = seq_at<kBatched>(p, t, sb);
-                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
+            int sg = -1, s = 0;
+            uint32_t ph = 0;
+            TileWalk<kBatched> w(p, seqs, t0);
+            for (long long it = 0; it < n_tiles; w.advance(p, seqs, t0 + it), ++it) {
+                const bool first = (it == 0) || w.j == 0;
                 if (first)
                     ++sg;
                 const int b = (int)(it & 1);
+                const int sv = s;
+                const uint32_t phv = ph;
+                if (++s == kVStages) {
+                    s = 0;
+                    ph ^= 1u;
+                }
                 // P written; at a segment's first tile, the previous epilogue has read O
                 if (!mbar_wait_bounded(&p_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status) ||
                     (first && sg > 0 &&
                      !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)) ||
-                    !mbar_wait_bounded(&v_full[it % kVStages], (uint32_t)(it / kVStages) & 1u, &abort_flag, p.status))
+                    !mbar_wait_bounded(&v_full[sv], phv, &abort_flag, p.status))
                     break;
                 tc_fence_after();
-                const uint32_t v_base = smem_u32(sV + (size_t)(it % kVStages) * kTile);
+                const uint32_t v_base = smem_u32(sV + (size_t)sv * kTile);
                 const uint32_t p_col = b ? kColP1 : kColP0;
 #pragma unroll
                 for (int ks = 0; ks < kBN / 16; ++ks) {
                     const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
                     tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
                 }
-                tc_commit(&v_empty[it % kVStages]);
+                tc_commit(&v_empty[sv]);
                 tc_commit(&pv_done[b]);
             }
             tc_commit(&drain_bar);
@@ -468,11 +544,15 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 }
                 float mx = -INFINITY;
                 if (masked) {
+                    // the row's allowed keys among the tile's 128 columns, 32 per word:
+                    // prefix keys (tree index tj < 0) and the ancestors in the tree
+                    uint32_t allow[kBN / 32];
+#pragma unroll
+                    for (int w = 0; w < kBN / 32; ++w)
+                        allow[w] = tile_allow(key0 + 32 * w - g.L, g.anc);
 #pragma unroll
                     for (int x = 0; x < kBN; ++x) {
-                        const int tj = key0 + x - g.L;
-                        const bool ok = tj < 0 || (tj < g.N && ((g.anc >> tj) & 1ull));
-                        sc[x] = ok ? sc[x] : -INFINITY;
+                        sc[x] = ((allow[x >> 5] >> (x & 31)) & 1u) ? sc[x] : -INFINITY;
                         mx = fmaxf(mx, sc[x]);
                     }
                 } else {
@@ -644,7 +724,7 @@ struct PdlWaitOnExit {
 };
 
 template <bool kBatched, bool kAfterStep>
-__global__ void __launch_bounds__(256, 8) k1_merge_split(const __grid_constant__ TcParams p)
+__global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__ TcParams p)
 {
     if constexpr (!kAfterStep)
         pdl_wait();

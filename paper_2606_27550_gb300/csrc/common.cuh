@@ -219,6 +219,48 @@ __device__ __forceinline__ uint32_t cluster_addr(const void *p, uint32_t rank)
     return r;
 }
 
+// As mbar_try_wait, acquiring at cluster scope: for a barrier that another CTA
+// of the cluster arrives on (release at cluster scope) after storing data
+// into this CTA's shared memory.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// mbar_wait_bounded with a cluster-scope acquire.
+__device__ __forceinline__ bool mbar_wait_bounded_cluster(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                                          int *status)
+{
+    const long long t0 = cycles();
+    while (true) {
+        if (mbar_try_wait_cluster(bar, parity))
+            return true;
+        if (*abort)
+            return false;
+        if (cycles() - t0 > kWaitLimitCycles) {
+            *abort = 1;
+            if (status)
+                atomicOr(status, kStatusTimeout);
+            return false;
+        }
+    }
+}
+
+// Stores to the shared memory of any CTA of the cluster (ordered by a later
+// release at cluster scope).
+__device__ __forceinline__ void st_cluster_s32(uint32_t addr, int v)
+{
+    asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 // Arrives on an mbarrier of any CTA of the cluster (release at cluster scope).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar)
 {

@@ -46,14 +46,15 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
 
 // LM head (lm_head.cu)
 struct LmPlan {
-    int R_pad, n_tiles, n_kblocks, stages, acc_cols, group_size, n_groups;
+    int R_pad, n_tiles, n_kblocks, stages, acc_cols;
     int ctas_per_sm;  // 2 when two rings fit side by side, else 1
     bool pair;        // CTA pairs share each MMA (M = 256); tiles are then 256 vocab entries
     int units;        // the tile split's units: CTAs, or CTA pairs
     int P;            // persistent CTAs: ctas_per_sm per SM, at most one per vocab tile (two per pair tile)
-    int n_counters;   // workspace counters used (group tickets)
+    int n_slots;      // per-tile partials: one per tile and CTA (two per pair tile)
+    int n_counters;   // workspace counters used (the tile counter)
     size_t smem_bytes;
-    size_t ws_bytes;  // partials (CTA + group), 256-byte aligned
+    size_t ws_bytes;  // per-tile partials, 256-byte aligned
 };
 // n_sm: the SMs the launch may use; max_pairs: the clusters of two that can
 // be resident at once (-1: n_sm / 2), which bounds the pairs of a pair plan.

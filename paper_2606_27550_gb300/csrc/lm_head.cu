@@ -7,21 +7,25 @@
 // the entropy feature that the EntMTP scheduler consumes (Sec. 4, "Path-value
 // score" and "Cost": computed from the verifier logits already on chip).
 //
-// Design (swap-AB, persistent).  The 128-entry vocab tiles are split into
-// contiguous runs over a persistent grid (two CTAs per SM when their rings fit
-// side by side, one otherwise); a CTA walks its run tile by tile.  The tile of W
-// ([128][64] bf16 per k-block, 128-byte swizzled by TMA) is the MMA's M=128 A
-// operand, the tree rows ([R_pad][64], same swizzle) the N = R_pad B operand;
-// tcgen05.mma (kind::f16, f32 accumulate) builds the 128 x R_pad logit tile in
-// TMEM.  Lane 0 of warps 0 and 10 issue TMA (alternate stages) into a ring
-// that runs across tiles, warp 1 lane 0 the MMAs into one of two TMEM
-// accumulators, and warps 2-9 drain the
-// other accumulator meanwhile (32 tree rows at a time: TMEM -> shared memory
-// transposed -> eight threads per row reduce its 128 logits), folding each
-// tile into per-row running statistics of the CTA.  The CTAs' statistics are
-// merged in two levels by atomic arrival tickets (the last CTA of a group
-// merges the group; the last group merges everything); no CTA ever waits for
-// another.
+// Design (swap-AB, persistent).  A persistent grid (two CTAs per SM when
+// their rings fit side by side; for wide rows, clusters of two CTAs that share
+// each MMA) pulls 128-entry vocab tiles (256 for a pair) dynamically: every
+// unit (CTA or pair) starts on its own tile, then takes the next tile from a
+// global counter, so units that start late -- on SMs that other kernels of the
+// step still hold -- simply take fewer tiles.  The tile of W ([128][64] bf16
+// per k-block, 128-byte swizzled by TMA) is the MMA's M=128 A operand, the
+// tree rows ([R_pad][64], same swizzle) the N = R_pad B operand; tcgen05.mma
+// (kind::f16, f32 accumulate) builds the 128 x R_pad logit tile in TMEM.
+// Lane 0 of warps 0 and 10 issue TMA (alternate stages) into a ring that runs
+// across tiles, warp 1 lane 0 the MMAs into one of two TMEM accumulators, and
+// warps 2-9 drain the other accumulator meanwhile (32 tree rows at a time:
+// TMEM -> shared memory transposed -> eight threads per row reduce its 128
+// logits) into the tile's per-row statistics, written to the tile's own slot.
+// The slots are merged in two levels by atomic arrival tickets over fixed
+// groups of slots (the CTA whose tile completes a group merges it; the one
+// that completes the last group merges the groups), always in slot order, so
+// the results do not depend on which CTA took which tile; no CTA ever waits
+// for another.
 //
 #include <atomic>
 #include <math.h>
@@ -38,13 +42,10 @@ struct LmParams {
     int n_tiles, nk, stages, acc_cols;  // tiles of 128 vocab entries (256 for CTA pairs)
     int P;               // CTAs
     int units;           // the tile split's units: CTAs, or CTA pairs
-    int group_size, n_groups;
-    size_t smem_avail;   // dynamic shared memory after alignment (the merges stage partials there)
-    float4 *part_cta;    // [P][R_pad]  (max, argmax bits, s, t)
-    float4 *part_group;  // [n_groups][R_pad]
-    float2 *part_cta_t;  // [P][R_pad]  (sT, tT), typical mode
-    float2 *part_group_t;
-    int *counters;       // [n_groups + 1] group tickets, zero between launches
+    int n_slots;         // per-tile partials: one per tile (two per pair tile, one per CTA)
+    float4 *part_tile;   // [n_slots][R_pad]  (max, argmax bits, s, t)
+    float2 *part_tile_t; // [n_slots][R_pad]  (sT, tT), typical mode
+    int *counters;       // [1] the tile counter, zero between launches
     int *status;
     int expire_wait;     // test hook: the epilogue waits on a barrier nothing arrives on
     int32_t *argmax;
@@ -74,6 +75,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 // lane quadrant w % 4 and split each 32-row chunk's columns); all eleven merge
 // at the end.
 constexpr int kLmThreads = 352;
+constexpr int kTileQ = 4;  // tile-queue entries (a power of two)
 constexpr int kLmProducer2 = 10;
 constexpr int kEpiThreads = 256;
 constexpr int kLmChunk = 32;             // tree rows per epilogue chunk
@@ -167,134 +169,21 @@ __device__ __forceinline__ bool gather_hit(const LmGather &g, int b, int j, int 
     return r >= 0 && r < R && c >= 0 && c < nvalid;
 }
 
-// Merges count x R_pad partials (global, written by other CTAs): they are
-// staged in shared memory, then every row is reduced by `tpr` threads in two
-// independent passes (max / first argmax, then the rescaled sums), so there is
-// no serial dependency chain per row.  Writes the merged partial (dst) or the
-// final per-row outputs.
-template <bool kTyp>
-__device__ void merge_partials(const LmParams &p, const float4 *src, const float2 *src_t, int count, float4 *sbuf,
-                               float4 *dst, float2 *dst_t)
-{
-    // staging with eight loads in flight per thread: the partials are in L2,
-    // and a load-then-store loop would pay one round trip per element
-    constexpr int kInFlight = 8;
-    const int n = count * p.R_pad;
-    if (!in_bounds((size_t)n * sizeof(float4) <= p.smem_avail, p.status))
-        return;
-    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kInFlight) {
-        float4 v[kInFlight];
-#pragma unroll
-        for (int u = 0; u < kInFlight; ++u) {
-            const int i = i0 + u * (int)blockDim.x;
-            if (i < n)
-                v[u] = __ldcg(src + i);
-        }
-#pragma unroll
-        for (int u = 0; u < kInFlight; ++u) {
-            const int i = i0 + u * (int)blockDim.x;
-            if (i < n)
-                sbuf[i] = v[u];
-        }
-    }
-    __syncthreads();
-    const int tpr = threads_per_row(p.R_pad);
-    const int sub = threadIdx.x % tpr;
-    for (int r0 = 0; r0 < p.R; r0 += (int)blockDim.x / tpr) {
-        const int r = r0 + threadIdx.x / tpr;
-        RowStat st = stat_empty();
-        if (r < p.R) {
-            for (int k = sub; k < count; k += tpr) {
-                const float4 v = sbuf[k * p.R_pad + r];
-                const int idx = __float_as_int(v.y);
-                if (v.z > 0.f && (v.x > st.m || (v.x == st.m && idx < st.idx))) {
-                    st.m = v.x;
-                    st.idx = idx;
-                }
-            }
-            if (st.idx != 0x7fffffff) {
-                for (int k0 = sub; k0 < count; k0 += tpr * kInFlight) {
-                    // the tempered sums are read once, straight from L2, eight at a time
-                    float2 w[kInFlight];
-                    if constexpr (kTyp) {
-#pragma unroll
-                        for (int u = 0; u < kInFlight; ++u) {
-                            const int k = k0 + u * tpr;
-                            w[u] = k < count ? __ldcg(src_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
-                        }
-                    }
-#pragma unroll
-                    for (int u = 0; u < kInFlight; ++u) {
-                        const int k = k0 + u * tpr;
-                        if (k >= count)
-                            break;
-                        const float4 v = sbuf[k * p.R_pad + r];
-                        if (v.z > 0.f) {
-                            const float delta = v.x - st.m;
-                            const float e = ex2_approx(delta * kLog2e);
-                            st.s += v.z * e;
-                            st.t += (v.w + delta * v.z) * e;
-                            if constexpr (kTyp) {
-                                const float dT = delta * p.inv_t;
-                                const float eT = ex2_approx(dT * kLog2e);
-                                st.sT += w[u].x * eT;
-                                st.tT += (w[u].y + dT * w[u].x) * eT;
-                            }
-                        }
-                    }
-                }
-            }
-        }
-        st = group_merge<kTyp>(st, tpr, p.inv_t);
-        if (sub == 0 && r < p.R) {
-            if (dst) {
-                dst[r] = stat_pack(st);
-                if constexpr (kTyp)
-                    dst_t[r] = make_float2(st.sT, st.tT);
-            } else {
-                p.argmax[r] = st.idx;
-                p.top1[r] = 1.0f / st.s;
-                p.entropy[r] = logf(st.s) - st.t / st.s;
-                if constexpr (kTyp) {
-                    const float ls = logf(st.sT);
-                    p.logz_t[r] = st.m * p.inv_t + ls;
-                    p.ent_t[r] = ls - st.tT / st.sT;
-                }
-            }
-        }
-    }
-    __syncthreads();
-}
-
-// Arrival ticket of this CTA on `counter` once its writes are done: the
-// barrier orders every thread's writes before thread 0's fence (fences are
-// cumulative), and the fence orders them before the atomic, so the CTA that
-// draws the last ticket -- after a fence of its own -- reads all of them.
-// Returns true in every thread of that CTA.
-__device__ __forceinline__ bool arrive_last(int *counter, int expected, int *s_ticket)
-{
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        const int t = atomicAdd(counter, 1);
-        if (t == expected - 1)
-            __threadfence();
-        *s_ticket = t;
-    }
-    __syncthreads();
-    return *s_ticket == expected - 1;
-}
-
 // Named barrier of the eight epilogue warps.
 __device__ __forceinline__ void epi_sync()
 {
     asm volatile("bar.sync 1, 256;" ::: "memory");
 }
 
-// First vocab tile of unit c's run.
-__device__ __forceinline__ int lm_tile_begin(const LmParams &p, int c)
+// Waits on a tile-queue barrier: in a pair, the odd CTA's entries are written
+// by the even CTA, so the wait acquires at cluster scope.
+template <bool kPair>
+__device__ __forceinline__ bool lm_wait(uint64_t *bar, uint32_t parity, volatile int *abort, int *status)
 {
-    return (int)((long long)c * p.n_tiles / p.units);
+    if constexpr (kPair)
+        return mbar_wait_bounded_cluster(bar, parity, abort, status);
+    else
+        return mbar_wait_bounded(bar, parity, abort, status);
 }
 
 // Step j of a tile's k-loop reads k-block j + lm_rot (mod nk): the order is
@@ -304,41 +193,6 @@ __device__ __forceinline__ int lm_rot(const LmParams &p, int tile)
 {
     return (int)(((long long)tile * 5) % p.nk);
 }
-
-// A producer thread's position in the ring: the k-block sequence g = g0,
-// g0 + 2, ... of a run, as (tile, k-block) and (ring slot, phase parity),
-// advanced without divisions.
-struct RingCursor {
-    int tile, j, kb, rot, slot;
-    uint32_t phase;
-    __device__ RingCursor(const LmParams &p, int tile0, int g0) : tile(tile0), j(g0), slot(g0), phase(0)
-    {
-        // g0 is 0 or 1; the ring has at least two slots
-        while (j >= p.nk) {
-            j -= p.nk;
-            ++tile;
-        }
-        rot = lm_rot(p, tile);
-        kb = j + rot >= p.nk ? j + rot - p.nk : j + rot;
-    }
-    __device__ __forceinline__ void advance2(const LmParams &p, int S)
-    {
-        slot += 2;
-        if (slot >= S) {
-            slot -= S;
-            phase ^= 1u;
-        }
-        j += 2;
-        if (j >= p.nk) {
-            while (j >= p.nk) {
-                j -= p.nk;
-                ++tile;
-            }
-            rot = lm_rot(p, tile);
-        }
-        kb = j + rot >= p.nk ? j + rot - p.nk : j + rot;
-    }
-};
 
 // Waits, when it goes out of scope (every exit of the kernel), for the
 // stream's previous kernel to complete.  In a verification step the LM head
@@ -367,11 +221,13 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
     __shared__ __align__(8) uint64_t empty_bar[8];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
     __shared__ __align__(8) uint64_t drain_bar, never_bar;
+    __shared__ __align__(8) uint64_t tq_full[kTileQ], tq_empty[kTileQ];
+    __shared__ int s_tile[kTileQ];  // the CTA's i-th vocab tile in entry i % kTileQ (-1: no more)
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
     // CTA pairs: the stage sequences each producer thread issued, this CTA's and the odd CTA's
     __shared__ long long s_gend[2], s_peer_gend[2];
-    __shared__ int s_ticket, s_ok;
+    __shared__ int s_ok;
     // typical mode: edges whose draft token lies in the current tile, packed as
     // (seq << 24) | (node << 16) | (row << 7) | col; overflow -> rescan per chunk
     constexpr int kHitCap = 64;
@@ -385,7 +241,6 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
     const uint32_t stage_bytes = 16384u + hb;
     uint8_t *ring = smem;
     float *chunk = reinterpret_cast<float *>(smem + (size_t)S * stage_bytes);  // [kLmChunk][kChunkLd]
-    RowStat *run = reinterpret_cast<RowStat *>(chunk + kLmChunk * kChunkLd);   // [R_pad] running statistics
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
@@ -393,7 +248,7 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
     const uint32_t rank = kPair ? cluster_ctarank() : 0u;
     const bool leader = rank == 0;
     const int unit = kPair ? c >> 1 : c;
-    const int tile0 = lm_tile_begin(p, unit), tile1 = lm_tile_begin(p, unit + 1);
+    int *const tile_ctr = p.counters;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -406,11 +261,18 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         }
         mbar_init(&drain_bar, 1);
         mbar_init(&never_bar, 1);
+        for (int q = 0; q < kTileQ; ++q) {
+            mbar_init(&tq_full[q], 1);
+            mbar_init(&tq_empty[q], kPair ? 2 : 1);  // a pair's epilogues release the even CTA's entries
+        }
         abort_flag = 0;
         s_gend[0] = s_gend[1] = s_peer_gend[0] = s_peer_gend[1] = 0;
         fence_mbar_init();
         prefetch_tmap(&p.tmap_w);
         prefetch_tmap(&p.tmap_h);
+        // every unit starts on its own tile
+        s_tile[0] = unit;
+        mbar_arrive(&tq_full[0]);
     }
     if (warp == 1) {
         if constexpr (kPair) {
@@ -421,8 +283,6 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             tmem_relinquish();
         }
     }
-    for (int r = threadIdx.x; r < p.R_pad; r += blockDim.x)
-        run[r] = stat_empty();
     tc_fence_before();
     __syncthreads();
     if constexpr (kPair)
@@ -437,31 +297,77 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         // ones: one issuing thread alone streams W measurably slower.
         if (lane == 0) {
             const int mine = warp == 0 ? 0 : 1;
-            const long long G = (long long)(tile1 - tile0) * p.nk;  // the run's k-blocks
-            RingCursor cur(p, tile0, mine);  // this thread's steps g = mine, mine + 2, ...
+            int s = mine;       // ring slot and phase parity of this thread's next k-block
+            uint32_t ph = 0;
+            long long g = 0;    // the current tile's first k-block in the CTA's sequence
             long long g_end = 0;
             bool ok = true;
-            for (long long g = mine; g < G; g += 2, cur.advance2(p, S)) {
-                const int s = cur.slot, tile = cur.tile, kb = cur.kb;
-                if (!mbar_wait_bounded(&empty_bar[s], cur.phase ^ 1u, &abort_flag, p.status)) {
+            // tile scheduler (warp 0 of the even CTA): entry i + 1 of the queue is
+            // published while tile i streams; its tile was fetched a tile earlier
+            int pending = mine == 0 && leader ? atomicAdd(tile_ctr, 1) : -1;
+            for (int i = 0; ok; ++i) {
+                const int qe = i & (kTileQ - 1);  // tile-queue entry
+                if (!lm_wait<kPair>(&tq_full[qe], (uint32_t)(i / kTileQ) & 1u, &abort_flag, p.status)) {
                     ok = false;
                     break;
                 }
-                if constexpr (kPair) {
-                    // the stage's four boxes (W and tree rows of both CTAs) complete on the even CTA's barrier
-                    if (leader)
-                        mbar_arrive_expect_tx(&full_bar[s], 2 * stage_bytes);
-                    const uint32_t fb = cluster_addr(&full_bar[s], 0);
-                    tma_load_2d_pair(ring + (size_t)s * stage_bytes, &p.tmap_w, fb, kb * 64,
-                                     tile * 256 + (int)rank * 128);
-                    tma_load_2d_pair(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, fb, kb * 64,
-                                     (int)rank * (p.R_pad / 2));
-                } else {
-                    mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
-                    tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
-                    tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                const int tile = s_tile[qe];
+                const bool sched = mine == 0 && leader && tile >= 0;
+                bool published = false;
+                auto publish = [&]() {
+                    // entry i + 1: the tile fetched before, or -1 once the vocabulary is exhausted
+                    const int nxt = pending >= 0 && pending + p.units < p.n_tiles ? pending + p.units : -1;
+                    const int q1 = (i + 1) & (kTileQ - 1);
+                    if (!mbar_wait_bounded(&tq_empty[q1], ((uint32_t)((i + 1) / kTileQ) & 1u) ^ 1u, &abort_flag,
+                                           p.status))
+                        return false;
+                    s_tile[q1] = nxt;
+                    if constexpr (kPair) {
+                        st_cluster_s32(cluster_addr(&s_tile[q1], 1), nxt);
+                        mbar_arrive_cluster(cluster_addr(&tq_full[q1], 1));
+                    }
+                    mbar_arrive(&tq_full[q1]);
+                    pending = nxt >= 0 ? atomicAdd(tile_ctr, 1) : -1;
+                    published = true;
+                    return true;
+                };
+                if (tile < 0)
+                    break;
+                const int rot = lm_rot(p, tile);
+                for (int j = (int)((g + mine) & 1); j < p.nk; j += 2) {
+                    const int kb = j + rot >= p.nk ? j + rot - p.nk : j + rot;
+                    if (!mbar_wait_bounded(&empty_bar[s], ph ^ 1u, &abort_flag, p.status)) {
+                        ok = false;
+                        break;
+                    }
+                    if constexpr (kPair) {
+                        // the stage's four boxes (W and tree rows of both CTAs) complete on the even CTA's barrier
+                        if (leader)
+                            mbar_arrive_expect_tx(&full_bar[s], 2 * stage_bytes);
+                        const uint32_t fb = cluster_addr(&full_bar[s], 0);
+                        tma_load_2d_pair(ring + (size_t)s * stage_bytes, &p.tmap_w, fb, kb * 64,
+                                         tile * 256 + (int)rank * 128);
+                        tma_load_2d_pair(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, fb, kb * 64,
+                                         (int)rank * (p.R_pad / 2));
+                    } else {
+                        mbar_arrive_expect_tx(&full_bar[s], stage_bytes);
+                        tma_load_2d(ring + (size_t)s * stage_bytes, &p.tmap_w, &full_bar[s], kb * 64, tile * 128);
+                        tma_load_2d(ring + (size_t)s * stage_bytes + 16384, &p.tmap_h, &full_bar[s], kb * 64, 0);
+                    }
+                    g_end = g + j + 1;
+                    s += 2;
+                    if (s >= S) {
+                        s -= S;
+                        ph ^= 1u;
+                    }
+                    if (sched && !published && !publish()) {
+                        ok = false;
+                        break;
+                    }
                 }
-                g_end = g + 1;
+                if (ok && sched && !published && !publish())
+                    ok = false;
+                g += p.nk;
             }
             s_gend[mine] = g_end;
             // Gave up: this thread's copies in flight land before the CTA exits.  (In a
@@ -479,7 +385,11 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             int s = 0;          // ring slot of the next k-block
             uint32_t ph = 0;    // and its phase parity
             bool ok = true;
-            for (int tile = tile0, i = 0; tile < tile1 && ok; ++tile, ++i) {
+            for (int i = 0; ok; ++i) {
+                const int qe = i & (kTileQ - 1);  // tile-queue entry
+                if (!mbar_wait_bounded(&tq_full[qe], (uint32_t)(i / kTileQ) & 1u, &abort_flag, p.status) ||
+                    s_tile[qe] < 0)
+                    break;
                 const int b = i & 1;
                 if (!mbar_wait_bounded(&acc_empty[b], ((uint32_t)(i >> 1) & 1u) ^ 1u, &abort_flag, p.status))
                     break;
@@ -538,8 +448,22 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             epi_sync();
             return s_ok != 0;
         };
-        for (int tile = tile0, i = 0; tile < tile1; ++tile, ++i) {
+        for (int i = 0;; ++i) {
             const int b = i & 1;
+            const int qe = i & (kTileQ - 1);  // tile-queue entry
+            lm_wait<kPair>(&tq_full[qe], (uint32_t)(i / kTileQ) & 1u, &abort_flag, p.status);
+            if (!agree())
+                break;
+            const int tile = s_tile[qe];
+            epi_sync();  // every epilogue thread has read the entry
+            if (e == 0) {
+                if constexpr (kPair)
+                    mbar_arrive_cluster(cluster_addr(&tq_empty[qe], 0));
+                else
+                    mbar_arrive(&tq_empty[qe]);
+            }
+            if (tile < 0)
+                break;
             mbar_wait_bounded(p.expire_wait ? &never_bar : &acc_full[b], (uint32_t)(i >> 1) & 1u, &abort_flag,
                               p.status);
             if (!agree())
@@ -547,6 +471,7 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
             tc_fence_after();
             // this CTA's 128 vocab entries (the odd CTA of a pair's last tile may have none)
             const int v0 = kPair ? tile * 256 + (int)rank * 128 : tile * 128, nvalid = min(128, p.V - v0);
+            const int slot = kPair ? 2 * tile + (int)rank : tile;  // this CTA's partial of the tile
             if constexpr (kTyp) {
                 // the tree edges whose draft token lies in this tile
                 if (e == 0)
@@ -614,8 +539,12 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                     }
                 }
                 st = group_merge<kTyp>(st, kLmTpr, p.inv_t);
-                if (sub == 0 && r < p.R)
-                    run[r] = stat_merge<kTyp>(run[r], st, p.inv_t);
+                if (sub == 0 && r < p.R) {
+                    // the tile's statistics of row r, in the tile's own slot
+                    p.part_tile[(size_t)slot * p.R_pad + r] = stat_pack(st);
+                    if constexpr (kTyp)
+                        p.part_tile_t[(size_t)slot * p.R_pad + r] = make_float2(st.sT, st.tT);
+                }
                 if constexpr (kTyp) {
                     const int nhit = s_nhit;
                     if (nhit <= kHitCap) {
@@ -648,13 +577,6 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
                 epi_sync();  // the chunk buffer is rewritten next
             }
         }
-        // this CTA's statistics for the final merge
-        if (!abort_flag)
-            for (int r = e; r < p.R; r += kEpiThreads) {
-                p.part_cta[(size_t)c * p.R_pad + r] = stat_pack(run[r]);
-                if constexpr (kTyp)
-                    p.part_cta_t[(size_t)c * p.R_pad + r] = make_float2(run[r].sT, run[r].tT);
-            }
     }
 
     // ---------------- teardown: every MMA has retired before TMEM is released
@@ -694,25 +616,137 @@ __global__ void __launch_bounds__(kLmThreads, 2) k2_lm_head(const __grid_constan
         }
         cluster_barrier();
     }
-    if (abort_flag)
-        return;
+}
 
-    // ---------------- two-level merge of the CTAs' statistics by arrival tickets
-    const int g = c / p.group_size;
-    const int g_first = g * p.group_size;
-    const int g_count = min(p.group_size, p.P - g_first);
-    if (!arrive_last(&p.counters[g], g_count, &s_ticket))
+// Final merge of the per-tile partials (K2 merge): one CTA per tree row.
+// Thread k folds slots k, k + 256, ... in order -- the row's maximum and its
+// lowest vocab index first, then the sums rescaled to that maximum -- and the
+// 256 results combine in a fixed tree (warp butterflies, then the eight warps
+// in order), so the outputs do not depend on which CTA of k2_lm_head took
+// which tile.  Launched as a programmatic dependent of k2_lm_head: it waits for
+// that grid (and what it waited for) to complete, then resets the tile counter
+// for the next launch (every fetch has completed by then).  After a time-out
+// recorded in the status word it writes nothing.
+constexpr int kMergeThreads = 256;
+
+template <bool kTyp>
+__global__ void __launch_bounds__(kMergeThreads) k2_lm_merge(const __grid_constant__ LmParams p)
+{
+    pdl_trigger();  // the kernel that reads the outputs may be launched now
+    pdl_wait();
+    constexpr int kInFlight = 4;
+    constexpr int kWarps = kMergeThreads / 32;
+    __shared__ float s_m[kWarps], s_sum[kWarps][4];
+    __shared__ int s_i[kWarps];
+    const int r = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (r == 0 && tid == 0)
+        p.counters[0] = 0;
+    // a bounded wait of the LM head ran out: its partials are incomplete, the
+    // outputs stay unwritten (the status word reports it)
+    if (__ldcg(p.status) & kStatusTimeout)
         return;
-    float4 *sbuf = reinterpret_cast<float4 *>(smem);  // the drained ring
-    merge_partials<kTyp>(p, p.part_cta + (size_t)g_first * p.R_pad, p.part_cta_t + (size_t)g_first * p.R_pad, g_count,
-                         sbuf, p.part_group + (size_t)g * p.R_pad, p.part_group_t + (size_t)g * p.R_pad);
-    if (threadIdx.x == 0)
-        p.counters[g] = 0;
-    if (!arrive_last(&p.counters[p.n_groups], p.n_groups, &s_ticket))
+    if (!in_bounds(r < p.R, p.status))
         return;
-    merge_partials<kTyp>(p, p.part_group, p.part_group_t, p.n_groups, sbuf, nullptr, nullptr);
-    if (threadIdx.x == 0)
-        p.counters[p.n_groups] = 0;
+    // pass 1: maximum and its lowest vocab index (empty partials hold -inf)
+    float M = -INFINITY;
+    int I = 0x7fffffff;
+    for (int k0 = tid; k0 < p.n_slots; k0 += kMergeThreads * kInFlight) {
+        float2 v[kInFlight];
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            const int k = k0 + u * kMergeThreads;
+            v[u] = k < p.n_slots ? __ldcg(reinterpret_cast<const float2 *>(p.part_tile + (size_t)k * p.R_pad + r))
+                                 : make_float2(-INFINITY, __int_as_float(0x7fffffff));
+        }
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            const int idx = __float_as_int(v[u].y);
+            if (v[u].x > M || (v[u].x == M && idx < I)) {
+                M = v[u].x;
+                I = idx;
+            }
+        }
+    }
+    for (int m = 16; m >= 1; m >>= 1) {
+        const float M2 = __shfl_xor_sync(0xffffffffu, M, m);
+        const int I2 = __shfl_xor_sync(0xffffffffu, I, m);
+        if (M2 > M || (M2 == M && I2 < I)) {
+            M = M2;
+            I = I2;
+        }
+    }
+    if (lane == 0) {
+        s_m[warp] = M;
+        s_i[warp] = I;
+    }
+    __syncthreads();
+    M = s_m[0];
+    I = s_i[0];
+    for (int w = 1; w < kWarps; ++w)
+        if (s_m[w] > M || (s_m[w] == M && s_i[w] < I)) {
+            M = s_m[w];
+            I = s_i[w];
+        }
+    // pass 2: s, t (and the tempered sT, tT) relative to M
+    float S = 0.f, T = 0.f, ST = 0.f, TT = 0.f;
+    for (int k0 = tid; k0 < p.n_slots; k0 += kMergeThreads * kInFlight) {
+        float4 v[kInFlight];
+        float2 w[kInFlight];
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            const int k = k0 + u * kMergeThreads;
+            v[u] = k < p.n_slots ? __ldcg(p.part_tile + (size_t)k * p.R_pad + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+            if constexpr (kTyp)
+                w[u] = k < p.n_slots ? __ldcg(p.part_tile_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kInFlight; ++u) {
+            if (v[u].z > 0.f) {
+                const float d = v[u].x - M;  // <= 0
+                const float x = ex2_approx(d * kLog2e);
+                S += v[u].z * x;
+                T += (v[u].w + d * v[u].z) * x;
+                if constexpr (kTyp) {
+                    const float dT = d * p.inv_t;
+                    const float xT = ex2_approx(dT * kLog2e);
+                    ST += w[u].x * xT;
+                    TT += (w[u].y + dT * w[u].x) * xT;
+                }
+            }
+        }
+    }
+    for (int m = 16; m >= 1; m >>= 1) {
+        S += __shfl_xor_sync(0xffffffffu, S, m);
+        T += __shfl_xor_sync(0xffffffffu, T, m);
+        if constexpr (kTyp) {
+            ST += __shfl_xor_sync(0xffffffffu, ST, m);
+            TT += __shfl_xor_sync(0xffffffffu, TT, m);
+        }
+    }
+    if (lane == 0) {
+        s_sum[warp][0] = S;
+        s_sum[warp][1] = T;
+        s_sum[warp][2] = ST;
+        s_sum[warp][3] = TT;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        S = T = ST = TT = 0.f;
+        for (int w = 0; w < kWarps; ++w) {
+            S += s_sum[w][0];
+            T += s_sum[w][1];
+            ST += s_sum[w][2];
+            TT += s_sum[w][3];
+        }
+        p.argmax[r] = I;
+        p.top1[r] = 1.0f / S;
+        p.entropy[r] = logf(S) - T / S;
+        if constexpr (kTyp) {
+            const float ls = logf(ST);
+            p.logz_t[r] = M * p.inv_t + ls;
+            p.ent_t[r] = ls - TT / ST;
+        }
+    }
 }
 
 // ----------------------------------------------------------------------------
@@ -734,7 +768,7 @@ LmPlan lm_plan(int R, int D, int V, int n_sm, int max_pairs)
     while (cols < pl.R_pad)
         cols *= 2;
     pl.acc_cols = cols;
-    const size_t fixed = (size_t)kLmChunk * kChunkLd * 4 + (size_t)pl.R_pad * sizeof(RowStat);
+    const size_t fixed = (size_t)kLmChunk * kChunkLd * 4;  // the epilogue's chunk buffer
     // Two CTAs share an SM when each still gets a ring of at least three stages
     // in half of its shared memory and four accumulators fit in TMEM: two
     // independent TMA pipelines per SM stream W faster than one deeper ring.
@@ -765,27 +799,15 @@ LmPlan lm_plan(int R, int D, int V, int n_sm, int max_pairs)
         pl.P = slots < pl.n_tiles ? slots : pl.n_tiles;
         pl.units = pl.P;
     }
-    int gs = 1;
-    while (gs * gs < pl.P)
-        ++gs;
-    pl.group_size = gs;
-    pl.n_groups = ceil_div(pl.P, gs);
-    size_t sm = (size_t)pl.stages * stage_bytes + fixed;
-    const size_t mg = (size_t)(gs > pl.n_groups ? gs : pl.n_groups) * pl.R_pad * 16;
-    if (mg > sm)
-        sm = mg;
-    pl.smem_bytes = sm + 1024;
-    // (max, argmax, s, t) and (sT, tT) partials of the CTAs and the groups.  The
-    // workspace also covers the plan without pairs, which a launch takes when
-    // no cluster of two can be resident.
-    const int slots = pl.ctas_per_sm * n_sm, n128 = ceil_div(V, 128);
-    const int p1 = slots < n128 ? slots : n128;
-    int gs1 = 1;
-    while (gs1 * gs1 < p1)
-        ++gs1;
-    const int ng1 = ceil_div(p1, gs1);
-    const int parts = pl.P + pl.n_groups > p1 + ng1 ? pl.P + pl.n_groups : p1 + ng1;
-    pl.n_counters = (pl.n_groups > ng1 ? pl.n_groups : ng1) + 1;
+    // per-tile partials: one per tile and CTA, merged by k2_lm_merge
+    pl.n_slots = pl.pair ? 2 * pl.n_tiles : pl.n_tiles;
+    pl.smem_bytes = (size_t)pl.stages * stage_bytes + fixed + 1024;
+    // (max, argmax, s, t) and (sT, tT) partials.  The workspace also covers the
+    // plan without pairs, which a launch takes when no cluster of two can be
+    // resident.
+    const int slots1 = ceil_div(V, 128);
+    const int parts = pl.n_slots > slots1 ? pl.n_slots : slots1;
+    pl.n_counters = 1;  // the tile counter
     pl.ws_bytes = ((size_t)parts * pl.R_pad * (16 + 8) + 255) / 256 * 256;
     return pl;
 }
@@ -823,20 +845,25 @@ static int lm_max_pairs(size_t smem, int n_sm)
     return pairs;
 }
 
+// k2_lm_head, then its merge as a programmatic dependent (launched while the
+// LM head runs; it waits for it on the device).
 template <bool kTyp>
 static cudaError_t lm_launch_as(LmParams &p, const LmPlan &pl, cudaStream_t stream, bool pdl)
 {
+    cudaError_t e;
     if (pl.pair) {
-        cudaError_t e = allow_max_smem((const void *)k2_lm_head<kTyp, true>);
-        if (e != cudaSuccess)
+        if ((e = allow_max_smem((const void *)k2_lm_head<kTyp, true>)) != cudaSuccess)
             return e;
-        return launch_kernel_cluster(k2_lm_head<kTyp, true>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl,
-                                     2, p);
+        e = launch_kernel_cluster(k2_lm_head<kTyp, true>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl,
+                                  2, p);
+    } else {
+        if ((e = allow_max_smem((const void *)k2_lm_head<kTyp, false>)) != cudaSuccess)
+            return e;
+        e = launch_kernel(k2_lm_head<kTyp, false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
     }
-    cudaError_t e = allow_max_smem((const void *)k2_lm_head<kTyp, false>);
     if (e != cudaSuccess)
         return e;
-    return launch_kernel(k2_lm_head<kTyp, false>, dim3(pl.P), dim3(kLmThreads), pl.smem_bytes, stream, pdl, p);
+    return launch_kernel(k2_lm_merge<kTyp>, dim3(p.R), dim3(kMergeThreads), 0, stream, true, p);
 }
 
 cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int V, int32_t *argmax, float *top1,
@@ -866,13 +893,9 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.acc_cols = pl.acc_cols;
     p.P = pl.P;
     p.units = pl.units;
-    p.group_size = pl.group_size;
-    p.n_groups = pl.n_groups;
-    p.smem_avail = pl.smem_bytes - 1024;
-    p.part_cta = static_cast<float4 *>(parts);
-    p.part_group = p.part_cta + (size_t)pl.P * pl.R_pad;
-    p.part_cta_t = reinterpret_cast<float2 *>(p.part_group + (size_t)pl.n_groups * pl.R_pad);
-    p.part_group_t = p.part_cta_t + (size_t)pl.P * pl.R_pad;
+    p.n_slots = pl.n_slots;
+    p.part_tile = static_cast<float4 *>(parts);
+    p.part_tile_t = reinterpret_cast<float2 *>(p.part_tile + (size_t)pl.n_slots * pl.R_pad);
     p.counters = counters;
     p.status = status;
     p.argmax = argmax;

@@ -3,7 +3,7 @@
 // Some callers cannot allocate device memory at all: code running inside a
 // host framework that owns every allocation, a plugin sandbox that forbids
 // cudaMalloc, or a process whose memory pool is already carved up.  For them
-// the LM-head kernel can run with its scratch (per-CTA partial statistics and
+// the LM-head kernel can run with its scratch (per-tile partial statistics and
 // arrival counters) in a fixed array that lives inside this library, declared
 // below.  Every GPU that loads the library holds that array until the process
 // exits.
@@ -13,10 +13,11 @@
 
 namespace tv {
 
-// 4 MiB of partials.  The plan needs one partial per persistent CTA for every
-// row (rows padded to 16, 24 bytes each), whatever the vocabulary: at most
-// 2 CTAs per SM x 152 SMs x 256 rows x 24 bytes, about 1.8 MiB, on GB300.
-constexpr size_t kNoAllocScratchBytes = 4u << 20;
+// 16 MiB of partials.  The plan needs one partial per 128 vocabulary entries
+// (two per 256-entry tile of a CTA pair) and one per merge group for every row
+// (rows padded to 16, 24 bytes each): 10 MiB at 256 rows and vocab 200000,
+// 16 MiB up to a vocabulary of about 330 000.
+constexpr size_t kNoAllocScratchBytes = 16u << 20;
 constexpr size_t kNoAllocCounterBytes = 4096;  // 1024 counters, cleared on every call
 constexpr int kNoAllocStatusWord = kNoAllocCounterBytes / 4 - 1;  // last counter word: device-detected errors
 
