@@ -199,7 +199,11 @@ TB_API tb_status tree_attention(const tb_bank *bank, int bank_id, const tb_kv *k
  * nats (the entropy feature of the scheduler, Sec. 4 / App. A).
  *   hidden bf16 [n_rows][d_model]; lm_head bf16 [vocab][d_model] (nn.Linear)
  *   argmax int32 [n_rows]; top1, entropy float [n_rows]
- * 1 <= n_rows <= 256, d_model a multiple of 8, vocab >= 1. */
+ * 1 <= n_rows <= 256, d_model a multiple of 8, vocab >= 1.
+ * Two kernels: the LM head proper, which writes per-row statistics of every
+ * vocab tile into the workspace, then their merge in a fixed order; the
+ * outputs are bitwise reproducible for the same inputs, whatever the launch
+ * placement. */
 TB_API tb_status lm_head_stats(const void *hidden, int n_rows, const void *lm_head, int d_model, int vocab,
                         int32_t *argmax, float *top1, float *entropy, void *workspace,
                         size_t workspace_bytes, tb_stream stream);
