@@ -40,7 +40,6 @@
 // Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that the rows
 // are spread over the four lane quadrants (all four SM sub-partitions share
 // the softmax).
-#include <limits.h>
 #include <string.h>
 
 #include "kernels.cuh"
@@ -151,45 +150,6 @@ __device__ __forceinline__ int tc_cta_of(long long total, int P, long long t)
                                                                            : (int)(x / (unsigned long long)total);
 }
 
-// One role's walk over its CTA's tiles t0, t0 + 1, ...: the sequence, the unit
-// within it, the unit's kv head and layer, and the key tile within the unit,
-// advanced without 64-bit divisions (tile ranges of the sequences are
-// contiguous and in order).
-template <bool kBatched>
-struct TileWalk {
-    int sb, u, j, head, layer_rel;
-    long long next_base;  // first tile of the next sequence
-    __device__ void locate(const TcParams &p, const TcSeq *seqs, long long t)
-    {
-        sb = seq_at<kBatched>(p, t, kBatched ? sb : 0);
-        const TcSeq &sq = seqs[sb];
-        const long long tl = t - sq.tile_base;
-        u = (int)(tl / sq.T);
-        j = (int)(tl - (long long)u * sq.T);
-        next_base = (kBatched && sb + 1 < p.n_seq) ? p.seq[sb + 1].tile_base : LLONG_MAX;
-        unit_changed(p, sq);
-    }
-    __device__ __forceinline__ void unit_changed(const TcParams &p, const TcSeq &sq)
-    {
-        head = (u / sq.row_blocks) % p.Hkv;
-        layer_rel = u / (sq.row_blocks * p.Hkv);
-    }
-    __device__ TileWalk(const TcParams &p, const TcSeq *seqs, long long t0) : sb(0) { locate(p, seqs, t0); }
-    // to tile t + 1 (t is the current tile)
-    __device__ __forceinline__ void advance(const TcParams &p, const TcSeq *seqs, long long t)
-    {
-        if (t + 1 >= next_base) {
-            locate(p, seqs, t + 1);
-            return;
-        }
-        if (++j == seqs[sb].T) {
-            j = 0;
-            ++u;
-            unit_changed(p, seqs[sb]);
-        }
-    }
-};
-
 // MN-major (N contiguous) 128-byte-swizzled operand: lbo = stride between
 // 64-element column atoms, sbo = stride between groups of 8 K rows.
 __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t lbo, uint32_t sbo)
@@ -288,33 +248,32 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // warp 0 streams the K tiles, warp 7 the V tiles, each through its own
         // half of the 3-stage ring: QK^T releases a K slot, P V a V slot.
         if (lane == 0) {
-            static_assert(kKStages == kVStages, "one ring depth for K and V");
-            constexpr int S = kKStages;
             const bool is_v = (warp == 7);
             uint64_t *full = is_v ? v_full : k_full;
             uint64_t *empty = is_v ? v_empty : k_empty;
+            const int S = is_v ? kVStages : kKStages;
             uint8_t *ring = is_v ? sV : sK;
             long long issued = 0;
-            int s = 0;
-            uint32_t ph = 0;
-            if (n_tiles > 0) {
-                TileWalk<kBatched> w(p, seqs, t0);
-                for (long long it = 0; it < n_tiles; ++it) {
-                    if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
-                        break;
-                    const CUtensorMap *m = &p.tmap[2 * w.sb + (is_v ? 1 : 0)];
-                    uint8_t *dst = ring + (size_t)s * kTile;
-                    const int layer = p.layer_begin + w.layer_rel;
-                    mbar_arrive_expect_tx(&full[s], kTile);
-                    tma_load_4d(dst, m, &full[s], 0, w.j * kBN, w.head, layer);
-                    tma_load_4d(dst + kAtom, m, &full[s], 64, w.j * kBN, w.head, layer);
-                    issued = it + 1;
-                    if (++s == S) {
-                        s = 0;
-                        ph ^= 1u;
-                    }
-                    w.advance(p, seqs, t0 + it);
-                }
+            int sb = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
+                const int s = (int)(it % S);
+                const uint32_t ph = (uint32_t)(it / S) & 1u;
+                if (!mbar_wait_bounded(&empty[s], ph ^ 1u, &abort_flag, p.status))
+                    break;
+                const long long t = t0 + it;
+                sb = seq_at<kBatched>(p, t, sb);
+                const TcSeq &sq = seqs[sb];
+                const long long tl = t - sq.tile_base;
+                const int u = (int)(tl / sq.T);
+                const int j = (int)(tl % sq.T);
+                const int head = (u / sq.row_blocks) % p.Hkv;
+                const int layer = p.layer_begin + u / (sq.row_blocks * p.Hkv);
+                const CUtensorMap *m = &p.tmap[2 * sb + (is_v ? 1 : 0)];
+                uint8_t *dst = ring + (size_t)s * kTile;
+                mbar_arrive_expect_tx(&full[s], kTile);
+                tma_load_4d(dst, m, &full[s], 0, j * kBN, head, layer);
+                tma_load_4d(dst + kAtom, m, &full[s], 64, j * kBN, head, layer);
+                issued = it + 1;
             }
             if (issued < n_tiles)
                 for (long long it = (issued > S ? issued - S : 0); it < issued; ++it)
@@ -324,30 +283,25 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // ------------------------------------------------------------ QK^T issuer
         if (lane == 0) {
             const uint32_t idesc_s = idesc_bf16_f32(128, kBN);
-            int sg = -1, s = 0;
-            uint32_t ph = 0;
-            TileWalk<kBatched> w(p, seqs, t0);
-            for (long long it = 0; it < n_tiles; w.advance(p, seqs, t0 + it), ++it) {
-                const bool first = (it == 0) || w.j == 0;
+            int sg = -1, sb = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
+                const long long t = t0 + it;
+                sb = seq_at<kBatched>(p, t, sb);
+                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
                 if (first)
                     ++sg;
+                const int s = (int)(it % kKStages);
                 const int b = (int)(it & 1);
-                const int sk = s;
-                const uint32_t phk = ph;
-                if (++s == kKStages) {
-                    s = 0;
-                    ph ^= 1u;
-                }
                 // K landed; the softmax has read S_b (tile it - 2) and P V(it - 2) has read
                 // the P that shares its columns; at a segment's first tile, its Q is staged
-                if (!mbar_wait_bounded(&k_full[sk], phk, &abort_flag, p.status) ||
+                if (!mbar_wait_bounded(&k_full[s], (uint32_t)(it / kKStages) & 1u, &abort_flag, p.status) ||
                     !mbar_wait_bounded(&s_free[b], ((uint32_t)(it >> 1) & 1u) ^ 1u, &abort_flag, p.status) ||
                     (it >= 2 &&
                      !mbar_wait_bounded(&pv_done[b], (uint32_t)((it - 2) >> 1) & 1u, &abort_flag, p.status)) ||
                     (first && !mbar_wait_bounded(&q_full, (uint32_t)sg & 1u, &abort_flag, p.status)))
                     break;
                 tc_fence_after();
-                const uint32_t k_base = smem_u32(sK + (size_t)sk * kTile);
+                const uint32_t k_base = smem_u32(sK + (size_t)s * kTile);
                 const uint32_t s_col = b ? kColS1 : kColS0;
 #pragma unroll
                 for (int kk = 0; kk < kD / 16; ++kk) {
@@ -356,7 +310,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     tc_mma_f16_ts(tmem + s_col, tmem + kColQ + kk * 8, bdesc, idesc_s, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(&s_full[b]);
-                tc_commit(&k_empty[sk]);
+                tc_commit(&k_empty[s]);
             }
             // arrives when every MMA issued above has retired (waited for before TMEM is released)
             tc_commit(&drain_bar);
@@ -369,35 +323,29 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         // that much sooner.
         if (lane == 0) {
             const uint32_t idesc_pv = idesc_bf16_f32(128, kD, false, true);
-            int sg = -1, s = 0;
-            uint32_t ph = 0;
-            TileWalk<kBatched> w(p, seqs, t0);
-            for (long long it = 0; it < n_tiles; w.advance(p, seqs, t0 + it), ++it) {
-                const bool first = (it == 0) || w.j == 0;
+            int sg = -1, sb = 0;
+            for (long long it = 0; it < n_tiles; ++it) {
+                const long long t = t0 + it;
+                sb = seq_at<kBatched>(p, t, sb);
+                const bool first = (it == 0) || ((t - seqs[sb].tile_base) % seqs[sb].T == 0);
                 if (first)
                     ++sg;
                 const int b = (int)(it & 1);
-                const int sv = s;
-                const uint32_t phv = ph;
-                if (++s == kVStages) {
-                    s = 0;
-                    ph ^= 1u;
-                }
                 // P written; at a segment's first tile, the previous epilogue has read O
                 if (!mbar_wait_bounded(&p_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status) ||
                     (first && sg > 0 &&
                      !mbar_wait_bounded(&o_free, (uint32_t)(sg - 1) & 1u, &abort_flag, p.status)) ||
-                    !mbar_wait_bounded(&v_full[sv], phv, &abort_flag, p.status))
+                    !mbar_wait_bounded(&v_full[it % kVStages], (uint32_t)(it / kVStages) & 1u, &abort_flag, p.status))
                     break;
                 tc_fence_after();
-                const uint32_t v_base = smem_u32(sV + (size_t)sv * kTile);
+                const uint32_t v_base = smem_u32(sV + (size_t)(it % kVStages) * kTile);
                 const uint32_t p_col = b ? kColP1 : kColP0;
 #pragma unroll
                 for (int ks = 0; ks < kBN / 16; ++ks) {
                     const uint64_t bdesc = smem_desc_sw128_mn(v_base + ks * 2048, kAtom, 1024);
                     tc_mma_f16_ts(tmem + kColO, tmem + p_col + ks * 8, bdesc, idesc_pv, (first && ks == 0) ? 0u : 1u);
                 }
-                tc_commit(&v_empty[sv]);
+                tc_commit(&v_empty[it % kVStages]);
                 tc_commit(&pv_done[b]);
             }
             tc_commit(&drain_bar);
@@ -456,12 +404,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             const uint4 *src =
                 reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.ns + g.node) * p.Hq + g.qh) * kD);
             if (!p.rope_tab) {
-#pragma unroll 1
+                // the whole 256-byte row in flight at once, then four TMEM stores
+                uint4 qv[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    qv[i] = g.valid ? src[i] : make_uint4(0, 0, 0, 0);
+#pragma unroll
                 for (int qc = 0; qc < 4; ++qc) {
                     uint32_t w[16];
 #pragma unroll
                     for (int ch = 0; ch < 4; ++ch) {
-                        const uint4 v = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
+                        const uint4 v = qv[qc * 4 + ch];
                         w[4 * ch] = v.x;
                         w[4 * ch + 1] = v.y;
                         w[4 * ch + 2] = v.z;

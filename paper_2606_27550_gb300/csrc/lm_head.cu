@@ -647,16 +647,23 @@ __global__ void __launch_bounds__(kMergeThreads) k2_lm_merge(const __grid_consta
         return;
     if (!in_bounds(r < p.R, p.status))
         return;
-    // pass 1: maximum and its lowest vocab index (empty partials hold -inf)
+    // A thread's slots k = tid + 256 u.  Up to 256 x kInFlight slots (every
+    // vocabulary up to 131072) its partials are loaded once and both passes
+    // read registers; beyond that pass 2 reads them again.
+    const bool held = p.n_slots <= kMergeThreads * kInFlight;
+    float4 v[kInFlight];
+    float2 w[kInFlight];
+    // pass 1: maximum and its lowest vocab index (empty partials hold -inf, s = 0)
     float M = -INFINITY;
     int I = 0x7fffffff;
     for (int k0 = tid; k0 < p.n_slots; k0 += kMergeThreads * kInFlight) {
-        float2 v[kInFlight];
 #pragma unroll
         for (int u = 0; u < kInFlight; ++u) {
             const int k = k0 + u * kMergeThreads;
-            v[u] = k < p.n_slots ? __ldcg(reinterpret_cast<const float2 *>(p.part_tile + (size_t)k * p.R_pad + r))
-                                 : make_float2(-INFINITY, __int_as_float(0x7fffffff));
+            v[u] = k < p.n_slots ? __ldcg(p.part_tile + (size_t)k * p.R_pad + r)
+                                 : make_float4(-INFINITY, __int_as_float(0x7fffffff), 0.f, 0.f);
+            if constexpr (kTyp)
+                w[u] = k < p.n_slots ? __ldcg(p.part_tile_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
         }
 #pragma unroll
         for (int u = 0; u < kInFlight; ++u) {
@@ -682,22 +689,22 @@ __global__ void __launch_bounds__(kMergeThreads) k2_lm_merge(const __grid_consta
     __syncthreads();
     M = s_m[0];
     I = s_i[0];
-    for (int w = 1; w < kWarps; ++w)
-        if (s_m[w] > M || (s_m[w] == M && s_i[w] < I)) {
-            M = s_m[w];
-            I = s_i[w];
+    for (int wp = 1; wp < kWarps; ++wp)
+        if (s_m[wp] > M || (s_m[wp] == M && s_i[wp] < I)) {
+            M = s_m[wp];
+            I = s_i[wp];
         }
     // pass 2: s, t (and the tempered sT, tT) relative to M
     float S = 0.f, T = 0.f, ST = 0.f, TT = 0.f;
     for (int k0 = tid; k0 < p.n_slots; k0 += kMergeThreads * kInFlight) {
-        float4 v[kInFlight];
-        float2 w[kInFlight];
+        if (!held) {
 #pragma unroll
-        for (int u = 0; u < kInFlight; ++u) {
-            const int k = k0 + u * kMergeThreads;
-            v[u] = k < p.n_slots ? __ldcg(p.part_tile + (size_t)k * p.R_pad + r) : make_float4(0.f, 0.f, 0.f, 0.f);
-            if constexpr (kTyp)
-                w[u] = k < p.n_slots ? __ldcg(p.part_tile_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
+            for (int u = 0; u < kInFlight; ++u) {
+                const int k = k0 + u * kMergeThreads;
+                v[u] = k < p.n_slots ? __ldcg(p.part_tile + (size_t)k * p.R_pad + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+                if constexpr (kTyp)
+                    w[u] = k < p.n_slots ? __ldcg(p.part_tile_t + (size_t)k * p.R_pad + r) : make_float2(0.f, 0.f);
+            }
         }
 #pragma unroll
         for (int u = 0; u < kInFlight; ++u) {
@@ -732,11 +739,11 @@ __global__ void __launch_bounds__(kMergeThreads) k2_lm_merge(const __grid_consta
     __syncthreads();
     if (tid == 0) {
         S = T = ST = TT = 0.f;
-        for (int w = 0; w < kWarps; ++w) {
-            S += s_sum[w][0];
-            T += s_sum[w][1];
-            ST += s_sum[w][2];
-            TT += s_sum[w][3];
+        for (int wp = 0; wp < kWarps; ++wp) {
+            S += s_sum[wp][0];
+            T += s_sum[wp][1];
+            ST += s_sum[wp][2];
+            TT += s_sum[wp][3];
         }
         p.argmax[r] = I;
         p.top1[r] = 1.0f / S;
