@@ -73,6 +73,56 @@ struct AcceptBatch {
     AcceptParams seq[TB_MAX_BATCH];
 };
 
+// A warp's registers with the tree of a step: lane l holds nodes l and l + 32
+// (parent, ancestor set, depth, draft token; the tokens of existing nodes only).
+struct TreeRegs {
+    int n;
+    int par[2], dep[2], tok[2];
+    uint64_t anc[2];
+    __device__ __forceinline__ void load(const TreeDesc *t, const int32_t *draft, int lane)
+    {
+        n = t->n;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int i = lane + 32 * h;
+            par[h] = t->parent[i];
+            dep[h] = t->depth[i];
+            anc[h] = t->anc[i];
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int i = lane + 32 * h;
+            tok[h] = i < n && i < kMaxNodes ? draft[i] : 0;
+        }
+    }
+    // the ancestor set of node j (every lane of the warp calls it)
+    __device__ __forceinline__ uint64_t anc_of(int j) const
+    {
+        const uint64_t a0 = __shfl_sync(0xffffffffu, anc[0], j & 31);
+        const uint64_t a1 = __shfl_sync(0xffffffffu, anc[1], j & 31);
+        return j < 32 ? a0 : a1;
+    }
+};
+
+// Asks L2 for the tree's cache rows (positions L + 1 .. L + n - 1) of the
+// (layer, kv head, K|V) units this warp compacts: the copy then reads them
+// from L2.  A prefetch is only a hint; it changes no data.
+__device__ __forceinline__ void prefetch_tree_rows(const AcceptParams &p, int L, int n, int warp, int lane)
+{
+    const int units = p.n_layers * p.n_kv_heads * 2;
+    const int warps_per_cta = blockDim.x >> 5;
+    for (int unit = blockIdx.x * warps_per_cta + warp; unit < units; unit += gridDim.x * warps_per_cta) {
+        const int which = unit & 1;
+        const int lh = unit >> 1;
+        const int head = lh % p.n_kv_heads, layer = lh / p.n_kv_heads;
+        const uint8_t *base = (which ? p.v : p.k) + layer * p.layer_stride_b + head * p.head_stride_b +
+                              (size_t)L * p.row_bytes;
+        for (int j = 1 + lane; j < n && j < kMaxNodes && L + j < p.L_cap; j += 32)
+            for (int off = 0; off < p.row_bytes; off += 128)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(base + (size_t)j * p.row_bytes + off));
+    }
+}
+
 // Per-step tree selection on the device (Sec. 4, "Path-value score" and
 // "Policy"): the feature of the step just verified, then the next rung.
 // Writes the state words rung, L, step, feature (bits), accept_len.
@@ -119,18 +169,31 @@ __device__ void policy_step(const AcceptParams &p, int rung, int L, int len, int
 // blockIdx.y selects the sequence; every CTA of a sequence recomputes its acceptance.
 __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__ AcceptBatch pb)
 {
-    // launched as a programmatic dependent of the step's LM head: its launch
-    // overlaps the LM head's tail, and it reads the LM head's outputs (and the
-    // cache the attention has finished reading) after this wait; the split-unit
-    // merge that follows may then start beside it
-    pdl_wait();
-    pdl_trigger();
     const AcceptParams &p = pb.seq[blockIdx.y];
     __shared__ int s_path[kMaxNodes];
     __shared__ float s_lp[kMaxNodes];
     __shared__ int s_len;
     __shared__ int s_rung, s_L, s_err;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // Launched as a programmatic dependent of the step's LM head, it starts
+    // while the LM head runs.  What no kernel of the step writes -- the tree,
+    // the draft tokens, and the tree's cache rows the compaction may move (the
+    // attention only reads them) -- is fetched before the wait below; the LM
+    // head's statistics, the status word and every cache write come after it,
+    // and so does the trigger that lets the split-unit merge start beside this
+    // kernel.  Scheduled steps and a path from a previous kernel learn their
+    // tree after the wait.
+    TreeRegs tr;
+    const bool early = !p.sched && !p.from_result;
+    if (early) {
+        if (warp == 0)
+            tr.load(p.tree, p.draft, lane);
+        if (p.n_layers > 0)
+            prefetch_tree_rows(p, p.L, p.tree->n, warp, lane);
+    }
+    pdl_wait();
+    pdl_trigger();
 
     const TreeDesc *tree = p.tree;
     const int32_t *draft = p.draft;
@@ -164,23 +227,24 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
         __syncthreads();
     } else {
         if (warp == 0) {
-            const TreeDesc *t = tree;
-            const int n = t->n;
+            if (!early)
+                tr.load(tree, draft, lane);
+            const int n = tr.n;
             uint64_t match = 0;
             bool bad = false;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 const int i = lane + 32 * h;
                 bool m = false;
-                if (i >= 1 && i < n && in_bounds(n <= kMaxNodes && t->parent[i] >= 0 && t->parent[i] < i,
+                if (i >= 1 && i < n && in_bounds(n <= kMaxNodes && tr.par[h] >= 0 && tr.par[h] < i,
                                                  const_cast<int *>(p.ws_status))) {
-                    const int tok = draft[i];
+                    const int tok = tr.tok[h];
                     const bool bad_tok = (tok < 0 || tok >= p.vocab);
                     bad |= bad_tok;
                     if (!p.typical) {
-                        m = (tok == p.argmax[t->parent[i]]);
+                        m = (tok == p.argmax[tr.par[h]]);
                     } else {
-                        const int u = t->parent[i];
+                        const int u = tr.par[h];
                         float lp = -INFINITY;
                         if (!bad_tok) {
                             lp = p.draft_logit[i] * p.inv_t - p.logz_t[u];
@@ -202,9 +266,9 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                 for (int h = 0; h < 2; ++h) {
                     const int i = lane + 32 * h;
                     if (i < n) {
-                        const uint64_t a = t->anc[i];
+                        const uint64_t a = tr.anc[h];
                         if ((a & ~match & ~1ull) == 0ull) {
-                            const int key = t->depth[i] * 128 + (127 - i);
+                            const int key = tr.dep[h] * 128 + (127 - i);
                             best = max(best, key);
                         }
                     }
@@ -225,7 +289,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                     dep[h] = -1;
                     ll[h] = -INFINITY;
                     if (i < n) {
-                        uint64_t a = t->anc[i];
+                        uint64_t a = tr.anc[h];
                         if ((a & ~match & ~1ull) == 0ull) {
                             float acc = 0.f;
                             a &= ~1ull;
@@ -233,7 +297,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                                 acc += s_lp[__ffsll((long long)a) - 1];
                                 a &= a - 1;
                             }
-                            dep[h] = t->depth[i];
+                            dep[h] = tr.dep[h];
                             ll[h] = acc;
                             bdep = max(bdep, dep[h]);
                         }
@@ -260,7 +324,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
                     bid = min(bid, __shfl_xor_sync(0xffffffffu, bid, m));
                 jstar = bid < n ? bid : 0;
             }
-            const uint64_t pa = t->anc[jstar];
+            const uint64_t pa = tr.anc_of(jstar);
             const int len = __popcll(pa);
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
