@@ -269,7 +269,11 @@ def make_result(device="cuda"):
 
 
 def parse_result(res) -> dict:
-    r = [int(x) for x in (res.cpu() if hasattr(res, "cpu") else res)]
+    """The tb_result block (a device or host tensor, or a sequence of ints) as a dict."""
+    if hasattr(res, "cpu"):
+        r = res.cpu().tolist()  # one copy and one conversion (iterating a tensor makes a tensor per element)
+    else:
+        r = [int(x) for x in res]
     k = r[0]
     return {"accept_len": k, "bonus_token": r[1], "new_L": r[2], "status": r[3], "path": r[4:4 + k]}
 
