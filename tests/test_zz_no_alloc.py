@@ -74,12 +74,15 @@ def test_noalloc_matches_workspace_entry_point_and_oracle(built):
             assert np.abs(got[2] - en_ref).max() <= STAT_TOL, f"R={R} V={V}: entropy vs oracle"
 
 
-def test_noalloc_timeout_is_reported_and_next_call_recovers(built):
+@pytest.mark.parametrize("R", [7, 232])
+def test_noalloc_timeout_is_reported_and_next_call_recovers(built, R):
     """A bounded device wait that runs out (the TB_DEBUG_EXPIRE_WAIT test hook:
     the epilogue waits on a barrier nothing arrives on) leaves the outputs
     unwritten and shows only in lm_head_stats_noalloc_status; the next call
-    clears the status word and computes the right result."""
-    R, D, V = 7, 256, 1000
+    clears the status word and computes the right result.  7 rows run the
+    plan of independent CTAs, 232 rows the CTA-pair plan, whose CTAs give up
+    together and drain each other's copies before they exit."""
+    D, V = 256, 1000
     W_h = synth.gen_lm_head(5, V, D)
     h_h, am_ref, t1_ref, en_ref = gap_filtered_hidden(6, R, W_h)
     W, h = _dev(W_h), _dev(h_h)
