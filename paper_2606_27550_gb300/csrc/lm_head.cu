@@ -40,7 +40,6 @@ struct LmParams {
     CUtensorMap tmap_h;  // (d_model, rows),  box (64, R_pad) (R_pad / 2 for CTA pairs), 128B swizzle
     int R, R_pad, D, V;
     int n_tiles, nk, stages, acc_cols;  // tiles of 128 vocab entries (256 for CTA pairs)
-    int P;               // CTAs
     int units;           // the tile split's units: CTAs, or CTA pairs
     int n_slots;         // per-tile partials: one per tile (two per pair tile, one per CTA)
     float4 *part_tile;   // [n_slots][R_pad]  (max, argmax bits, s, t)
@@ -129,22 +128,6 @@ __device__ __forceinline__ RowStat stat_shfl_xor(RowStat a, int mask)
 __device__ __forceinline__ float4 stat_pack(RowStat a)
 {
     return make_float4(a.m, __int_as_float(a.idx), a.s, a.t);
-}
-
-__device__ __forceinline__ RowStat stat_unpack(float4 v)
-{
-    return RowStat{v.x, __float_as_int(v.y), v.z, v.w, 0.f, 0.f};
-}
-
-// Threads per row for the merges of partial statistics by all of the CTA's
-// threads: the largest power of two with tpr x R_pad <= blockDim.x, at most 8
-// (a row's partials are few, so more threads per row would mostly idle).
-__device__ __forceinline__ int threads_per_row(int R_pad)
-{
-    int tpr = 1;
-    while (tpr < 8 && tpr * 2 * R_pad <= (int)blockDim.x)
-        tpr *= 2;
-    return tpr;
 }
 
 // Combines the statistics held by the tpr consecutive lanes of each row group.
@@ -898,7 +881,6 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
     p.nk = pl.n_kblocks;
     p.stages = pl.stages;
     p.acc_cols = pl.acc_cols;
-    p.P = pl.P;
     p.units = pl.units;
     p.n_slots = pl.n_slots;
     p.part_tile = static_cast<float4 *>(parts);
