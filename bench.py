@@ -148,14 +148,6 @@ def kernel_source_hash(files: str) -> str:
     return h.hexdigest()[:16]
 
 
-def launches_per_step(head_dim: int, rope: bool, accept: str) -> int:
-    """Kernels the library launches for one verify step of a multi-tile problem: the LM
-    head and its merge, the attention, the split-unit merge (head_dim 128), acceptance +
-    compaction; + the tree-key rotation (which also writes the rotary table) with rope;
-    sampled acceptance launches the walk, then the compaction."""
-    return (5 if head_dim == 128 else 4) + (1 if rope else 0) + (1 if accept == "sampled" else 0)
-
-
 def acceptance_label(args) -> str:
     if getattr(args, "accept", "greedy") == "typical":
         return "typical (T=0.7, eps=0.09, alpha=0.3)"
@@ -285,10 +277,12 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = tv.tb_launch_count()
     e0.record(stream)
     for i in range(args.steps):
         rstep(args.warmup + i)
     e1.record(stream)
+    n_launch = tv.tb_launch_count() - n0
     torch.cuda.synchronize()
     elapsed_ms = e0.elapsed_time(e1)
     if world > 1:
@@ -399,7 +393,7 @@ def run_gpu(args):
     if rank != 0:
         return
 
-    k1_name = "k1_tree_attention_tc" if d == 128 else "k1_tree_attention"
+    k1_name = "k1_tree_attention_tc"
     peaks, peak_src = load_peaks()
     hbm = float(peaks["hbm_gbs"])
     ms = elapsed_ms / args.steps
@@ -457,7 +451,7 @@ def run_gpu(args):
         "accept_len_last": r["accept_len"],
         "e2e": {"value": round(job_throughput(n_e2e, e2e_s, world), 3), "unit": "verify-steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": launches_per_step(d, args.rope, args.accept) * args.steps,
+        "gpu_launches": n_launch,
         "clocks": clocks,
     }
     if args.layers:
@@ -533,10 +527,13 @@ def run_gpu_batched(args):
     if world > 1:
         dist.barrier()
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    n_launch = 0
     for i in range(args.steps):
         flush.zero_()
         ev[i][0].record(stream)
+        n0 = tv.tb_launch_count()
         step()
+        n_launch += tv.tb_launch_count() - n0
         ev[i][1].record(stream)
     torch.cuda.synchronize()
     elapsed_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in ev), dev)
@@ -565,7 +562,7 @@ def run_gpu_batched(args):
         "roofline": {"bound": "max(hbm, tensor)", "t_mem_ms": round(t_mem, 4), "t_compute_ms": round(t_comp, 4),
                      "frac": round(max(t_mem, t_comp) / ms, 4), "bytes_per_step": kv_bytes + w_bytes,
                      "flops_per_step": flops, "peak_gbs": hbm, "peak_tflops_sustained": tflops, "peak_src": peak_src},
-        "gpu_launches": 5 * args.steps,
+        "gpu_launches": n_launch,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -644,9 +641,11 @@ def run_gpu_bank_loop(args):
                            if os.environ.get("CUDA_VISIBLE_DEVICES") else str(local))
     sampler.start()
     torch.cuda.synchronize()
+    n0 = tv.tb_launch_count()
     t0 = time.perf_counter()
     L_end, _, toks, kv_b, accepted, hist = loop(args.warmup, args.warmup + steps, L, kix)
     el = time.perf_counter() - t0
+    n_launch = tv.tb_launch_count() - n0
     clocks = sampler.stop()
     bank.close()
     if rank != 0:
@@ -666,7 +665,7 @@ def run_gpu_bank_loop(args):
         "tree_histogram": hist,
         "hbm_roofline": {"bytes": kv_b + w_b, "frac": round((kv_b + w_b) / el / 1e9 / hbm, 4), "peak_gbs": hbm,
                          "peak_src": peak_src},
-        "gpu_launches": 5 * steps,
+        "gpu_launches": n_launch,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
@@ -708,9 +707,11 @@ def bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs,
     cs = torch.cuda.Stream()
     cs.wait_stream(stream)
     g = torch.cuda.CUDAGraph()
+    n0 = tv.tb_launch_count()
     with torch.cuda.graph(g, stream=cs):
         for t in range(G):
             sstep(t, cs)
+    per_graph = tv.tb_launch_count() - n0  # kernels in the graph, launched again by every replay
     n_rep = (steps + G - 1) // G
     state.copy_(tv.make_state(0, L0, dev))
     torch.cuda.synchronize()
@@ -741,7 +742,7 @@ def bank_loop_scheduled(args, tv, torch, dev, bank, ids, trees, k, v, W, qs, hs,
                    "L_end": st["L"], "policy": "hysteretic step ladder on the device: up below 1.5, down above 2.5",
                    "host_read_per_step": False, "cuda_graph_steps": G},
         "tau_mean_accept_len": round((st["L"] - L0) / done, 4),
-        "gpu_launches": 5 * done,
+        "gpu_launches": per_graph * n_rep,
         "clocks": clocks,
         "hbm_roofline": {"peak_gbs": float(peaks["hbm_gbs"]), "peak_src": peak_src},
     }
@@ -795,6 +796,7 @@ def run_gpu_sweep(args):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
     rows = []
+    n_launch = 0
     shapes = {"7b-1layer-L2048": (1, 2048), "7b-32layer-L16384": (32, 16384)}
     for sname, (nl, L) in shapes.items():
         H, d, D, V = 32, 128, 4096, 32000
@@ -824,8 +826,10 @@ def run_gpu_sweep(args):
             for i in range(n_steps):
                 flush.zero_()
                 ev[i][0].record(stream)
+                n0 = tv.tb_launch_count()
                 tv.verify_step(bank, ids[j], kv, qn, hid[:n], W, drafts[:n], out, am[:n], t1[:n], en[:n], res, ws,
                                0, stream)
+                n_launch += tv.tb_launch_count() - n0
                 ev[i][1].record(stream)
             torch.cuda.synchronize()
             ms = statistics.median(a.elapsed_time(b) for a, b in ev)
@@ -856,7 +860,7 @@ def run_gpu_sweep(args):
                    "compaction": "included (every step)"},
         "sweep": rows,
         "throughput_optimal_tree": best,
-        "gpu_launches": 5 * max(10, min(args.steps, 100)) * len(rows),
+        "gpu_launches": n_launch,
     }
     print(json.dumps(line), flush=True)
 

@@ -176,6 +176,13 @@ TB_API tb_status tb_workspace_status(const void *workspace, int32_t *status);
 TB_API tb_status tb_debug_bounds_violations(uint32_t *count);
 TB_API int tb_debug_bounds_build(void);
 
+/* Instrumentation (the paper has no counterpart): stores in *count the number
+ * of kernels the library has enqueued in this process so far, counted on the
+ * host as each launch is accepted.  Kernels that a CUDA graph replays are not
+ * counted again: a graph holds the kernels counted while it was captured.
+ * TB_EINVAL if count is NULL; never touches the device. */
+TB_API tb_status tb_launch_count(uint64_t *count);
+
 /* ------------------------------------------------------------------------
  * The verification pass and its stages
  * ---------------------------------------------------------------------- */
@@ -289,8 +296,8 @@ typedef struct tb_seq {
  * reads W once for the whole batch: hidden holds the rows of every sequence,
  * sequence 0 first (sum of N_b rows, at most 1024); argmax / top1 / entropy
  * follow the same row order.  Tree attention of every sequence runs in one
- * launch (head_dim 128) whose work is balanced over the GPU whatever the
- * prefix lengths; acceptance and compaction run in one launch.  `seqs` is a
+ * launch whose work is balanced over the GPU whatever the prefix lengths;
+ * acceptance and compaction run in one launch.  `seqs` is a
  * host array; everything else is as for verify_step. */
 TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_seq *seqs, int n_q_heads,
                                      const void *hidden, const void *lm_head, int d_model, int vocab, int32_t *argmax,
@@ -440,7 +447,7 @@ TB_API tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const tb_
  * live in device memory (tb_state); the acceptance kernel's last CTA updates
  * them after each step, so consecutive verify_step_scheduled calls need no
  * host read in between and a sequence of them can be captured into one CUDA
- * graph.  head_dim 128 only.
+ * graph.
  * ---------------------------------------------------------------------- */
 
 /* Device-resident state (caller-allocated device memory, 4-byte aligned). */

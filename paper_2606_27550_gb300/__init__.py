@@ -37,7 +37,7 @@ API = ("tb_canonicalize", "tb_create", "tb_add_topology", "tb_get_topology", "tb
        "tb_schedule_hysteretic_ladder", "tb_schedule_binary", "tb_schedule_threshold_ladder",
        "lm_head_stats_typical", "typical_accept", "verify_step_typical", "verify_step_batched_typical",
        "verify_step_scheduled", "spec_sample_accept", "verify_step_sampled", "tb_debug_bounds_violations",
-       "tb_debug_bounds_build")
+       "tb_debug_bounds_build", "tb_launch_count")
 
 
 class TreeVerifyError(RuntimeError):
@@ -110,6 +110,7 @@ def load(path: str = LIB_PATH):
         "lm_head_stats_noalloc_status": [P, P],
         "tb_debug_bounds_violations": [P],
         "tb_debug_bounds_build": [],
+        "tb_launch_count": [P],
         "verify_step_batched": [P, i32, P, i32, P, P, i32, i32, P, P, P, P, sz, i32, P],
         "tb_last_error": [],
         "lm_head_stats_typical": [P, i32, P, P, i32, i32, ctypes.c_float, P, P, P, P, P, P, P, P, sz, P],
@@ -334,6 +335,14 @@ def tb_debug_bounds_violations() -> int:
 
 def tb_debug_bounds_build() -> bool:
     return bool(load().tb_debug_bounds_build())
+
+
+def tb_launch_count() -> int:
+    """Kernels the library has enqueued in this process (host-side count; a
+    CUDA graph's replays are not counted again)."""
+    n = ctypes.c_uint64(0)
+    _check(load().tb_launch_count(ctypes.byref(n)), "tb_launch_count")
+    return int(n.value)
 
 
 def lm_head_stats_noalloc_status(stream=None) -> int:

@@ -1,10 +1,10 @@
 // attention_tc.cu -- tree-masked attention on the 5th-generation tensor cores
-// (K1, head_dim 128).
+// (K1, head_dim 64 or 128: one kernel template, kD).
 //
-// Same operation and work split as attention.cu (tree decoding, Sec. 3.2;
-// ancestor-bitset mask, Sec. 2.3; flattened (layer, kv head, row block) x
-// key-tile space split evenly over a persistent grid), with the contractions
-// on tcgen05.  A CTA that covers a whole unit writes its output; a unit split
+// Tree decoding (Sec. 3.2) with the ancestor-bitset mask (Sec. 2.3): the
+// flattened (layer, kv head, row block) x key-tile space is split evenly over
+// a persistent grid, with the contractions on tcgen05.  A CTA that covers a
+// whole unit writes its output; a unit split
 // between CTAs leaves one (O, m, l) partial per CTA, and a second small kernel
 // (k1_merge_split, one warp per query row) combines them by log-sum-exp after
 // the first one has finished (in a verification step, beside the acceptance
@@ -12,16 +12,16 @@
 // output):
 //
 //   S   = Q K^T   tcgen05.mma kind::f16, M = 128 query rows, N = 128 keys,
-//                 K = 128 = head_dim; Q (bf16) is the TMEM A operand, the K
+//                 K = kD = head_dim; Q (bf16) is the TMEM A operand, the K
 //                 tile a 128-byte-swizzled K-major shared-memory operand; S
 //                 accumulates in TMEM.
-//   O  += P V     M = 128 rows, N = 128 = head_dim, K = 128 keys; P (bf16)
+//   O  += P V     M = 128 rows, N = kD, K = 128 keys; P (bf16)
 //                 is the TMEM A operand, the V tile an MN-major shared-memory
 //                 operand; O accumulates in TMEM.
 //
 // One CTA per SM, 8 warps:
 //   warps 0, 7   TMA producers: 128-key K tiles (warp 0) and V tiles (warp 7),
-//                two boxes of 64 x 128 each, through separate 3-stage rings:
+//                kD / 64 boxes of 64 x 128 each, through separate 3-stage rings:
 //                QK^T releases a K slot, P V a V slot, so the next K tiles
 //                never wait for a P V.
 //   warp 1       TMEM allocation (512 columns) and the QK^T-issuing thread;
@@ -35,7 +35,7 @@
 //                TMEM, and the segment epilogue (normalise, or write a partial
 //                for the merge).
 // TMEM columns: S0 [0,128), S1 [128,256) with P0 / P1 aliased onto their first
-// halves, O [256,384), Q [384,448).  Both QK^T and P V take their A operand
+// halves, O [256,256+kD), Q [384,384+kD/2).  Both QK^T and P V take their A operand
 // from TMEM, so each MMA reads only the 128 x 16 B operand from shared memory.
 // Query row r of a block sits in TMEM lane 32*(r%4) + r/4 so that the rows
 // are spread over the four lane quadrants (all four SM sub-partitions share
@@ -48,42 +48,49 @@ namespace tv {
 
 namespace {
 
-constexpr int kD = 128;            // head_dim
 constexpr int kBN = 128;           // keys per tile
 constexpr int kKStages = 3;        // K ring depth
 constexpr int kVStages = 3;        // V ring depth
 constexpr int kMaxStages = kKStages > kVStages ? kKStages : kVStages;
 constexpr int kAtom = 128 * 128;   // one 64-column swizzle atom of a 128-row tile (16 KB)
-constexpr int kTile = 2 * kAtom;   // K or V tile: 128 keys x 128 (32 KB)
 constexpr int kTcThreads = 256;    // 8 warps: K loads, QK^T issuer, 4 softmax, P V issuer, V loads
-constexpr int kSlot = 128 * kD + 256;  // floats per partial slot: O[128][128], m[128], l[128]
+// bytes of a K or V tile (128 keys x head_dim: kD / 64 atoms)
+constexpr int tile_bytes(int d)
+{
+    return d / 64 * kAtom;
+}
+// floats per partial slot: O[128][kD], m[128], l[128]
+constexpr int slot_floats(int d)
+{
+    return 128 * d + 256;
+}
 // TMEM columns.  P_b (bf16 pairs) overwrites the first half of S_b once the
 // softmax has read S_b into registers; Q (bf16 pairs) is the A operand of QK^T.
 constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 0, kColP1 = 128, kColO = 256, kColQ = 384;
 constexpr int kQPrefetchTiles = 3;  // tiles before a segment's end at which the next unit's q rows are prefetched
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
+constexpr int kWholeUnitMaxTiles = 3;  // see attn_tc_plan
 
 // One sequence of a (possibly batched) launch: its own KV cache (tensor maps),
 // prefix length, tree, queries and outputs.  Its tiles occupy
 // [tile_base, tile_base + n_units * T) of the flattened tile space.
 struct TcSeq {
     long long tile_base;
-    const __nv_bfloat16 *q;  // [n_layers][nstride][Hq][128]
+    const __nv_bfloat16 *q;  // [n_layers][nstride][Hq][head_dim]
     __nv_bfloat16 *out;      // same layout
     const TreeDesc *tree;
-    int L, N, rows, row_blocks, T, unit_base;
+    int L, N, rows, row_blocks, T;
     int nstride;             // nodes per layer in q / out (N, or the largest tree of a scheduled loop)
 };
 
 struct TcParams {
-    CUtensorMap tmap[2 * kMaxSeqPerLaunch];  // K, V of each sequence: (128, L + N, Hkv, layers), box (64, 128, 1, 1)
+    CUtensorMap tmap[2 * kMaxSeqPerLaunch];  // K, V of each sequence: (head_dim, L + N, Hkv, layers), box (64, 128, 1, 1)
     TcSeq seq[kMaxSeqPerLaunch];
     int n_seq, Hq, Hkv, group, layer_begin;
     long long total;
     int P;
     float scale_log2;
     float *part;
-    int *counters;
     int *status;
     // scheduled mode (sched != null): the tree and the prefix length come from
     // device memory (sched[0] = rung into rung_tree, sched[1] = L) and every
@@ -92,6 +99,7 @@ struct TcParams {
     const TreeDesc *rung_tree[8];
     int n_rungs, n_layers, L_cap;
     int max_rows;  // query rows of the largest row block (the split merge's grid)
+    int d;         // head_dim: the kernels' kD (host side: picks the instantiation)
     // rotary embedding (null: the queries are already rotated): per sequence a
     // table of (cos, sin) at position L + depth for every pair of head elements
     const float2 *rope_tab;
@@ -104,7 +112,6 @@ __device__ void sched_plan(const TcParams &p, TcSeq *sq, long long *total)
 {
     *sq = p.seq[0];
     sq->tile_base = 0;
-    sq->unit_base = 0;
     const int rung = p.sched[0], L = p.sched[1];
     const bool ok = rung >= 0 && rung < p.n_rungs && L >= 0;
     const TreeDesc *tr = p.rung_tree[ok ? rung : 0];
@@ -175,9 +182,12 @@ __device__ __forceinline__ uint32_t tile_allow(int tj0, uint64_t anc)
     return ((1u << pre) - 1u) | (uint32_t)(anc << pre);
 }
 
-template <bool kBatched>
+template <int kD, bool kBatched>
 __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __grid_constant__ TcParams p)
 {
+    static_assert(kD == 64 || kD == 128, "head_dim 64 or 128");
+    constexpr int kTile = tile_bytes(kD);
+    constexpr int kSlot = slot_floats(kD);
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t k_full[kMaxStages], k_empty[kMaxStages], v_full[kMaxStages], v_empty[kMaxStages];
     __shared__ __align__(8) uint64_t s_full[2], s_free[2], p_full[2], pv_done[2];
@@ -271,8 +281,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                 const CUtensorMap *m = &p.tmap[2 * sb + (is_v ? 1 : 0)];
                 uint8_t *dst = ring + (size_t)s * kTile;
                 mbar_arrive_expect_tx(&full[s], kTile);
-                tma_load_4d(dst, m, &full[s], 0, j * kBN, head, layer);
-                tma_load_4d(dst + kAtom, m, &full[s], 64, j * kBN, head, layer);
+#pragma unroll
+                for (int a = 0; a < kD / 64; ++a)
+                    tma_load_4d(dst + a * kAtom, m, &full[s], 64 * a, j * kBN, head, layer);
                 issued = it + 1;
             }
             if (issued < n_tiles)
@@ -358,7 +369,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 
         struct Seg {
             long long start, end, u_first, u_last;  // flattened tile indices
-            int b, u, ucount, rb, head, layer_rel, rows_here, node, qh, L, N, ns, dep;
+            int b, u, rb, head, layer_rel, rows_here, node, qh, L, N, ns, dep;
             bool valid;
             uint64_t anc;
             const __nv_bfloat16 *q;
@@ -372,7 +383,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             g.b = sb;
             g.start = t;
             g.u = (int)((t - sq.tile_base) / sq.T);
-            g.ucount = sq.unit_base + g.u;
             g.u_first = sq.tile_base + (long long)g.u * sq.T;
             g.u_last = g.u_first + sq.T;
             g.end = t1 < g.u_last ? t1 : g.u_last;
@@ -398,19 +408,19 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
             g.out = sq.out;
             return g;
         };
-        // Q row of this thread -> its TMEM lane as 64 columns of bf16 pairs (the A
-        // operand of QK^T); zeros for padding rows
+        // Q row of this thread -> its TMEM lane as kD / 2 columns of bf16 pairs (the
+        // A operand of QK^T); zeros for padding rows
         auto write_q = [&](const Seg &g) {
             const uint4 *src =
                 reinterpret_cast<const uint4 *>(g.q + (((size_t)g.layer_rel * g.ns + g.node) * p.Hq + g.qh) * kD);
             if (!p.rope_tab) {
-                // the whole 256-byte row in flight at once, then four TMEM stores
-                uint4 qv[16];
+                // the whole row (2 kD bytes) in flight at once, then kD / 32 TMEM stores
+                uint4 qv[kD / 8];
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
+                for (int i = 0; i < kD / 8; ++i)
                     qv[i] = g.valid ? src[i] : make_uint4(0, 0, 0, 0);
 #pragma unroll
-                for (int qc = 0; qc < 4; ++qc) {
+                for (int qc = 0; qc < kD / 32; ++qc) {
                     uint32_t w[16];
 #pragma unroll
                     for (int ch = 0; ch < 4; ++ch) {
@@ -423,16 +433,17 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, w);
                 }
             } else {
-                // pre-rotary query: element i pairs with i + 64, rotated at position
+                // pre-rotary query: element i pairs with i + kD / 2, rotated at position
                 // L + depth(node) with the sequence's (cos, sin) table
+                constexpr int kHalf = kD / 64;  // 32-element chunks per half row
                 const float2 *tab = p.rope_tab + (size_t)g.b * kRopeTableEntries + (size_t)g.dep * kRopeMaxHalf;
 #pragma unroll 1
-                for (int qc = 0; qc < 2; ++qc) {
+                for (int qc = 0; qc < kHalf; ++qc) {
                     uint32_t wl[16], wh[16];
 #pragma unroll
                     for (int ch = 0; ch < 4; ++ch) {
                         const uint4 lo = g.valid ? src[qc * 4 + ch] : make_uint4(0, 0, 0, 0);
-                        const uint4 hi = g.valid ? src[(qc + 2) * 4 + ch] : make_uint4(0, 0, 0, 0);
+                        const uint4 hi = g.valid ? src[(qc + kHalf) * 4 + ch] : make_uint4(0, 0, 0, 0);
                         const uint32_t lw[4] = {lo.x, lo.y, lo.z, lo.w}, hw[4] = {hi.x, hi.y, hi.z, hi.w};
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
@@ -445,7 +456,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                         }
                     }
                     tmem_st_32x32b_x16(lane_addr + kColQ + qc * 16, wl);
-                    tmem_st_32x32b_x16(lane_addr + kColQ + (qc + 2) * 16, wh);
+                    tmem_st_32x32b_x16(lane_addr + kColQ + (qc + kHalf) * 16, wh);
                 }
             }
             tmem_st_wait();
@@ -472,8 +483,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
                     if (nx.valid) {
                         const char *row = reinterpret_cast<const char *>(
                             nx.q + (((size_t)nx.layer_rel * nx.ns + nx.node) * p.Hq + nx.qh) * kD);
-                        asm volatile("prefetch.global.L2 [%0];" ::"l"(row));
-                        asm volatile("prefetch.global.L2 [%0];" ::"l"(row + 128));
+#pragma unroll
+                        for (int off = 0; off < 2 * kD; off += 128)
+                            asm volatile("prefetch.global.L2 [%0];" ::"l"(row + off));
                     }
                 }
                 if (!mbar_wait_bounded(&s_full[b], (uint32_t)(it >> 1) & 1u, &abort_flag, p.status)) {
@@ -662,8 +674,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 // is split exactly when a CTA range starts inside it, so the grid runs over
 // the CTA boundaries c = 1 .. P-1 (x) and groups of 8 query rows (y); the
 // first boundary inside a unit handles it.  One warp per query row, each lane
-// 4 of the 128 output columns, four slots' loads issued together; 32 registers
-// per thread keep every row's warp resident at once.
+// kD / 32 of the kD output columns, four slots' loads issued together; 32
+// registers per thread keep every row's warp resident at once.
 //
 // kAfterStep: launched as a programmatic dependent of a verification step's
 // acceptance kernel.  The attention it merges has completed by then (the
@@ -676,9 +688,33 @@ struct PdlWaitOnExit {
     __device__ ~PdlWaitOnExit() { pdl_wait(); }
 };
 
-template <bool kBatched, bool kAfterStep>
+// kD / 32 consecutive floats of a partial row (one lane's columns)
+template <int kCpl>
+struct ColVec;
+template <>
+struct ColVec<4> {
+    float v[4];
+    __device__ __forceinline__ void load(const float *src)
+    {
+        const float4 x = __ldcg(reinterpret_cast<const float4 *>(src));
+        v[0] = x.x, v[1] = x.y, v[2] = x.z, v[3] = x.w;
+    }
+};
+template <>
+struct ColVec<2> {
+    float v[2];
+    __device__ __forceinline__ void load(const float *src)
+    {
+        const float2 x = __ldcg(reinterpret_cast<const float2 *>(src));
+        v[0] = x.x, v[1] = x.y;
+    }
+};
+
+template <int kD, bool kBatched, bool kAfterStep>
 __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__ TcParams p)
 {
+    constexpr int kSlot = slot_floats(kD);
+    constexpr int kCpl = kD / 32;  // output columns per lane
     if constexpr (!kAfterStep)
         pdl_wait();
     pdl_trigger();
@@ -738,7 +774,7 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
     for (int m = 16; m >= 1; m >>= 1)
         M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, m));
     float lsum = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float acc[kCpl] = {};
     for (int j0 = 0; j0 < nseg; j0 += 32) {
         const int cc = c_lo + j0 + lane;
         const float *sl = p.part;
@@ -749,26 +785,29 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
             w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             lsum += w * __ldcg(sl + 128 * kD + 128 + r);
         }
-        const unsigned long long row_ptr = reinterpret_cast<unsigned long long>(sl + r * kD) + 16ull * lane;
+        const unsigned long long row_ptr = reinterpret_cast<unsigned long long>(sl + r * kD);
         const int cnt = min(32, nseg - j0);
         for (int j1 = 0; j1 < cnt; j1 += 4) {
-            float4 v[4];
+            ColVec<kCpl> v[4];
             float wk[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int src = (j1 + k) & 31;
-                // lane's 16-byte column block of slot j0 + j1 + k
-                const unsigned long long base = __shfl_sync(0xffffffffu, row_ptr - 16ull * lane, src) + 16ull * lane;
+                // lane's column block of slot j0 + j1 + k
+                const unsigned long long base = __shfl_sync(0xffffffffu, row_ptr, src) + 4ull * kCpl * lane;
                 wk[k] = __shfl_sync(0xffffffffu, w, src);
-                v[k] = (j1 + k < cnt) ? __ldcg(reinterpret_cast<const float4 *>(base)) : make_float4(0.f, 0.f, 0.f, 0.f);
+                if (j1 + k < cnt)
+                    v[k].load(reinterpret_cast<const float *>(base));
+                else
+#pragma unroll
+                    for (int x = 0; x < kCpl; ++x)
+                        v[k].v[x] = 0.f;
             }
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                acc.x += wk[k] * v[k].x;
-                acc.y += wk[k] * v[k].y;
-                acc.z += wk[k] * v[k].z;
-                acc.w += wk[k] * v[k].w;
-            }
+            for (int k = 0; k < 4; ++k)
+#pragma unroll
+                for (int x = 0; x < kCpl; ++x)
+                    acc[x] += wk[k] * v[k].v[x];
         }
     }
 #pragma unroll
@@ -778,8 +817,12 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
     const int grow = rb * 128 + r;
     const int node = grow / p.group;
     const int qh = head * p.group + grow % p.group;
-    uint2 *dst = reinterpret_cast<uint2 *>(sq.out + (((size_t)layer_rel * sq.nstride + node) * p.Hq + qh) * kD) + lane;
-    *dst = make_uint2(pack_bf16x2(acc.x * inv, acc.y * inv), pack_bf16x2(acc.z * inv, acc.w * inv));
+    __nv_bfloat16 *orow = sq.out + (((size_t)layer_rel * sq.nstride + node) * p.Hq + qh) * kD;
+    if constexpr (kCpl == 4)
+        reinterpret_cast<uint2 *>(orow)[lane] =
+            make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv), pack_bf16x2(acc[2] * inv, acc[3] * inv));
+    else
+        reinterpret_cast<uint32_t *>(orow)[lane] = pack_bf16x2(acc[0] * inv, acc[1] * inv);
 }
 
 // ----------------------------------------------------------------------------
@@ -787,16 +830,60 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
 
 // The split-unit merge of an attention launch with parameters p (nothing to
 // do when the grid is one CTA).  after_step: see k1_merge_split.
-static cudaError_t merge_launch(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
+template <int kD>
+static cudaError_t merge_launch_d(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
 {
-    if (p.P <= 1)
-        return cudaSuccess;
     const dim3 grid(p.P - 1, (p.max_rows + 7) / 8);
     if (batched)
-        return after_step ? launch_kernel(k1_merge_split<true, true>, grid, dim3(256), 0, stream, pdl, p)
-                          : launch_kernel(k1_merge_split<true, false>, grid, dim3(256), 0, stream, pdl, p);
-    return after_step ? launch_kernel(k1_merge_split<false, true>, grid, dim3(256), 0, stream, pdl, p)
-                      : launch_kernel(k1_merge_split<false, false>, grid, dim3(256), 0, stream, pdl, p);
+        return after_step ? launch_kernel(k1_merge_split<kD, true, true>, grid, dim3(256), 0, stream, pdl, p)
+                          : launch_kernel(k1_merge_split<kD, true, false>, grid, dim3(256), 0, stream, pdl, p);
+    return after_step ? launch_kernel(k1_merge_split<kD, false, true>, grid, dim3(256), 0, stream, pdl, p)
+                      : launch_kernel(k1_merge_split<kD, false, false>, grid, dim3(256), 0, stream, pdl, p);
+}
+
+// Whether a CTA range of the launch starts inside a unit (the split merge then
+// has work).  Scheduled mode plans on the device: assumed so.
+static bool any_split(const TcParams &p)
+{
+    if (p.P <= 1)
+        return false;
+    if (p.sched)
+        return true;
+    int b = 0;
+    for (int c = 1; c < p.P; ++c) {
+        const long long t = (long long)((unsigned long long)c * (unsigned long long)p.total / (unsigned long long)p.P);
+        while (b + 1 < p.n_seq && t >= p.seq[b + 1].tile_base)
+            ++b;
+        if ((t - p.seq[b].tile_base) % p.seq[b].T != 0)
+            return true;
+    }
+    return false;
+}
+
+static cudaError_t merge_launch(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
+{
+    if (!any_split(p))
+        return cudaSuccess;
+    return p.d == 64 ? merge_launch_d<64>(p, batched, stream, pdl, after_step)
+                     : merge_launch_d<128>(p, batched, stream, pdl, after_step);
+}
+
+// The attention kernel for p.d, one CTA per SM (each holds 512 TMEM columns).
+template <int kD, bool kBatched>
+static cudaError_t attn_kernel_launch_d(const TcParams &p, cudaStream_t stream, bool pdl)
+{
+    cudaError_t e;
+    if ((e = allow_max_smem((const void *)k1_tree_attention_tc<kD, kBatched>)) != cudaSuccess)
+        return e;
+    const size_t smem = (size_t)(kKStages + kVStages) * tile_bytes(kD) + 1024;
+    return launch_kernel(k1_tree_attention_tc<kD, kBatched>, dim3(p.P), dim3(kTcThreads), smem, stream, pdl, p);
+}
+
+static cudaError_t attn_kernel_launch(const TcParams &p, bool batched, cudaStream_t stream, bool pdl)
+{
+    if (p.d == 64)
+        return batched ? attn_kernel_launch_d<64, true>(p, stream, pdl) : attn_kernel_launch_d<64, false>(p, stream, pdl);
+    return batched ? attn_kernel_launch_d<128, true>(p, stream, pdl) : attn_kernel_launch_d<128, false>(p, stream, pdl);
 }
 
 // The attention launch's parameters, kept for a split-unit merge enqueued later.
@@ -805,18 +892,12 @@ static void stash_merge(const TcParams &p, bool batched, AttnMerge *m)
     static_assert(sizeof(TcParams) <= sizeof(m->params), "AttnMerge holds the attention launch's parameters");
     memcpy(m->params, &p, sizeof p);
     m->batched = batched;
-    m->pending = p.P > 1;
+    m->pending = any_split(p);
 }
 
-static size_t tc_smem_bytes()
+bool attn_tc_supported(int d)
 {
-    return (size_t)(kKStages + kVStages) * kTile + 1024;
-}
-
-bool attn_tc_supported(int d, int rows)
-{
-    (void)rows;
-    return d == kD;
+    return d == 64 || d == 128;
 }
 
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm)
@@ -831,13 +912,18 @@ AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm)
     long long P = n_sm;
     if (P > pl.total)
         P = pl.total;
+    // A problem of one wave whose units are a few tiles long runs a whole unit
+    // per CTA: a split would save those tiles' serial steps (about 1 us each on
+    // one SM) but add the split merge's launch and round trips.
+    if (pl.total <= n_sm && pl.T <= kWholeUnitMaxTiles)
+        P = pl.n_units;
     pl.P = (int)P;
     return pl;
 }
 
-size_t attn_tc_slot_floats()
+size_t attn_tc_slot_floats(int d)
 {
-    return (size_t)kSlot;
+    return (size_t)slot_floats(d);
 }
 
 int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers)
@@ -849,7 +935,7 @@ int attn_tc_units(const AttnSeq *seqs, int n_seq, int Hq, int Hkv, int n_layers)
 }
 
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
-                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
+                                 int *status, int n_sm, cudaStream_t stream, const char **err,
                                  const float2 *rope_tab, AttnMerge *merge_later)
 {
     if (n_seq < 1 || n_seq > kMaxSeqPerLaunch) {
@@ -858,14 +944,23 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     }
     TcParams p{};
     long long tiles = 0;
-    int units = 0, max_rows = 0;
+    int max_rows = 0;
     const int Hkv = seqs[0].kv->n_kv_heads;
+    const int d = seqs[0].kv->head_dim;
+    if (!attn_tc_supported(d)) {
+        *err = "head_dim 64 or 128";
+        return cudaErrorInvalidValue;
+    }
     for (int b = 0; b < n_seq; ++b) {
         const tb_kv *kv = seqs[b].kv;
+        if (kv->head_dim != d || kv->n_kv_heads != Hkv) {
+            *err = "the sequences of one attention launch share head_dim and kv heads";
+            return cudaErrorInvalidValue;
+        }
         const AttnPlan pl = attn_tc_plan(kv->L, seqs[b].N, Hq, Hkv, n_layers, n_sm);
-        if (!make_tmap_kv(&p.tmap[2 * b], kv->k, kD, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
+        if (!make_tmap_kv(&p.tmap[2 * b], kv->k, d, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
                           kv->head_stride, kv->layer_stride, kBN, err) ||
-            !make_tmap_kv(&p.tmap[2 * b + 1], kv->v, kD, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
+            !make_tmap_kv(&p.tmap[2 * b + 1], kv->v, d, kv->L + seqs[b].N, kv->n_kv_heads, kv->n_layers,
                           kv->head_stride, kv->layer_stride, kBN, err))
             return cudaErrorInvalidValue;
         TcSeq &sq = p.seq[b];
@@ -878,10 +973,8 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
         sq.rows = pl.rows;
         sq.row_blocks = pl.row_blocks;
         sq.T = pl.T;
-        sq.unit_base = units;
         sq.nstride = seqs[b].N;
         tiles += pl.total;
-        units += pl.n_units;
         max_rows = pl.rows < 128 ? (pl.rows > max_rows ? pl.rows : max_rows) : 128;
     }
     p.n_seq = n_seq;
@@ -891,10 +984,13 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     p.layer_begin = layer_begin;
     p.n_layers = n_layers;
     p.total = tiles;
-    p.P = (int)(tiles < n_sm ? tiles : n_sm);
-    p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
+    // one sequence: its plan (whole units for a short one-wave problem); a batch
+    // splits its tiles evenly (units of different lengths)
+    p.P = n_seq == 1 ? attn_tc_plan(seqs[0].kv->L, seqs[0].N, Hq, Hkv, n_layers, n_sm).P
+                     : (int)(tiles < n_sm ? tiles : n_sm);
+    p.d = d;
+    p.scale_log2 = 1.4426950408889634f / sqrtf((float)d);
     p.part = part;
-    p.counters = counters;
     p.status = status;
     p.rope_tab = rope_tab;
     p.max_rows = max_rows;
@@ -905,25 +1001,20 @@ cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin
     // capped beside a longer LM head (merge_later->pdl_launch) is launched as a
     // programmatic dependent and its CTAs wait on SMs that are free already.
     const bool pdl = merge_later && merge_later->pdl_launch;
-    if (batched) {
-        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<true>)) != cudaSuccess)
-            return e;
-        e = launch_kernel(k1_tree_attention_tc<true>, dim3(p.P), dim3(kTcThreads), tc_smem_bytes(), stream, pdl, p);
-    } else {
-        if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
-            return e;
-        e = launch_kernel(k1_tree_attention_tc<false>, dim3(p.P), dim3(kTcThreads), tc_smem_bytes(), stream, pdl, p);
-    }
-    if (e != cudaSuccess)
+    if ((e = attn_kernel_launch(p, batched, stream, pdl)) != cudaSuccess)
         return e;
     if (merge_later) {
         stash_merge(p, batched, merge_later);
         return cudaSuccess;
     }
+    // A plain dependent of the attention: launched as a programmatic one, its
+    // CTAs would take the SMs that attention CTAs release and hold them until
+    // the whole grid is done, away from an LM head beside it on another stream
+    // (measured on GB300: the ragged batch's step 20 us longer).
     return merge_launch(p, batched, stream, false, false);
 }
 
-cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
+cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *status, int n_sm,
                                  cudaStream_t stream, const char **err, AttnMerge *merge_later)
 {
     if (sc.n_rungs < 1 || sc.n_rungs > 8) {
@@ -931,11 +1022,16 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
         return cudaErrorInvalidValue;
     }
     const tb_kv *kv = sc.kv;
+    const int d = kv->head_dim;
+    if (!attn_tc_supported(d)) {
+        *err = "head_dim 64 or 128";
+        return cudaErrorInvalidValue;
+    }
     TcParams p{};
     // the cache's whole capacity: keys past L + N are masked by the kernel
-    if (!make_tmap_kv(&p.tmap[0], kv->k, kD, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+    if (!make_tmap_kv(&p.tmap[0], kv->k, d, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
                       kv->layer_stride, kBN, err) ||
-        !make_tmap_kv(&p.tmap[1], kv->v, kD, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
+        !make_tmap_kv(&p.tmap[1], kv->v, d, kv->L_cap, kv->n_kv_heads, kv->n_layers, kv->head_stride,
                       kv->layer_stride, kBN, err))
         return cudaErrorInvalidValue;
     TcSeq &sq = p.seq[0];
@@ -953,9 +1049,9 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
     p.n_layers = kv->n_layers;
     p.L_cap = kv->L_cap;
     p.P = n_sm;
-    p.scale_log2 = 1.4426950408889634f / sqrtf((float)kD);
+    p.d = d;
+    p.scale_log2 = 1.4426950408889634f / sqrtf((float)d);
     p.part = part;
-    p.counters = counters;
     p.status = status;
     p.sched = sc.sched;
     p.rope_tab = sc.rope_tab;
@@ -964,10 +1060,7 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
         p.rung_tree[r] = sc.rung_tree[r];
     p.max_rows = sc.N_max * p.group < 128 ? sc.N_max * p.group : 128;
     cudaError_t e;
-    if ((e = allow_max_smem((const void *)k1_tree_attention_tc<false>)) != cudaSuccess)
-        return e;
-    k1_tree_attention_tc<false><<<p.P, kTcThreads, tc_smem_bytes(), stream>>>(p);
-    if ((e = cudaGetLastError()) != cudaSuccess)
+    if ((e = attn_kernel_launch(p, false, stream, false)) != cudaSuccess)
         return e;
     if (merge_later) {
         stash_merge(p, false, merge_later);
@@ -977,12 +1070,12 @@ cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *
 }
 
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
-                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                           const void *q, int Hq, void *out, float *part, int *status, int n_sm,
                            cudaStream_t stream, const char **err, const float2 *rope_tab, AttnMerge *merge_later)
 {
     AttnSeq one{kv, d_tree, N, q, out};
-    return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, counters, status, n_sm, stream, err,
-                                rope_tab, merge_later);
+    return attn_tc_launch_batch(&one, 1, layer_begin, n_layers, Hq, part, status, n_sm, stream, err, rope_tab,
+                                merge_later);
 }
 
 cudaError_t attn_merge_launch(const AttnMerge &m, cudaStream_t stream, bool after_step)

@@ -5,6 +5,9 @@
 
 namespace tv {
 
+// Counts one kernel enqueued by the library (tb_launch_count).
+void count_launch();
+
 // Launches `kernel` on `stream` in clusters of `cluster_x` CTAs (1: none);
 // with pdl, with the programmatic-serialization attribute, so that it may be
 // launched while the previous kernel of the stream still runs (the kernel
@@ -34,7 +37,10 @@ cudaError_t launch_kernel_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 bloc
     }
     cfg.attrs = n ? attr : nullptr;
     cfg.numAttrs = n;
-    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+    if (e == cudaSuccess)
+        count_launch();
+    return e;
 }
 
 template <typename... KArgs, typename... Args>
@@ -86,17 +92,6 @@ cudaError_t lm_head_launch(const void *hidden, int R, const void *W, int D, int 
                            float *entropy, void *parts, int *counters, int *status, int n_sm, cudaStream_t stream,
                            const char **err, int expire_wait = 0, const LmTypical *typ = nullptr, bool pdl = false);
 
-// tree attention (attention.cu)
-struct AttnPlan {
-    int group, rows, row_blocks, T, n_units, P;
-    long long total;
-};
-AttnPlan attn_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
-size_t attn_slot_floats(int d);
-cudaError_t attn_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
-                        const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
-                        cudaStream_t stream, const char **err);
-
 // rotary embedding at the tree's position offsets (rope.cu)
 constexpr int kRopeMaxHalf = 64;                                // pairs per head (head_dim <= 128)
 constexpr int kRopeTableEntries = kMaxNodes * kRopeMaxHalf;    // cos / sin per (depth, pair)
@@ -121,9 +116,16 @@ void rope_inv_freq(double theta, int d, double *inv_freq);
 // layers [layer_begin, layer_begin + n_layers)
 cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_layers, cudaStream_t stream);
 
-// tree attention on tcgen05 (attention_tc.cu): head_dim 128, one or several
-// sequences (each with its own cache, prefix length and tree) per launch
+// tree attention on tcgen05 (attention_tc.cu): head_dim 64 or 128, one or
+// several sequences (each with its own cache, prefix length and tree; one
+// head_dim and kv-head count) per launch
 constexpr int kMaxSeqPerLaunch = TB_MAX_BATCH;
+// The work split of one sequence: (layer, kv head, row block) units of T
+// 128-key tiles each, over P persistent CTAs.
+struct AttnPlan {
+    int group, rows, row_blocks, T, n_units, P;
+    long long total;
+};
 struct AttnSeq {
     const tb_kv *kv;
     const TreeDesc *tree;
@@ -147,11 +149,11 @@ cudaError_t attn_merge_launch(const AttnMerge &m, cudaStream_t stream, bool afte
 // pre-rotary and are rotated at L + depth while they are staged
 // merge_later: the split-unit merge is not enqueued but kept there
 cudaError_t attn_tc_launch_batch(const AttnSeq *seqs, int n_seq, int layer_begin, int n_layers, int Hq, float *part,
-                                 int *counters, int *status, int n_sm, cudaStream_t stream, const char **err,
+                                 int *status, int n_sm, cudaStream_t stream, const char **err,
                                  const float2 *rope_tab = nullptr, AttnMerge *merge_later = nullptr);
-bool attn_tc_supported(int d, int rows);
+bool attn_tc_supported(int d);
 AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm);
-size_t attn_tc_slot_floats();
+size_t attn_tc_slot_floats(int d);  // floats per partial slot (two slots per CTA)
 // scheduled mode: the tree (rung_tree[sched[0]]) and L (sched[1]) are read on
 // the device; q / out hold N_max nodes per layer; all kv->n_layers layers
 struct AttnSched {
@@ -163,10 +165,10 @@ struct AttnSched {
     void *out;
     const float2 *rope_tab;  // null, or the rotary tables (pre-rotary queries)
 };
-cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *counters, int *status, int n_sm,
+cudaError_t attn_tc_launch_sched(const AttnSched &sc, int Hq, float *part, int *status, int n_sm,
                                  cudaStream_t stream, const char **err, AttnMerge *merge_later = nullptr);
 cudaError_t attn_tc_launch(const tb_kv *kv, const TreeDesc *d_tree, int N, int layer_begin, int n_layers,
-                           const void *q, int Hq, void *out, float *part, int *counters, int *status, int n_sm,
+                           const void *q, int Hq, void *out, float *part, int *status, int n_sm,
                            cudaStream_t stream, const char **err, const float2 *rope_tab = nullptr,
                            AttnMerge *merge_later = nullptr);
 
@@ -226,7 +228,6 @@ cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream);
 
 // Debug-bounds violation counters of the kernel translation units (0 in a
 // normal build); each call resets the count it returns.
-unsigned int bounds_violations_attention();
 unsigned int bounds_violations_attention_tc();
 unsigned int bounds_violations_lm_head();
 unsigned int bounds_violations_accept();

@@ -106,7 +106,10 @@ cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_lay
     const int n_rows = n_layers * p.Hkv;
     k0_rope_tree_k<<<dim3(max_nodes, (n_rows + kRopeRowsPerCta - 1) / kRopeRowsPerCta, n_seq), kRopeThreads, 0,
                      stream>>>(p, n_rows);
-    return cudaGetLastError();
+    const cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess)
+        count_launch();
+    return e;
 }
 
 TB_BOUNDS_COUNTER(bounds_violations_rope)

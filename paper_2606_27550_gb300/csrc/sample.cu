@@ -521,7 +521,10 @@ cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream)
         k4_spec_sample_cluster<16><<<kWalkCtas, kWalkThreads, 0, stream>>>(p);
     else
         k4_spec_sample<<<1, kSampleThreads, 0, stream>>>(p);
-    return cudaGetLastError();
+    const cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess)
+        count_launch();
+    return e;
 }
 
 TB_BOUNDS_COUNTER(bounds_violations_sample)

@@ -138,8 +138,7 @@ bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_h
 // ------------------------------------------------------------------ workspace layout
 //
 //   [0, 256)                    status word
-//   [256, 256 + 64 KiB)         attention unit counters (16384 int32)
-//   [.., + 4 KiB)               LM-head group counters (1024 int32)
+//   [256, 256 + 4 KiB)          LM-head counters (1024 int32; the tile counter)
 //   [.., + 12 KiB)              typical acceptance: logZ_T, H_T, draft logits (3 x 1024 float)
 //   [.., + 512 KiB)             rotary tables: (cos, sin) per (depth, pair), one per sequence
 //   [kPartBase, ..)             attention partials, then LM-head partials
@@ -147,9 +146,10 @@ bool make_tmap_kv(CUtensorMap *map, const void *base, int d, int n_keys, int n_h
 // workspace always find them zero; partials are written before they are read.
 
 constexpr size_t kTicketOff = 128;  // scheduled acceptance: arrival ticket, inside the status page
-constexpr size_t kAttnCounterOff = 256;
-constexpr int kMaxAttnUnits = 16384;
-constexpr size_t kLmCounterOff = kAttnCounterOff + (size_t)kMaxAttnUnits * 4;
+// (layer, kv head, row block) units of one attention launch: keeps the
+// kernels' 32-bit unit indices in range
+constexpr int kMaxAttnUnits = 1 << 24;
+constexpr size_t kLmCounterOff = 256;
 constexpr int kMaxLmCounters = 1024;
 constexpr int kMaxTypRows = 1024;
 constexpr size_t kTypOff = kLmCounterOff + (size_t)kMaxLmCounters * 4;
@@ -161,19 +161,10 @@ static size_t align256(size_t x)
     return (x + 255) / 256 * 256;
 }
 
-// Partial slots of the split-L merge: two per CTA of the attention kernel
-// that runs (the tcgen05 one for head_dim 128, the mma.sync one for head_dim 64).
+// Partial slots of the split-L merge: two per CTA of the attention kernel.
 static size_t attn_part_bytes(int n_sm, int d)
 {
-    if (attn_tc_supported(d, 0))
-        return align256((size_t)n_sm * 2 * attn_tc_slot_floats() * 4);
-    return align256((size_t)2 * n_sm * 2 * attn_slot_floats(d) * 4);
-}
-
-// head_dim 128 runs on the tcgen05 kernel; head_dim 64 on the mma.sync one.
-static bool use_tc_attention(int d, int rows)
-{
-    return attn_tc_supported(d, rows);
+    return align256((size_t)n_sm * 2 * attn_tc_slot_floats(d) * 4);
 }
 
 static int sm_count(int device)
@@ -544,6 +535,21 @@ extern "C" tb_status tb_workspace_status(const void *workspace, int32_t *status)
     return ok();
 }
 
+static std::atomic<unsigned long long> g_launches{0};
+
+void tv::count_launch()
+{
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+}
+
+extern "C" tb_status tb_launch_count(uint64_t *count)
+{
+    if (!count)
+        return fail(TB_EINVAL, "tb_launch_count: count is NULL");
+    *count = g_launches.load(std::memory_order_relaxed);
+    return ok();
+}
+
 extern "C" tb_status tb_debug_bounds_violations(uint32_t *count)
 {
     if (!count)
@@ -552,8 +558,8 @@ extern "C" tb_status tb_debug_bounds_violations(uint32_t *count)
     if (e != cudaSuccess)
         return cuda_fail(e, "tb_debug_bounds_violations");
     unsigned int n = 0;
-    for (unsigned int (*f)() : {bounds_violations_attention, bounds_violations_attention_tc, bounds_violations_lm_head,
-                                bounds_violations_accept, bounds_violations_rope, bounds_violations_sample}) {
+    for (unsigned int (*f)() : {bounds_violations_attention_tc, bounds_violations_lm_head, bounds_violations_accept,
+                                bounds_violations_rope, bounds_violations_sample}) {
         const unsigned int x = f();
         if (x == 0xffffffffu)
             return fail(TB_ECUDA, "tb_debug_bounds_violations: reading a device counter failed");
@@ -656,9 +662,7 @@ static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan
         return fail(TB_EUNSUPPORTED, "%s: N * group = %d > 256 query rows per kv head", fn,
                     N * (a.Hq / a.kv->n_kv_heads));
     const int nsm = sm_count(a.bank->device);
-    const int rows = N * (a.Hq / a.kv->n_kv_heads);
-    *plan = use_tc_attention(a.kv->head_dim, rows) ? attn_tc_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm)
-                                                   : attn_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
+    *plan = attn_tc_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
     if (plan->n_units > kMaxAttnUnits)
         return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, plan->n_units, kMaxAttnUnits);
     return TB_OK;
@@ -710,7 +714,6 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
 {
     const char *err = "";
     const int N = a.bank->h_desc[a.bank_id].n;
-    const int rows = N * (a.Hq / a.kv->n_kv_heads);
     const bool rope = a.kv->rope_theta != 0.f;
     if (rope) {
         RopeParams rp{};
@@ -726,16 +729,11 @@ static tb_status attn_enqueue(const AttnArgs &a, uint8_t *ws, size_t part_off, c
     }
     AttnMerge *merge_later = ss ? ss->merge_later() : nullptr;
     const int nsm = sm_count(a.bank->device);
-    cudaError_t e;
-    if (use_tc_attention(a.kv->head_dim, rows))
-        e = attn_tc_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
-                           reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                           reinterpret_cast<int *>(ws), a.max_ctas > 0 && a.max_ctas < nsm ? a.max_ctas : nsm, stream,
-                           &err, rope ? rope_table(ws) : nullptr, merge_later);
-    else
-        e = attn_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
-                        reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws + kAttnCounterOff),
-                        reinterpret_cast<int *>(ws), nsm, stream, &err);
+    const cudaError_t e =
+        attn_tc_launch(a.kv, a.bank->d_desc + a.bank_id, N, a.layer_begin, a.n_layers, a.q, a.Hq, a.out,
+                       reinterpret_cast<float *>(ws + part_off), reinterpret_cast<int *>(ws),
+                       a.max_ctas > 0 && a.max_ctas < nsm ? a.max_ctas : nsm, stream, &err,
+                       rope ? rope_table(ws) : nullptr, merge_later);
     if (e == cudaErrorInvalidValue && err[0])
         return fail(TB_EINVAL, "%s: %s", fn, err);
     if (e != cudaSuccess)
@@ -1224,15 +1222,12 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
     if ((st = lm_validate(hidden, chunk, lm_head, d_model, vocab, argmax, top1, entropy, fn, &lplan)) != TB_OK)
         return st;
     const int nsm = sm_count(bank->device);
-    const bool tc = use_tc_attention(kv0.head_dim, 0);
-    if (tc) {
-        AttnSeq as[TB_MAX_BATCH];
-        for (int b = 0; b < batch; ++b)
-            as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
-        const int units = attn_tc_units(as, batch, n_q_heads, kv0.n_kv_heads, kv0.n_layers);
-        if (units > kMaxAttnUnits)
-            return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, units, kMaxAttnUnits);
-    }
+    AttnSeq as[TB_MAX_BATCH];
+    for (int b = 0; b < batch; ++b)
+        as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
+    const int units = attn_tc_units(as, batch, n_q_heads, kv0.n_kv_heads, kv0.n_layers);
+    if (units > kMaxAttnUnits)
+        return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, units, kMaxAttnUnits);
     const size_t attn_bytes = attn_part_bytes(nsm, kv0.head_dim);
     const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
     if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)
@@ -1244,7 +1239,7 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
     cudaError_t e = cudaSuccess;
     StepStreams ss(bank, s, false);  // the batch's attention takes every SM
     // tree attention of every sequence (after the rotary embedding of their tree keys)
-    if (tc) {
+    {
         const bool rope = kv0.rope_theta != 0.f;
         if (rope) {
             RopeParams rp{};
@@ -1258,27 +1253,14 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
         }
         if ((st = ss.before_attention(fn)) != TB_OK)
             return st;
-        AttnSeq as[TB_MAX_BATCH];
-        for (int b = 0; b < batch; ++b)
-            as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
         const char *err = "";
         e = attn_tc_launch_batch(as, batch, 0, kv0.n_layers, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
-                                 reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err, rope ? rope_table(ws) : nullptr, ss.merge_later());
+                                 reinterpret_cast<int *>(ws), nsm, s, &err, rope ? rope_table(ws) : nullptr,
+                                 ss.merge_later());
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)
             return cuda_fail(e, fn);
-    } else {
-        for (int b = 0; b < batch; ++b) {
-            AttnArgs a{bank, seqs[b].bank_id, &seqs[b].kv, 0, kv0.n_layers, seqs[b].q, n_q_heads, seqs[b].attn_out};
-            AttnPlan plan;
-            if ((st = attn_validate(a, fn, &plan)) != TB_OK)
-                return st;
-            // the fork before the first launch
-            if ((st = attn_enqueue(a, ws, kPartBase, s, fn, b == 0 ? &ss : nullptr)) != TB_OK)
-                return st;
-        }
     }
     // LM head over every row of the batch, in chunks of up to 256 rows; in
     // typical mode each chunk gathers the draft logits of the edges whose
@@ -1415,8 +1397,6 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
     kv0.L = 0;  // the prefix length lives in *state
     if ((st = check_kv(&kv0, N_max, fn)) != TB_OK)
         return st;
-    if (kv->head_dim != 128)
-        return fail(TB_EUNSUPPORTED, "%s: head_dim %d (the device-driven loop runs head_dim 128)", fn, kv->head_dim);
     if ((st = check_rope(kv, fn)) != TB_OK)
         return st;
     if (n_q_heads < kv->n_kv_heads || n_q_heads % kv->n_kv_heads)
@@ -1466,8 +1446,7 @@ extern "C" tb_status verify_step_scheduled(const tb_bank *bank, const tb_policy 
             return st;
         const char *err = "";
         cudaError_t e = attn_tc_launch_sched(sc, n_q_heads, reinterpret_cast<float *>(ws + kPartBase),
-                                 reinterpret_cast<int *>(ws + kAttnCounterOff), reinterpret_cast<int *>(ws), nsm, s,
-                                 &err, ss.merge_later());
+                                             reinterpret_cast<int *>(ws), nsm, s, &err, ss.merge_later());
         if (e == cudaErrorInvalidValue && err[0])
             return fail(TB_EINVAL, "%s: %s", fn, err);
         if (e != cudaSuccess)

@@ -100,3 +100,15 @@ def test_no_device_calls_fail_cleanly(lib):
     assert lib.tb_create(ctypes.byref(h), 4, 0) != tv.TB_OK
     assert lib.tb_last_error()
     assert lib.tb_workspace_size(64, 32, 32, 32, 128, 32000, 0) == 0
+
+
+def test_launch_count_is_host_only(lib):
+    """tb_launch_count reads a host counter: callable without a device, and
+    TB_EINVAL for a NULL pointer."""
+    n = ctypes.c_uint64(12345)
+    assert lib.tb_launch_count(ctypes.byref(n)) == tv.TB_OK
+    before = n.value
+    assert lib.tb_launch_count(ctypes.byref(n)) == tv.TB_OK
+    assert n.value == before  # nothing launched in between
+    assert lib.tb_launch_count(None) == tv.TB_EINVAL
+    assert tv.tb_launch_count() == before

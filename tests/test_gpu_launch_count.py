@@ -1,13 +1,14 @@
 """The kernels one verify step launches, counted by the profiler (CUDA activity
-tracing), against the per-step count the benchmark reports (`gpu_launches`):
-greedy, typical, rotary and speculative-sampling steps of a problem that spans
-several attention tiles (so that the split-unit merge runs)."""
+tracing), against the library's own launch counter (tb_launch_count, from which
+the benchmark reports `gpu_launches`) and the step's structure: greedy, typical,
+rotary and speculative-sampling steps of a problem whose attention units span
+several tiles (so that the split-unit merge runs), and a short one that runs a
+whole unit per CTA (no merge)."""
 import re
 
 import numpy as np
 import pytest
 
-import bench
 from helpers import TYPICAL, make_case, softmax_rows, to_dev
 from paper_2606_27550_gb300 import synth
 
@@ -35,12 +36,14 @@ def dev():
     return dev
 
 
-@pytest.mark.parametrize("mode", ["greedy", "typical", "rope", "sampled"])
-def test_launches_per_step(dev, mode):
+@pytest.mark.parametrize("mode,d,L", [("greedy", 128, 600), ("greedy", 64, 600), ("typical", 128, 600),
+                                      ("rope", 128, 600), ("sampled", 128, 600), ("greedy", 64, 100),
+                                      ("greedy", 128, 250)])
+def test_launches_per_step(dev, mode, d, L):
     from torch.profiler import ProfilerActivity, profile
 
     parent = synth.full_tree((2, 2))
-    L, H, d, D, V = 300, 4, 128, 256, 1000
+    H, D, V = 4, 256, 1000
     case = make_case(5, parent, L, 1, H, H, d, D, V, 0.7)
     N = case.N
     b = tv.Bank(4, 0)
@@ -71,7 +74,9 @@ def test_launches_per_step(dev, mode):
     kernels = []
     for _ in range(2):  # a second session if the first one recorded nothing
         with profile(activities=[ProfilerActivity.CUDA]) as prof:
+            n0 = tv.tb_launch_count()
             step()
+            counted = tv.tb_launch_count() - n0
             torch.cuda.synchronize()
         kernels = [e.name for e in prof.events() if e.device_type == torch.autograd.DeviceType.CUDA]
         if kernels:
@@ -79,7 +84,13 @@ def test_launches_per_step(dev, mode):
     if not kernels:
         pytest.skip("CUDA activity tracing recorded nothing on this box")
     ours = [k for k in kernels if OURS.search(k)]
-    want = bench.launches_per_step(d, mode == "rope", "sampled" if mode == "sampled" else "greedy")
+    assert len(ours) == counted, ours
+    # LM head + its row merge, attention, acceptance + compaction; the split-unit
+    # merge when units span more tiles than a one-wave problem runs whole
+    # ((L + N) / 128 > 3 here); + the key rotation; + the sampling walk
+    split = (L + N + 127) // 128 > 3
+    want = 4 + int(split) + int(mode == "rope") + int(mode == "sampled")
     assert len(ours) == want, ours
+    assert any("k1_merge_split" in k for k in ours) == split, ours
     assert tv.parse_result(res)["status"] == 0
     b.close()

@@ -39,16 +39,16 @@ class Loop:
     N_MAX nodes and one draft row per rung (drafts copy the parent's oracle
     greedy token with probability p_match)."""
 
-    def __init__(self, dev, steps, L0, seed=0, p_match=0.7, rungs=tuple(range(len(TREES)))):
+    def __init__(self, dev, steps, L0, seed=0, p_match=0.7, rungs=tuple(range(len(TREES))), d_head=D_HEAD):
         self.dev, self.steps, self.L0 = dev, steps, L0
         self.trees = [TREES[i] for i in rungs]  # the tree of each rung; draft rows follow the rungs
         self.L_cap = L0 + steps * 7 + N_MAX + 8
         self.bank = tv.Bank(16, 0)
         self.ids = [self.bank.add(t)[0] for t in self.trees]
         # every slot holds finite random K/V (the tree slots of each step are read where L lands)
-        self.k, self.v = synth.gen_kv(seed, LAYERS, HKV, self.L_cap, D_HEAD, self.L_cap)
+        self.k, self.v = synth.gen_kv(seed, LAYERS, HKV, self.L_cap, d_head, self.L_cap)
         self.W = synth.gen_lm_head(seed, V, D_MODEL)
-        self.q = [synth.gen_q(seed + 10 + t, LAYERS, N_MAX, HQ, D_HEAD) for t in range(steps)]
+        self.q = [synth.gen_q(seed + 10 + t, LAYERS, N_MAX, HQ, d_head) for t in range(steps)]
         self.h, self.am, self.t1, self.en = [], [], [], []
         self.drafts = []
         for t in range(steps):
@@ -66,12 +66,12 @@ class Loop:
         self.qd = [to_dev(x, dev) for x in self.q]
         self.hd = [to_dev(x, dev) for x in self.h]
         self.dd = [to_dev(x, dev) for x in self.drafts]
-        self.out = torch.empty((LAYERS, N_MAX, HQ, D_HEAD), dtype=torch.bfloat16, device=dev)
+        self.out = torch.empty((LAYERS, N_MAX, HQ, d_head), dtype=torch.bfloat16, device=dev)
         self.g_am = torch.empty(N_MAX, dtype=torch.int32, device=dev)
         self.g_t1 = torch.empty(N_MAX, dtype=torch.float32, device=dev)
         self.g_en = torch.empty(N_MAX, dtype=torch.float32, device=dev)
         self.res = tv.make_result(dev)
-        self.ws = tv.make_workspace(tv.tb_workspace_size(N_MAX, LAYERS, HKV, HQ, D_HEAD, V, 0), dev)
+        self.ws = tv.make_workspace(tv.tb_workspace_size(N_MAX, LAYERS, HKV, HQ, d_head, V, 0), dev)
 
     def kv(self):
         return tv.KvCache(self.kd, self.vd, 0)
@@ -87,9 +87,10 @@ def _trace(steps, seed=3):
     return np.round(g.uniform(0.5, 3.5, steps) * 64).astype(np.float32) / np.float32(64)
 
 
-def test_scheduled_loop_matches_oracle(dev):
+@pytest.mark.parametrize("d_head", [128, 64])
+def test_scheduled_loop_matches_oracle(dev, d_head):
     steps = 24
-    lp = Loop(dev, steps, L0=100)
+    lp = Loop(dev, steps, L0=100, d_head=d_head)
     trace = _trace(steps)
     tr_d = to_dev(trace, dev)
     pol = tv.make_policy(tv.TB_POLICY_HYSTERETIC_LADDER, tv.TB_FEATURE_TRACE, lp.ids, a=1.5, b=2.5, trace=tr_d,
