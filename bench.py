@@ -1005,7 +1005,7 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--rope", action="store_true",
-                    help="c1/c2/c4: pre-rotary inputs, rotary embedding applied by the library (head_dim 128)")
+                    help="c1/c2/c4: pre-rotary inputs, rotary embedding applied by the library")
     ap.add_argument("--scheduled", action="store_true",
                     help="c3 only: the device-driven loop (tree and L on the device, CUDA-graph replay)")
     ap.add_argument("--accept", default="greedy", choices=["greedy", "typical", "sampled"],

@@ -112,7 +112,7 @@ TB_API tb_status tb_destroy(tb_bank *bank);
  * elements and must be multiples of 8; head_dim is 64 or 128.
  *
  * rope_theta = 0: the queries and every key are already rotary-embedded.
- * rope_theta > 0 (head_dim 128): the calls apply the base model's rotary
+ * rope_theta > 0: the calls apply the base model's rotary
  * embedding (Llama convention: frequencies rope_theta^(-2i/d), element i
  * paired with element i + d/2) at the tree's position offsets, node i at
  * position L + depth(i): the queries are passed pre-rotary, and the tree

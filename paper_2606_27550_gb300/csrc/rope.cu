@@ -6,9 +6,9 @@
 // element i + d/2) the step's queries and tree keys are rotated at those
 // positions; the prefix keys were rotated when they entered the cache.
 //
-//   k0_rope_tree_k  one launch: a CTA per (tree node, 64 (layer, kv head)
-//                   rows of it).  Every thread first loads its 8 pairs of
-//                   two rows (16 bytes from each half: the long-context
+//   k0_rope_tree_k  one launch: a CTA per (tree node, 64 or 128 (layer, kv
+//                   head) rows of it).  Every thread first loads its 8 pairs
+//                   of two rows (16 bytes from each half: the long-context
 //                   step's 1024 CTAs are about one wave), then 64 threads form the
 //                   (cos, sin) of (L + depth) * theta_i for the node's depth
 //                   while the loads are in flight: the angle is formed and
@@ -17,7 +17,8 @@
 //                   are written back to the bf16 cache in place.  The first
 //                   node of each depth (canonical order: depths do not
 //                   decrease with the id) also writes its table row to the
-//                   workspace for the query rotation.  head_dim 128.
+//                   workspace for the query rotation.  head_dim 64 or 128
+//                   (template kD: kD / 16 threads per row).
 // The queries are rotated inside the attention kernel as they are staged
 // into tensor memory (attention_tc.cu), with the same table.
 #include <cuda_bf16.h>
@@ -26,12 +27,20 @@
 
 namespace tv {
 
-constexpr int kRopeThreads = 256;                        // 8 threads per 128-wide row
-constexpr int kRopeRowsPerThread = 2;                    // rows r and r + 32, four 16-byte loads in flight
-constexpr int kRopeRowsPerCta = kRopeThreads / 8 * kRopeRowsPerThread;
+constexpr int kRopeThreads = 256;      // kD / 16 threads per row of kD elements
+constexpr int kRopeRowsPerThread = 2;  // two rows a CTA-width apart: four 16-byte loads in flight
 
+constexpr int rope_rows_per_cta(int d)
+{
+    return kRopeThreads / (d / 16) * kRopeRowsPerThread;
+}
+
+template <int kD>
 __global__ void __launch_bounds__(kRopeThreads) k0_rope_tree_k(const __grid_constant__ RopeParams p, int n_rows)
 {
+    static_assert(kD == 64 || kD == 128, "head_dim 64 or 128");
+    constexpr int kTpr = kD / 16;  // threads per row, 8 pairs each
+    constexpr int kRowsPerCta = rope_rows_per_cta(kD);
     __shared__ float2 cs[kRopeMaxHalf];
     const RopeSeq &sq = p.seq[blockIdx.z];
     const TreeDesc *tree = sq.tree;
@@ -47,13 +56,13 @@ __global__ void __launch_bounds__(kRopeThreads) k0_rope_tree_k(const __grid_cons
     if (j >= tree->n)
         return;
     const int dep = tree->depth[j];
-    constexpr int kHalf = 64;  // pairs of a 128-wide row
-    const int ch = (threadIdx.x & 7) * 8;
+    constexpr int kHalf = kD / 2;  // pairs of a row
+    const int ch = (threadIdx.x % kTpr) * 8;
     __nv_bfloat16 *row[kRopeRowsPerThread];
-    uint4 lo[kRopeRowsPerThread], hi[kRopeRowsPerThread];  // elements [ch, ch + 8) and [64 + ch, 64 + ch + 8)
+    uint4 lo[kRopeRowsPerThread], hi[kRopeRowsPerThread];  // elements [ch, ch + 8) and [kHalf + ch, kHalf + ch + 8)
 #pragma unroll
     for (int k = 0; k < kRopeRowsPerThread; ++k) {
-        const int r = blockIdx.y * kRopeRowsPerCta + k * (kRopeThreads / 8) + (threadIdx.x >> 3);
+        const int r = blockIdx.y * kRowsPerCta + k * (kRopeThreads / kTpr) + (int)(threadIdx.x / kTpr);
         row[k] = nullptr;
         lo[k] = hi[k] = make_uint4(0, 0, 0, 0);
         if (r < n_rows && in_bounds((long long)(L + j + 1) * (2 * kHalf) <= sq.head_stride && dep < kMaxNodes, nullptr)) {
@@ -101,11 +110,15 @@ void rope_inv_freq(double theta, int d, double *inv_freq)
 
 cudaError_t rope_launch(const RopeParams &p, int n_seq, int max_nodes, int n_layers, cudaStream_t stream)
 {
-    if (n_seq < 1 || n_seq > TB_MAX_BATCH || p.d != 2 * kRopeMaxHalf || max_nodes < 1 || max_nodes > kMaxNodes)
+    if (n_seq < 1 || n_seq > TB_MAX_BATCH || (p.d != 64 && p.d != 128) || max_nodes < 1 || max_nodes > kMaxNodes)
         return cudaErrorInvalidValue;
     const int n_rows = n_layers * p.Hkv;
-    k0_rope_tree_k<<<dim3(max_nodes, (n_rows + kRopeRowsPerCta - 1) / kRopeRowsPerCta, n_seq), kRopeThreads, 0,
-                     stream>>>(p, n_rows);
+    const int per_cta = rope_rows_per_cta(p.d);
+    const dim3 grid(max_nodes, (n_rows + per_cta - 1) / per_cta, n_seq);
+    if (p.d == 64)
+        k0_rope_tree_k<64><<<grid, kRopeThreads, 0, stream>>>(p, n_rows);
+    else
+        k0_rope_tree_k<128><<<grid, kRopeThreads, 0, stream>>>(p, n_rows);
     const cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess)
         count_launch();

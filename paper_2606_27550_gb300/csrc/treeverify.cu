@@ -674,8 +674,6 @@ static tb_status check_rope(const tb_kv *kv, const char *fn)
         return TB_OK;
     if (!(kv->rope_theta > 0.f) || !std::isfinite(kv->rope_theta))
         return fail(TB_EINVAL, "%s: rope_theta %g (0, or a positive base)", fn, (double)kv->rope_theta);
-    if (kv->head_dim != 128)
-        return fail(TB_EUNSUPPORTED, "%s: the rotary embedding runs with head_dim 128 (got %d)", fn, kv->head_dim);
     return TB_OK;
 }
 
