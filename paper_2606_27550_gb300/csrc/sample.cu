@@ -27,14 +27,15 @@
 // and q_u in registers (loaded once per node), so a rejection costs a block
 // reduction and one cluster barrier.  What the decisions read -- for every
 // non-root node c with parent u, p_u(t_c), q_u(t_c) and unif[c] -- depends on
-// the tree and the drafts only, so rank 0 gathers all of it at the start (one
-// round of dependent loads for the whole walk) and the slices of a node are
-// loaded only when a child of it is rejected or the draw happens there.  The
-// control flow -- the children tried, the decisions, the number of cluster
-// barriers -- depends only on values every CTA copies from rank 0's shared
-// memory and on the cluster sums (the same eight CTA partials added in the
-// same order everywhere), so every CTA takes the same decisions and the same
-// barriers whatever the inputs hold.
+// the tree and the drafts only, so every CTA gathers all of it at the start
+// (one round of dependent loads for the whole walk) and the slices of a node
+// are loaded only when a child of it is rejected or the draw happens there.
+// The control flow -- the children tried, the decisions, the number of
+// cluster barriers -- depends only on those values (the same read-only words,
+// turned into the same numbers by the same instructions in every CTA) and on
+// the cluster sums (the same eight CTA partials added in the same order
+// everywhere), so every CTA takes the same decisions and the same barriers
+// whatever the inputs hold.
 //
 // k4_spec_sample (larger vocabularies): one CTA of 1024 threads; the residual
 // is kept explicitly in the scratch row, one read-modify-write pass per
@@ -277,11 +278,11 @@ __device__ __forceinline__ float ld_dsmem_f32(uint32_t a)
     return v;
 }
 
-__device__ __forceinline__ int ld_dsmem_s32(uint32_t a)
+// Atomic minimum on a 32-bit shared variable of another CTA of the cluster
+// (ordered for the others by the next cluster barrier).
+__device__ __forceinline__ void red_min_dsmem_s32(uint32_t a, int v)
 {
-    int v;
-    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
-    return v;
+    asm volatile("red.relaxed.cluster.shared::cluster.min.s32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
 }
 
 // Sum of x over the cluster.  Every thread of every CTA gets the same bits:
@@ -353,15 +354,11 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
 {
     __shared__ float red[32];
     __shared__ float s_part[2];             // this CTA's partial of the last two cluster sums
-    __shared__ uint64_t s_kids[kMaxNodes];  // rank 0: the children of each node (bitset)
-    __shared__ int s_ok[kMaxNodes];         // rank 0, per non-root node c with parent u: draft token in [0, V),
-    __shared__ float s_pt[kMaxNodes];       // ... p_u(t_c), q_u(t_c) and the uniform deciding c
-    __shared__ float s_qt[kMaxNodes];
-    __shared__ float s_uf[kMaxNodes];
-    __shared__ uint64_t l_kids[kMaxNodes];  // every CTA: its copy of rank 0's records
-    __shared__ int l_ok[kMaxNodes];
-    __shared__ float l_pt[kMaxNodes], l_qt[kMaxNodes], l_uf[kMaxNodes];
-    __shared__ int s_tok;
+    __shared__ uint64_t l_kids[kMaxNodes];  // the children of each node (bitset)
+    __shared__ int l_ok[kMaxNodes];         // per non-root node c with parent u: draft token in [0, V),
+    __shared__ float l_pt[kMaxNodes];       // ... p_u(t_c), q_u(t_c) and the uniform deciding c
+    __shared__ float l_qt[kMaxNodes], l_uf[kMaxNodes];
+    __shared__ int s_tok;                   // rank 0: the drawn token (minimum over the claiming threads)
 
     constexpr float kLog2e = 1.4426950408889634f;
     const float scale = p.inv_t * kLog2e;
@@ -372,34 +369,25 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
     if (!in_bounds(n >= 1 && n <= kMaxNodes, const_cast<int *>(p.ws_status)))
         return;  // the same tree in every CTA: the whole cluster returns before its first barrier
     if (tid < kMaxNodes)
-        s_kids[tid] = 0;
+        l_kids[tid] = 0;
     if (tid == 0)
         s_tok = 0x7fffffff;
     __syncthreads();
-    // rank 0 gathers what every decision of the walk reads: they depend on the
-    // tree and the drafts only, so all of them are loaded at once, up front
-    if (rank == 0 && tid > 0 && tid < n && tid < kMaxNodes) {
+    // every CTA gathers what every decision of the walk reads: they depend on
+    // the tree and the drafts only, so all of them are loaded at once, up front
+    // (no CTA reads another's shared memory before the first cluster barrier)
+    if (tid > 0 && tid < n && tid < kMaxNodes) {
         const int c = tid, pa = t->parent[c];
         if (pa >= 0 && pa < c) {  // canonical order: a parent precedes its children
-            atomicOr(reinterpret_cast<unsigned long long *>(&s_kids[pa]), 1ull << c);
+            atomicOr(reinterpret_cast<unsigned long long *>(&l_kids[pa]), 1ull << c);
             const int tok = p.draft[c];
             const bool ok = tok >= 0 && tok < p.V;
             const float zt = ok ? p.logits[(size_t)pa * p.V + tok] : 0.f;
-            s_ok[c] = ok;
-            s_pt[c] = ok ? ex2_approx(fmaf(zt, scale, -p.logz_t[pa] * kLog2e)) : 0.f;
-            s_qt[c] = ok ? p.q[(size_t)pa * p.V + tok] : 0.f;
-            s_uf[c] = p.unif[c];
+            l_ok[c] = ok;
+            l_pt[c] = ok ? ex2_approx(fmaf(zt, scale, -p.logz_t[pa] * kLog2e)) : 0.f;
+            l_qt[c] = ok ? p.q[(size_t)pa * p.V + tok] : 0.f;
+            l_uf[c] = p.unif[c];
         }
-    }
-    cluster_sync();  // rank 0's records are written
-    if (tid < kMaxNodes) {
-        const uint32_t lo = ld_dsmem_s32(dsmem(&s_kids[tid], 0));
-        const uint32_t hi = ld_dsmem_s32(dsmem(reinterpret_cast<const uint32_t *>(&s_kids[tid]) + 1, 0));
-        l_kids[tid] = (uint64_t)hi << 32 | lo;
-        l_ok[tid] = ld_dsmem_s32(dsmem(&s_ok[tid], 0));
-        l_pt[tid] = ld_dsmem_f32(dsmem(&s_pt[tid], 0));
-        l_qt[tid] = ld_dsmem_f32(dsmem(&s_qt[tid], 0));
-        l_uf[tid] = ld_dsmem_f32(dsmem(&s_uf[tid], 0));
     }
     __syncthreads();
 
@@ -487,13 +475,12 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
                     pick = v0 + j;
             }
         }
-        atomicMin(&s_tok, pick >= 0 ? pick : last);  // rounding can let two neighbouring chunks claim the threshold
+        // into rank 0's s_tok (rounding can let two neighbouring chunks claim the threshold)
+        red_min_dsmem_s32(dsmem(&s_tok, 0), pick >= 0 ? pick : last);
     }
-    cluster_sync();
+    cluster_sync();  // every claim has reached rank 0; no CTA touches another's shared memory after it
     if (rank == 0 && tid == 0) {
-        int tok = 0x7fffffff;
-        for (int r = 0; r < kWalkCtas; ++r)
-            tok = min(tok, ld_dsmem_s32(dsmem(&s_tok, r)));
+        const int tok = s_tok;
         tb_result *res = p.result;
         const uint64_t anc = t->anc[u];
         const int len = __popcll(anc);
@@ -510,7 +497,6 @@ __global__ void __cluster_dims__(kWalkCtas, 1, 1) __launch_bounds__(kWalkThreads
         res->status = (ws & kStatusTimeout) ? TB_ETIMEOUT
                                             : ((bad || (ws & (kStatusBadToken | kStatusBounds))) ? TB_EINVAL : TB_OK);
     }
-    cluster_sync();  // no CTA exits while rank 0 reads its shared memory
 }
 
 cudaError_t sample_launch(const SampleParams &p, cudaStream_t stream)
