@@ -798,6 +798,9 @@ def run_gpu_sweep(args):
     rows = []
     n_launch = 0
     shapes = {"7b-1layer-L2048": (1, 2048), "7b-32layer-L16384": (32, 16384)}
+    visible = os.environ.get("CUDA_VISIBLE_DEVICES")
+    sampler = ClockSampler(visible.split(",")[local] if visible else str(local))
+    sampler.start()
     for sname, (nl, L) in shapes.items():
         H, d, D, V = 32, 128, 4096, 32000
         seed = 99 + nl
@@ -840,6 +843,7 @@ def run_gpu_sweep(args):
                          "expected_accept_len": taus})
         del k, v, W, q, hid, ws
         torch.cuda.empty_cache()
+    clocks = sampler.stop()
     bank.close()
     if rank != 0:
         return
@@ -861,6 +865,7 @@ def run_gpu_sweep(args):
         "sweep": rows,
         "throughput_optimal_tree": best,
         "gpu_launches": n_launch,
+        "clocks": clocks,
     }
     print(json.dumps(line), flush=True)
 

@@ -69,7 +69,7 @@ constexpr int slot_floats(int d)
 constexpr uint32_t kColS0 = 0, kColS1 = 128, kColP0 = 0, kColP1 = 128, kColO = 256, kColQ = 384;
 constexpr int kQPrefetchTiles = 3;  // tiles before a segment's end at which the next unit's q rows are prefetched
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
-constexpr int kWholeUnitMaxTiles = 3;  // see attn_tc_plan
+constexpr int kWholeUnitMaxTiles = 6;  // see attn_tc_plan
 
 // One sequence of a (possibly batched) launch: its own KV cache (tensor maps),
 // prefix length, tree, queries and outputs.  Its tiles occupy
@@ -914,7 +914,8 @@ AttnPlan attn_tc_plan(int L, int N, int Hq, int Hkv, int n_layers, int n_sm)
         P = pl.total;
     // A problem of one wave whose units are a few tiles long runs a whole unit
     // per CTA: a split would save those tiles' serial steps (about 1 us each on
-    // one SM) but add the split merge's launch and round trips.
+    // one SM) but add the split merge's launch and round trips (measured on
+    // GB300: whole units faster up to 5 tiles, even at 6-7).
     if (pl.total <= n_sm && pl.T <= kWholeUnitMaxTiles)
         P = pl.n_units;
     pl.P = (int)P;

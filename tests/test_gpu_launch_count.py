@@ -36,9 +36,9 @@ def dev():
     return dev
 
 
-@pytest.mark.parametrize("mode,d,L", [("greedy", 128, 600), ("greedy", 64, 600), ("typical", 128, 600),
-                                      ("rope", 128, 600), ("sampled", 128, 600), ("greedy", 64, 100),
-                                      ("greedy", 128, 250)])
+@pytest.mark.parametrize("mode,d,L", [("greedy", 128, 1000), ("greedy", 64, 1000), ("typical", 128, 1000),
+                                      ("rope", 128, 1000), ("sampled", 128, 1000), ("greedy", 64, 100),
+                                      ("greedy", 128, 600)])
 def test_launches_per_step(dev, mode, d, L):
     from torch.profiler import ProfilerActivity, profile
 
@@ -87,8 +87,8 @@ def test_launches_per_step(dev, mode, d, L):
     assert len(ours) == counted, ours
     # LM head + its row merge, attention, acceptance + compaction; the split-unit
     # merge when units span more tiles than a one-wave problem runs whole
-    # ((L + N) / 128 > 3 here); + the key rotation; + the sampling walk
-    split = (L + N + 127) // 128 > 3
+    # ((L + N) / 128 > 6 here); + the key rotation; + the sampling walk
+    split = (L + N + 127) // 128 > 6
     want = 4 + int(split) + int(mode == "rope") + int(mode == "sampled")
     assert len(ours) == want, ours
     assert any("k1_merge_split" in k for k in ours) == split, ours

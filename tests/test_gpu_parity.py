@@ -88,6 +88,18 @@ def test_tree_attention_parity(dev, bank, name, parent, L, n_layers, Hq, Hkv, d)
     _run_attention(bank, dev, parent, L, n_layers, Hq, Hkv, d, seed=zlib.crc32(name.encode()) % 1000)
 
 
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("L", [100, 250, 650, 800])
+@pytest.mark.parametrize("parent,Hq,Hkv", [(synth.shape_c2().parent, 8, 2), (synth.bank_trees()[-1], 8, 2)],
+                         ids=["tree26-gqa4", "tree64-gqa4-two-row-blocks"])
+def test_tree_attention_whole_or_split_units(dev, bank, parent, Hq, Hkv, L, d):
+    """Around the plan's whole-unit limit: units of 1-3, 6 and 7 key tiles
+    ((L + N) / 128 rounded up), one or two 128-row blocks, both head widths.
+    Up to six tiles a one-wave problem runs a whole unit per CTA; past that
+    the tiles are split evenly and the split merge combines the pieces."""
+    _run_attention(bank, dev, parent, L, 1, Hq, Hkv, d, seed=L + d + len(parent))
+
+
 def test_tree_attention_non_bfs_input(dev, bank):
     """A topology given in non-breadth-first order is canonicalised; queries and
     tree K/V are then laid out in canonical order (order[c] = caller index)."""
