@@ -227,10 +227,16 @@ TB_API tb_status greedy_accept(const tb_bank *bank, int bank_id, const int32_t *
                         tb_stream stream);
 
 /* KV-cache update after acceptance (Sec. 3.2): for every layer and kv head of
- * kv, slot L + j receives the K and V of slot L + path[j], j < accept_len,
- * read from the device tb_result written by greedy_accept.  In place; all
- * other slots are untouched. */
-TB_API tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream);
+ * kv, slot L + j receives the K and V of slot L + path[j], j < accept_len.
+ * path: device int32 [accept_len], canonical node ids from the root, each at
+ * least its position (path[j] >= j, as every root path of a canonical tree
+ * is); accept_len: device int32, clamped to 1..TB_MAX_NODES; both are read on
+ * the device, so they may come from a kernel earlier on `stream` -- for the
+ * result of greedy_accept: path = result->path, accept_len =
+ * &result->accept_len.  In place; all other slots are untouched, and so is
+ * slot L + j when path[j] <= j or L + path[j] >= L_cap.  TB_EINVAL for a NULL
+ * pointer or a bad kv. */
+TB_API tb_status kv_compact(const tb_kv *kv, const int32_t *path, const int32_t *accept_len, tb_stream stream);
 
 #define TB_NO_COMPACT 1 /* verify_step flag: skip the KV-cache update */
 /* verify_step test hook for failure detection: the LM-head kernel waits on a

@@ -104,7 +104,7 @@ def load(path: str = LIB_PATH):
         "tree_attention": [P, i32, P, i32, i32, P, i32, P, P, sz, P],
         "lm_head_stats": [P, i32, P, i32, i32, P, P, P, P, sz, P],
         "greedy_accept": [P, i32, P, P, i32, i32, P, P],
-        "kv_compact": [P, P, P],
+        "kv_compact": [P, P, P, P],
         "verify_step": [P, i32, P, P, i32, P, P, i32, i32, P, P, P, P, P, P, P, sz, i32, P],
         "lm_head_stats_noalloc": [P, i32, P, i32, i32, P, P, P, i32, P],
         "lm_head_stats_noalloc_status": [P, P],
@@ -303,9 +303,17 @@ def greedy_accept(bank: Bank, bank_id: int, draft, argmax, vocab: int, L: int, r
                                 _stream(stream)), "greedy_accept")
 
 
-def kv_compact(kv: KvCache, result, stream=None):
+def kv_compact_path(kv: KvCache, path, accept_len, stream=None):
+    """KV-cache update from a device path (int32 [accept_len]) and a device
+    accept_len (int32 [1])."""
     c = kv.as_c()
-    _check(load().kv_compact(ctypes.byref(c), _ptr(result), _stream(stream)), "kv_compact")
+    _check(load().kv_compact(ctypes.byref(c), _ptr(path), _ptr(accept_len), _stream(stream)), "kv_compact")
+
+
+def kv_compact(kv: KvCache, result, stream=None):
+    """KV-cache update from a device result block (greedy_accept's): its path
+    and accept_len fields."""
+    kv_compact_path(kv, result[4:], result[:1], stream)
 
 
 def verify_step(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_head, draft, attn_out, argmax, top1, entropy,

@@ -185,7 +185,7 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
     // kernel.  Scheduled steps and a path from a previous kernel learn their
     // tree after the wait.
     TreeRegs tr;
-    const bool early = !p.sched && !p.from_result;
+    const bool early = !p.sched && !p.from_len;
     if (early) {
         if (warp == 0)
             tr.load(p.tree, p.draft, lane);
@@ -219,11 +219,13 @@ __global__ void __launch_bounds__(256) k3_accept_compact(const __grid_constant__
         L = s_L;
     }
 
-    if (p.from_result) {
+    if (p.from_len) {
+        // path entries past accept_len are not read (a caller's array may end there)
+        const int len = min(max(*p.from_len, 1), kMaxNodes);
         if (threadIdx.x < kMaxNodes)
-            s_path[threadIdx.x] = p.result->path[threadIdx.x];
+            s_path[threadIdx.x] = threadIdx.x < len ? p.from_path[threadIdx.x] : (int)threadIdx.x;
         if (threadIdx.x == 0)
-            s_len = min(max(p.result->accept_len, 1), kMaxNodes);
+            s_len = len;
         __syncthreads();
     } else {
         if (warp == 0) {

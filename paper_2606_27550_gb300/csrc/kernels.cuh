@@ -191,7 +191,9 @@ struct AcceptParams {
     long long layer_stride_b, head_stride_b;
     int n_layers, n_kv_heads, row_bytes;
     int L_cap;        // slots per head: copies touching slots >= L_cap are skipped
-    int from_result;  // compaction driven by an existing result (kv_compact): no acceptance
+    // compaction of an existing path (kv_compact, a sampled step): no acceptance;
+    // from_len: device accept_len, from_path: device path[accept_len]
+    const int32_t *from_path, *from_len;
     // scheduled mode (sched != null, one sequence): tree = rung_tree[sched[0]],
     // drafts = draft + sched[0] * n_max, L = sched[1]; the last CTA to finish
     // (arrival ticket) evaluates the feature and the policy and writes the

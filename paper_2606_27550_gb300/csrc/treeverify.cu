@@ -1060,8 +1060,8 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
         return st;
     if (!(flags & TB_NO_COMPACT)) {
         AcceptParams p{};
-        p.result = result;
-        p.from_result = 1;
+        p.from_path = result->path;
+        p.from_len = &result->accept_len;
         add_compaction(p, kv);
         cudaError_t e = accept_launch(p, sm_count(bank->device), s, ss.accept_pdl());
         if (e != cudaSuccess)
@@ -1072,17 +1072,17 @@ extern "C" tb_status verify_step_sampled(const tb_bank *bank, int bank_id, const
     return ok();
 }
 
-extern "C" tb_status kv_compact(const tb_kv *kv, const tb_result *result, tb_stream stream)
+extern "C" tb_status kv_compact(const tb_kv *kv, const int32_t *path, const int32_t *accept_len, tb_stream stream)
 {
     const char *fn = "kv_compact";
     tb_status st = check_kv(kv, 0, fn);
     if (st != TB_OK)
         return st;
-    if (!result)
-        return fail(TB_EINVAL, "%s: result is NULL", fn);
+    if (!path || !accept_len)
+        return fail(TB_EINVAL, "%s: path / accept_len is NULL", fn);
     AcceptParams p{};
-    p.result = const_cast<tb_result *>(result);
-    p.from_result = 1;
+    p.from_path = path;
+    p.from_len = accept_len;
     add_compaction(p, kv);
     cudaError_t e = accept_launch(p, sm_count(current_device()), (cudaStream_t)stream);
     if (e != cudaSuccess)

@@ -226,6 +226,30 @@ def test_kv_compact_vs_oracle(dev, bank):
         assert np.array_equal(bits(vd), oracle.kv_compact(v, L, path))
 
 
+def test_kv_compact_from_path_arrays(dev, bank):
+    """kv_compact from a caller's device path (exactly accept_len entries) and a
+    device accept_len, as the boundary declares it: accepted paths of random
+    drafts, the identity path and the root alone."""
+    g = synth.rng(13)
+    n_layers, H, d, L = 2, 4, 64, 33
+    parent = synth.bank_trees()[-1]
+    N = len(parent)
+    k, v = synth.gen_kv(13, n_layers, H, L + N + 5, d, L + N)
+    paths = []
+    for trial in range(4):
+        draft = g.integers(0, 3, size=N).astype(np.int32)
+        argmax = g.integers(0, 3, size=N).astype(np.int32)
+        paths.append(oracle.accept(parent, draft, argmax)[1])
+    paths += [[0, 1, 2, 3], [0]]
+    for path in paths:
+        kd, vd = to_dev(k, dev), to_dev(v, dev)
+        tv.kv_compact_path(tv.KvCache(kd, vd, L), to_dev(np.asarray(path, np.int32), dev),
+                           to_dev(np.asarray([len(path)], np.int32), dev))
+        torch.cuda.synchronize()
+        assert np.array_equal(bits(kd), oracle.kv_compact(k, L, path)), path
+        assert np.array_equal(bits(vd), oracle.kv_compact(v, L, path)), path
+
+
 def _full_step(dev, bank, case, Hq, Hkv, d, flags=0):
     bid, _ = bank.add(case.parent)
     N, V, D = case.N, case.W.shape[0], case.W.shape[1]
