@@ -80,8 +80,24 @@ static tb_status cuda_fail(cudaError_t e, const char *what)
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static std::once_flag g_encode_once;
 
+// cuTensorMapEncodeTiled is a driver entry point: it needs the device's
+// context current on the calling thread, which the runtime makes so only at
+// the thread's first runtime call that touches the device.  A host thread
+// whose first library call encodes a tensor map before any launch (a
+// verification step run as one chain) would otherwise find none.
+static void ensure_context()
+{
+    static thread_local bool done = false;
+    if (done)
+        return;
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && cudaSetDevice(dev) == cudaSuccess)
+        done = true;
+}
+
 static bool get_encode(const char **err)
 {
+    ensure_context();
     std::call_once(g_encode_once, [] {
         void *fn = nullptr;
         cudaDriverEntryPointQueryResult q;
@@ -952,13 +968,19 @@ extern "C" tb_status typical_accept(const tb_bank *bank, int bank_id, const int3
 // the SMs the LM head's CTAs leave free, and both run from the start.  That
 // pays when the attention on those SMs still ends well before the LM head:
 // about 3 us per 128-key tile a CTA walks plus 6 us, against the weight
-// bytes at 5 TB/s plus 8 us (measured on GB300 at 7B shapes).  0: no cap.
+// bytes at 5 TB/s plus 8 us (measured on GB300 at 7B shapes).  An attention
+// grid that already fits beside the LM head (a small problem) keeps its own
+// size and the step runs as the same chain: both start at once, and the
+// programmatic launches hide the launch latencies (the tiny step: 60-65 k
+// verify-steps/s against 47-57 k with the LM head forked).  0: no cap.
 static int attn_ctas_beside_lm(const AttnPlan &ap, const LmPlan &lp, int d_model, int vocab, int n_sm)
 {
     const int lm_sms = (lp.P + lp.ctas_per_sm - 1) / lp.ctas_per_sm;
     const int free_sms = n_sm - lm_sms;
     if (free_sms < 1 || ap.total < 1)
         return 0;
+    if (ap.P <= free_sms)
+        return ap.P;  // the same split as the uncapped plan (whole units stay whole)
     const double t_attn = 3.0 * (double)((ap.total + free_sms - 1) / free_sms) + 6.0;
     const double t_lm = 2.0 * (double)vocab * (double)d_model / 5.0e6 + 8.0;
     return t_attn < 0.75 * t_lm ? free_sms : 0;

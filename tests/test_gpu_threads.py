@@ -1,12 +1,15 @@
 """Several host threads sharing one TopologyBank, each with its own stream,
 cache, workspace and result block, calling verify_step concurrently.
 
-The bank's helper stream and its fork / join events are shared: a step whose
-LM head is forked onto the helper stream holds the bank's mutex from the fork
-to the join, so the steps of different threads never interleave their
-fork / join sequences.  Every step of every thread must still match the fp64
-oracle exactly (argmax, acceptance, path, bonus) and within the attention
-tolerance, and the compacted caches must equal the oracle's.
+Two step structures: a short attention that fits beside the LM head runs as
+one chain on the caller's stream (each new thread's first call then encodes
+its tensor maps before any other CUDA call of that thread); a longer one
+forks the LM head onto the bank's helper stream, whose fork / join events are
+shared and held under the bank's mutex, so the steps of different threads
+never interleave their fork / join sequences.  Every step of every thread
+must still match the fp64 oracle exactly (argmax, acceptance, path, bonus)
+and within the attention tolerance, and the compacted caches must equal the
+oracle's.
 """
 import threading
 
@@ -33,12 +36,13 @@ def dev():
 
 
 @pytest.mark.parametrize("d", [128, 64])
-def test_threads_share_a_bank(dev, d):
+@pytest.mark.parametrize("structure,Hkv,L", [("chain", 2, 300), ("fork", 8, 3000)])
+def test_threads_share_a_bank(dev, d, structure, Hkv, L):
     trees = [synth.full_tree((2, 2)), synth.bank_trees()[5], synth.bank_trees()[-1]]
     bank = tv.Bank(8, 0)
     ids = [bank.add(t)[0] for t in trees]
     n_threads, steps = 4, 12
-    H, Hkv, D, V, L = 8, 2, 256, 1000, 300
+    H, D, V = 8, 256, 1000
     workers = []
     for w in range(n_threads):
         j = w % len(trees)
