@@ -80,18 +80,19 @@ static tb_status cuda_fail(cudaError_t e, const char *what)
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static std::once_flag g_encode_once;
 
-// cuTensorMapEncodeTiled is a driver entry point: it needs the device's
-// context current on the calling thread, which the runtime makes so only at
-// the thread's first runtime call that touches the device.  A host thread
-// whose first library call encodes a tensor map before any launch (a
-// verification step run as one chain) would otherwise find none.
+// cuTensorMapEncodeTiled is a driver entry point: it needs a context current
+// on the calling thread, which the runtime binds (the device's primary
+// context, unless the caller made another one current) only at the thread's
+// first runtime call that needs one.  A host thread whose first library call
+// encodes a tensor map before any launch (a verification step run as one
+// chain) would otherwise find none.  cudaFree(nullptr) is such a call and
+// does nothing else.
 static void ensure_context()
 {
     static thread_local bool done = false;
     if (done)
         return;
-    int dev = 0;
-    if (cudaGetDevice(&dev) == cudaSuccess && cudaSetDevice(dev) == cudaSuccess)
+    if (cudaFree(nullptr) == cudaSuccess)
         done = true;
 }
 
