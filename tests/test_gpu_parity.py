@@ -80,6 +80,8 @@ ATTN_CASES = [
     ("bank40-gqa4-d64", synth.bank_trees()[6], 190, 1, 8, 2, 64),
     ("bank64-gqa4-L2k", synth.bank_trees()[-1], 2048, 1, 32, 8, 128),
     ("chain2-L0", [-1, 0], 0, 1, 1, 1, 64),
+    ("bank26-gqa8-d64", synth.bank_trees()[5], 700, 1, 16, 2, 64),      # 208 rows per kv head: two row blocks
+    ("bank26-gqa8-d128", synth.bank_trees()[5], 700, 2, 16, 2, 128),
 ]
 
 
@@ -248,6 +250,25 @@ def test_kv_compact_from_path_arrays(dev, bank):
         torch.cuda.synchronize()
         assert np.array_equal(bits(kd), oracle.kv_compact(k, L, path)), path
         assert np.array_equal(bits(vd), oracle.kv_compact(v, L, path)), path
+
+
+def test_kv_compact_skips_invalid_path_entries(dev):
+    """Entries the header declares untouched: path[j] <= j (the copy would go
+    backwards) and a source slot at or past L_cap; the valid entry between
+    them is still applied."""
+    n_layers, H, d, L = 1, 2, 128, 20
+    L_cap = L + 10
+    k, v = synth.gen_kv(14, n_layers, H, L_cap, d, L_cap)
+    path = [0, 0, 5, 1, L_cap - L + 3]
+    kd, vd = to_dev(k, dev), to_dev(v, dev)
+    tv.kv_compact_path(tv.KvCache(kd, vd, L), to_dev(np.asarray(path, np.int32), dev),
+                       to_dev(np.asarray([len(path)], np.int32), dev))
+    torch.cuda.synchronize()
+    want_k, want_v = k.copy(), v.copy()
+    want_k[:, :, L + 2] = k[:, :, L + 5]  # the one valid move: slot L + 2 <- L + 5
+    want_v[:, :, L + 2] = v[:, :, L + 5]
+    assert np.array_equal(bits(kd), want_k)
+    assert np.array_equal(bits(vd), want_v)
 
 
 def _full_step(dev, bank, case, Hq, Hkv, d, flags=0):
