@@ -674,8 +674,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
 // is split exactly when a CTA range starts inside it, so the grid runs over
 // the CTA boundaries c = 1 .. P-1 (x) and groups of 8 query rows (y); the
 // first boundary inside a unit handles it.  One warp per query row, each lane
-// kD / 32 of the kD output columns, four slots' loads issued together; 32
-// registers per thread keep every row's warp resident at once.
+// kD / 32 of the kD output columns, four slots' loads issued together; at most
+// 64 registers per thread (four CTAs of 256 threads per SM).
 //
 // kAfterStep: launched as a programmatic dependent of a verification step's
 // acceptance kernel.  The attention it merges has completed by then (the
@@ -828,8 +828,8 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
 // ----------------------------------------------------------------------------
 // host side
 
-// The split-unit merge of an attention launch with parameters p (nothing to
-// do when the grid is one CTA).  after_step: see k1_merge_split.
+// The split-unit merge of an attention launch with parameters p, for head_dim
+// kD.  after_step: see k1_merge_split.
 template <int kD>
 static cudaError_t merge_launch_d(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
 {
@@ -860,6 +860,7 @@ static bool any_split(const TcParams &p)
     return false;
 }
 
+// The split-unit merge, when the launch split a unit (nothing to do otherwise).
 static cudaError_t merge_launch(const TcParams &p, bool batched, cudaStream_t stream, bool pdl, bool after_step)
 {
     if (!any_split(p))
