@@ -327,10 +327,9 @@ TB_API tb_status verify_step_batched(const tb_bank *bank, int batch, const tb_se
  *    results: calls that can overlap on the GPU (different streams without
  *    ordering) race.
  *  - The scratch is one partial per 128 vocabulary entries for every row
- *    (rows padded to 16, 24 bytes each) plus one per merge group: about
- *    (vocab / 128 + sqrt(vocab / 128)) x 24 x padded rows bytes, 10 MiB at
- *    256 rows and vocab 200000; a call that needs more than 16 MiB is
- *    rejected with TB_ECAPACITY before anything is enqueued.
+ *    (rows padded to 16, 24 bytes each): about vocab / 128 x 24 x padded
+ *    rows bytes, 10 MiB at 256 rows and vocab 200000; a call that needs more
+ *    than 16 MiB is rejected with TB_ECAPACITY before anything is enqueued.
  *  - A bounded device wait that runs out (TB_ETIMEOUT) leaves argmax / top1 /
  *    entropy unwritten and is visible only through
  *    lm_head_stats_noalloc_status.
