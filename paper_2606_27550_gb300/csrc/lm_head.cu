@@ -21,11 +21,10 @@
 // warps 2-9 drain the other accumulator meanwhile (32 tree rows at a time:
 // TMEM -> shared memory transposed -> eight threads per row reduce its 128
 // logits) into the tile's per-row statistics, written to the tile's own slot.
-// The slots are merged in two levels by atomic arrival tickets over fixed
-// groups of slots (the CTA whose tile completes a group merges it; the one
-// that completes the last group merges the groups), always in slot order, so
-// the results do not depend on which CTA took which tile; no CTA ever waits
-// for another.
+// A second kernel, k2_lm_merge (one CTA per row, launched as a programmatic
+// dependent that waits for the whole grid), merges every row's slots in slot
+// order, so the results do not depend on which CTA took which tile; no CTA of
+// the LM head ever waits for another.
 //
 #include <atomic>
 #include <math.h>

@@ -14,9 +14,9 @@
 namespace tv {
 
 // 16 MiB of partials.  The plan needs one partial per 128 vocabulary entries
-// (two per 256-entry tile of a CTA pair) and one per merge group for every row
-// (rows padded to 16, 24 bytes each): 10 MiB at 256 rows and vocab 200000,
-// 16 MiB up to a vocabulary of about 330 000.
+// (two per 256-entry tile of a CTA pair) for every row (rows padded to 16, 24
+// bytes each): 10 MiB at 256 rows and vocab 200000, 16 MiB up to a vocabulary
+// of about 330 000.
 constexpr size_t kNoAllocScratchBytes = 16u << 20;
 constexpr size_t kNoAllocCounterBytes = 4096;  // 1024 counters, cleared on every call
 constexpr int kNoAllocStatusWord = kNoAllocCounterBytes / 4 - 1;  // last counter word: device-detected errors
