@@ -15,7 +15,8 @@
 // j < accept_len, in every layer and kv head.  path[j] >= j and path is
 // increasing, so copying rows in increasing j never reads a row that an
 // earlier copy overwrote; one warp copies one (layer, head, K|V) row set in
-// that order, with a warp barrier between rows.
+// that order, in chunks of eight rows (each chunk loads all of its source
+// rows, then stores them; a warp barrier between chunks).
 //
 // Typical acceptance (the Medusa/Hydra rule the paper keeps, Sec. 5.1/5.2):
 // edge j passes when p_T(draft[j] | parent) > min(eps, alpha e^(-H_T(parent))),
