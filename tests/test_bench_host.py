@@ -1,5 +1,6 @@
 """Host-side logic of bench.py: the expected accept length of the synthetic
-draft model, checked against exhaustive enumeration of match patterns."""
+draft model, checked against exhaustive enumeration of match patterns, and
+the rule that ties a committed ncu traffic record to the kernel sources."""
 import itertools
 import os
 import sys
@@ -41,3 +42,39 @@ def test_expected_accept_len_limits():
         assert bench.expected_accept_len(t, 1.0) == synth.depth_of(t).max() + 1
     # a chain: 1 + p + p^2 + ... + p^D
     assert bench.expected_accept_len(synth.chain(5), 0.5) == pytest.approx(1 + 0.5 + 0.25 + 0.125 + 0.0625)
+
+
+def _profiles_tree(tmp_path, records):
+    """A copy of the kernel sources and a traffic file with the given records."""
+    import shutil
+
+    src = os.path.join(bench.ROOT, "paper_2606_27550_gb300", "csrc")
+    dst = tmp_path / "paper_2606_27550_gb300" / "csrc"
+    shutil.copytree(src, dst)
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "traffic.txt").write_text("# kernel files hash bytes [workload]\n" + records)
+    return dst
+
+
+def test_traffic_record_follows_the_kernel_sources(tmp_path, monkeypatch):
+    """The bench reports a kernel's DRAM traffic from a committed ncu record only
+    while the record's source hash matches the sources; an edit to any of them
+    turns it into null, and a record for another workload does not apply."""
+    files = "attention_tc.cu,common.cuh,kernels.cuh"
+    dst = _profiles_tree(tmp_path, "")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h = bench.kernel_source_hash(files)
+    assert len(h) == 16
+    (tmp_path / "profiles" / "traffic.txt").write_text(
+        f"k1_tree_attention_tc {files} {h} 12345\n"
+        f"k2_lm_head lm_head.cu,common.cuh,kernels.cuh {bench.kernel_source_hash('lm_head.cu,common.cuh,kernels.cuh')}"
+        " 678 some-workload\n")
+    assert bench.traffic_from_profiles("k1_tree_attention_tc") == 12345
+    assert bench.traffic_from_profiles("k2_lm_head", "some-workload") == 678
+    assert bench.traffic_from_profiles("k2_lm_head", "another-workload") is None
+    assert bench.traffic_from_profiles("k3_accept_compact") is None
+    with open(dst / "common.cuh", "a") as f:
+        f.write("\n// edited\n")
+    assert bench.traffic_from_profiles("k1_tree_attention_tc") is None
+    assert bench.traffic_from_profiles("k2_lm_head", "some-workload") is None
+
