@@ -13,7 +13,12 @@ attention of the same row over |V|, computed by the oracle), the error of an
 element is bounded by 2^-8 |O| + 2^-8 A, plus 2^-12 A for every fp32 step
 (scores, exponentials, accumulation, split merge), which are orders of
 magnitude smaller.  An element may exceed 1e-2 only where that bound does;
-the test reports how many elements need it."""
+the test reports how many elements need it.  The mean-abs bar likewise: the
+rounding of an fp32 value to bf16 averages about half of its 2^-8 bound, so
+rows whose outputs are of order 1 (prefixes of a few keys) cannot average
+below 1e-3 (rounding the oracle's own fp64 result to bf16 already gives
+0.8-1.0e-3 there); the mean may exceed 1e-3 only up to half the mean of the
+per-element bound."""
 import numpy as np
 import pytest
 
@@ -47,14 +52,18 @@ def check_attention_fuzz(got, ref, ref_abs_v, what):
     got = got.astype(np.float64)
     assert np.all(np.isfinite(got)), f"{what}: non-finite output"
     err = np.abs(got - ref)
-    bound = np.maximum(1e-2, attention_bound(ref, ref_abs_v))
+    elem = attention_bound(ref, ref_abs_v)
+    bound = np.maximum(1e-2, elem)
     worst = np.argmax(err - bound)
     n_over = int((err > 1e-2).sum())
     if n_over:
         print(f"{what}: {n_over} of {err.size} elements beyond 1e-2, within the derived bound")
     assert (err <= bound).all(), (f"{what}: |err| {err.flat[worst]:.3e} at |ref| {abs(ref.flat[worst]):.3f}, "
                                   f"bound {bound.flat[worst]:.3e}")
-    assert err.mean() <= 1e-3, f"{what}: mean |err| {err.mean():.3e}"
+    mean_bound = max(1e-3, 0.5 * float(elem.mean()))
+    if err.mean() > 1e-3:
+        print(f"{what}: mean |err| {err.mean():.3e} beyond 1e-3, within the derived {mean_bound:.3e}")
+    assert err.mean() <= mean_bound, f"{what}: mean |err| {err.mean():.3e} > {mean_bound:.3e}"
 
 
 def abs_bits(a):
@@ -66,7 +75,7 @@ def _hidden(g, n, W, gap_min=1e-2):
     """n hidden rows with a clear top-2 gap (V = 1 has a single token: no gap to keep)."""
     D, V = W.shape[1], W.shape[0]
     for _ in range(20):
-        pool = synth.normal_bf16(g, (n + 16, D))
+        pool = synth.normal_bf16(g, (2 * n + 64, D))
         am, t1, en, gap = oracle.lm_head(pool, W)
         keep = np.arange(len(gap)) if V == 1 else np.nonzero(gap > gap_min)[0]
         if len(keep) >= n:
@@ -138,7 +147,7 @@ def test_random_verify_step(dev, seed):
 @pytest.mark.parametrize("seed", range(12))
 def test_random_batched_step(dev, seed):
     g = synth.rng(9500 + seed)
-    d, Hkv = 128, int(g.choice([1, 2, 4]))
+    d, Hkv = (64 if seed % 3 == 2 else 128), int(g.choice([1, 2, 4]))
     group = int(g.choice([1, 2, 4]))
     Hq = Hkv * group
     D, V = int(g.choice([64, 256, 520])), int(g.choice([129, 1000, 3001]))
