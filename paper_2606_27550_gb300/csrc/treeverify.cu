@@ -678,10 +678,11 @@ static tb_status attn_validate(const AttnArgs &a, const char *fn, AttnPlan *plan
     if (N * (a.Hq / a.kv->n_kv_heads) > 256)
         return fail(TB_EUNSUPPORTED, "%s: N * group = %d > 256 query rows per kv head", fn,
                     N * (a.Hq / a.kv->n_kv_heads));
+    const long long units = (long long)a.n_layers * a.kv->n_kv_heads * ((N * (a.Hq / a.kv->n_kv_heads) + 127) / 128);
+    if (units > kMaxAttnUnits)
+        return fail(TB_EUNSUPPORTED, "%s: %lld attention units > %d", fn, units, kMaxAttnUnits);
     const int nsm = sm_count(a.bank->device);
     *plan = attn_tc_plan(a.kv->L, N, a.Hq, a.kv->n_kv_heads, a.n_layers, nsm);
-    if (plan->n_units > kMaxAttnUnits)
-        return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, plan->n_units, kMaxAttnUnits);
     return TB_OK;
 }
 
@@ -1244,11 +1245,13 @@ static tb_status verify_step_batched_impl(const tb_bank *bank, int batch, const 
         return st;
     const int nsm = sm_count(bank->device);
     AttnSeq as[TB_MAX_BATCH];
-    for (int b = 0; b < batch; ++b)
+    long long units = 0;  // counted wide first: the plan's counts are 32-bit
+    for (int b = 0; b < batch; ++b) {
         as[b] = AttnSeq{&seqs[b].kv, bank->d_desc + seqs[b].bank_id, Ns[b], seqs[b].q, seqs[b].attn_out};
-    const int units = attn_tc_units(as, batch, n_q_heads, kv0.n_kv_heads, kv0.n_layers);
-    if (units > kMaxAttnUnits)
-        return fail(TB_EUNSUPPORTED, "%s: %d attention units > %d", fn, units, kMaxAttnUnits);
+        units += (long long)kv0.n_layers * kv0.n_kv_heads * ((Ns[b] * group + 127) / 128);
+    }
+    if (units > kMaxAttnUnits || attn_tc_units(as, batch, n_q_heads, kv0.n_kv_heads, kv0.n_layers) != units)
+        return fail(TB_EUNSUPPORTED, "%s: %lld attention units > %d", fn, units, kMaxAttnUnits);
     const size_t attn_bytes = attn_part_bytes(nsm, kv0.head_dim);
     const size_t need = kPartBase + attn_bytes + lplan.ws_bytes;
     if ((st = check_ws(workspace, workspace_bytes, need, fn)) != TB_OK)

@@ -252,6 +252,23 @@ def test_kv_compact_from_path_arrays(dev, bank):
         assert np.array_equal(bits(vd), oracle.kv_compact(v, L, path)), path
 
 
+def test_attention_units_counted_without_overflow(dev, bank):
+    """A cache whose layer x kv-head count is far beyond any real one (2^30
+    units, past the 32-bit counts of the plan) is refused before anything is
+    enqueued."""
+    import ctypes
+
+    bid, _ = bank.add([-1, 0])
+    k = torch.zeros((1, 1, 64, 128), dtype=torch.bfloat16, device=dev)
+    c = tv.TbKv(k.data_ptr(), k.data_ptr(), (1 << 10) * 64 * 128, 64 * 128, 1 << 20, 1 << 10, 128, 0, 64, 0.0)
+    q = torch.zeros((1, 2, 1024, 128), dtype=torch.bfloat16, device=dev)
+    ws = tv.make_workspace(1 << 20, dev)
+    st = tv.load().tree_attention(bank.handle, bid, ctypes.byref(c), 0, 1 << 20, q.data_ptr(), 1024, q.data_ptr(),
+                                  ws.data_ptr(), ws.numel(), None)
+    assert st == tv.TB_EUNSUPPORTED
+    assert b"attention units" in tv.load().tb_last_error()
+
+
 def test_kv_compact_skips_invalid_path_entries(dev):
     """Entries the header declares untouched: path[j] <= j (the copy would go
     backwards) and a source slot at or past L_cap; the valid entry between
