@@ -86,6 +86,36 @@ def check_attention(got: np.ndarray, ref: np.ndarray, what: str = "attention"):
     return float(err.max()), float(err.mean())
 
 
+def attention_bound(ref, ref_abs_v):
+    """Per-element error bound of the kernels' attention: bf16 output and bf16
+    probabilities in P V (2^-8 each), and 2^-12 A for the fp32 steps."""
+    return 2.0 ** -8 * np.abs(ref) + (2.0 ** -8 + 2.0 ** -12) * ref_abs_v
+
+
+def check_attention_fuzz(got, ref, ref_abs_v, what):
+    """got vs the oracle's ref, with ref_abs_v the oracle's attention over |V|."""
+    got = got.astype(np.float64)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    err = np.abs(got - ref)
+    elem = attention_bound(ref, ref_abs_v)
+    bound = np.maximum(1e-2, elem)
+    worst = np.argmax(err - bound)
+    n_over = int((err > 1e-2).sum())
+    if n_over:
+        print(f"{what}: {n_over} of {err.size} elements beyond 1e-2, within the derived bound")
+    assert (err <= bound).all(), (f"{what}: |err| {err.flat[worst]:.3e} at |ref| {abs(ref.flat[worst]):.3f}, "
+                                  f"bound {bound.flat[worst]:.3e}")
+    mean_bound = max(1e-3, 0.5 * float(elem.mean()))
+    if err.mean() > 1e-3:
+        print(f"{what}: mean |err| {err.mean():.3e} beyond 1e-3, within the derived {mean_bound:.3e}")
+    assert err.mean() <= mean_bound, f"{what}: mean |err| {err.mean():.3e} > {mean_bound:.3e}"
+
+
+def abs_bits(a):
+    """|x| of bf16 bit patterns (sign bit cleared)."""
+    return (a & np.uint16(0x7FFF)).astype(np.uint16)
+
+
 # typical acceptance: the paper's settings (temperature, posterior threshold, mixing coefficient)
 TYPICAL = (0.7, 0.09, 0.3)
 MARGIN_MIN = 1e-3  # |p - threshold| / threshold of every edge, so fp32 and fp64 decide alike

@@ -11,8 +11,8 @@ import numpy as np
 import pytest
 
 import oracle
-from helpers import (LOGIT_TOL, STAT_TOL, TYPICAL, bits, check_attention, gap_filtered_hidden, to_dev,
-                     typical_ambiguity, typical_drafts)
+from helpers import (LOGIT_TOL, STAT_TOL, TYPICAL, abs_bits, bits, check_attention, check_attention_fuzz,
+                     gap_filtered_hidden, to_dev, typical_ambiguity, typical_drafts)
 from paper_2606_27550_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -322,4 +322,52 @@ def test_batched_typical_many_edges_in_one_vocab_tile(dev):
         r = tv.parse_result(s.result)
         ka, path, bonus = oracle.typical_accept(parent, drafts, lg, *TYPICAL)
         assert (r["accept_len"], r["path"], r["bonus_token"]) == (ka, path, bonus)
+    b.close()
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_random_typical_step(dev, seed):
+    """Random shapes through verify_step_typical: random trees, prefix lengths
+    0-2000, head_dim 64 and 128, GQA groups, one or two layers, vocabularies
+    with ragged last tiles; attention within the derived bound of the fuzz
+    tests, statistics, acceptance and compaction against the oracle."""
+    g = synth.rng(7700 + seed)
+    n = int(g.integers(1, 65))
+    parent = np.sort(synth.random_tree(g, n))
+    parent[0] = -1
+    d = int(g.choice([64, 128]))
+    Hkv = int(g.choice([1, 2, 4]))
+    group = int(g.choice([1, 2, 4]))
+    while n * group > 256:
+        group //= 2
+    Hq = Hkv * group
+    L = int(g.choice([0, 5, 130, 700, 2000]))
+    D = int(g.choice([64, 256]))
+    V = int(g.choice([129, 1000, 3001]))
+    layers = int(g.integers(1, 3))
+    c = _typical_case(500 + seed, parent, L, layers, Hq, Hkv, d, D, V)
+    b = tv.Bank(4, 0)
+    bid, _ = b.add(c["parent"])
+    kd, vd = to_dev(c["k"], dev), to_dev(c["v"], dev)
+    out = torch.empty((layers, n, Hq, d), dtype=torch.bfloat16, device=dev)
+    g_am = torch.empty(n, dtype=torch.int32, device=dev)
+    g_t1, g_en = _f32(n, dev), _f32(n, dev)
+    res = tv.make_result(dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(n, layers, Hkv, Hq, d, V, 0), dev)
+    tv.verify_step_typical(b, bid, tv.KvCache(kd, vd, L), to_dev(c["q"], dev), to_dev(c["hidden"], dev),
+                           to_dev(c["W"], dev), to_dev(c["drafts"], dev), out, g_am, g_t1, g_en, res, ws, *TYPICAL)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    for layer in range(layers):
+        q, k, v = c["q"][layer], c["k"][layer], c["v"][layer]
+        check_attention_fuzz(got[layer], oracle.tree_attention(q, k, v, L, parent),
+                             oracle.tree_attention(q, k, abs_bits(v), L, parent), f"seed {seed} layer {layer}")
+    assert np.array_equal(g_am.cpu().numpy(), c["am"])
+    assert np.abs(g_t1.cpu().numpy() - c["t1"]).max() <= STAT_TOL
+    assert np.abs(g_en.cpu().numpy() - c["en"]).max() <= STAT_TOL
+    k, path, bonus = oracle.typical_accept(c["parent"], c["drafts"], c["logits"], *TYPICAL)
+    r = tv.parse_result(res)
+    assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (k, path, bonus, L + k, 0)
+    assert np.array_equal(bits(kd), oracle.kv_compact(c["k"], L, path))
+    assert np.array_equal(bits(vd), oracle.kv_compact(c["v"], L, path))
     b.close()
