@@ -458,7 +458,8 @@ def verify_step_sampled(bank: Bank, bank_id: int, kv: KvCache, q, hidden, lm_hea
 
 def make_policy(kind: int, feature: int, bank_ids, a: float = 0.0, b: float = 0.0, edges=(), trace=None,
                 n_heads: int = 0, node_stride: int = 0) -> TbPolicy:
-    """tb_policy; `trace` is a device float tensor (kept alive by the caller)."""
+    """tb_policy; `trace` is a device float tensor, which the returned policy
+    keeps alive (the library holds only its address)."""
     pol = TbPolicy()
     pol.kind, pol.feature, pol.n_rungs = kind, feature, len(bank_ids)
     for i, x in enumerate(bank_ids):
@@ -468,6 +469,7 @@ def make_policy(kind: int, feature: int, bank_ids, a: float = 0.0, b: float = 0.
         pol.edges[i] = float(x)
     if trace is not None:
         pol.trace = _ptr(trace)
+        pol._trace_ref = trace
         pol.n_trace = trace.numel() // max(1, n_heads) if feature == TB_FEATURE_PATH_VALUE else trace.numel()
     pol.n_heads = n_heads
     pol.node_stride = node_stride
@@ -493,7 +495,7 @@ def parse_state(st) -> dict:
 
 def verify_step_scheduled(bank: Bank, policy: TbPolicy, state, kv: KvCache, q, hidden, lm_head, drafts, attn_out,
                           argmax, top1, entropy, result, ws, flags: int = 0, stream=None):
-    """q / attn_out [n_layers][N_max][Hq][128]; hidden [N_max][d_model]; drafts [n_rungs][N_max]."""
+    """q / attn_out [n_layers][N_max][Hq][head_dim]; hidden [N_max][d_model]; drafts [n_rungs][N_max]."""
     c = kv.as_c()
     _check(load().verify_step_scheduled(bank.handle, ctypes.byref(policy), _ptr(state), ctypes.byref(c), _ptr(q),
                                         q.shape[2], _ptr(hidden), _ptr(lm_head), hidden.shape[1], lm_head.shape[0],

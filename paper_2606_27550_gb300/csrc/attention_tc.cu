@@ -139,6 +139,16 @@ __device__ __forceinline__ int seq_at(const TcParams &p, long long t, int b)
     }
 }
 
+// CTAs the tile space is split over.  The host plans at most one CTA per
+// tile; scheduled mode plans on the device with a grid of one CTA per SM, and
+// a step with fewer tiles than that splits them over its first `total` CTAs
+// only (the others get nothing), so that no CTA range inside the split is
+// empty: the split merge combines the partials of consecutive CTAs.
+__device__ __forceinline__ int tc_split_ctas(const TcParams &p, long long total)
+{
+    return (p.sched && total < p.P) ? (int)(total > 0 ? total : 1) : p.P;
+}
+
 // First flattened tile of CTA c's range (the ranges split the tile space
 // evenly).  The quotients take 32-bit divisions whenever the operands fit.
 __device__ __forceinline__ long long tc_seg_begin(long long total, int P, int c)
@@ -218,7 +228,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) k1_tree_attention_tc(const __gr
         seqs = &s_seq;
         total = s_total;
     }
-    const long long t0 = tc_seg_begin(total, p.P, c), t1 = tc_seg_begin(total, p.P, c + 1);
+    const int P = tc_split_ctas(p, total);
+    const long long t0 = c < P ? tc_seg_begin(total, P, c) : total;
+    const long long t1 = c < P ? tc_seg_begin(total, P, c + 1) : total;
     const long long n_tiles = t1 - t0;
 
     if (threadIdx.x == 0) {
@@ -731,8 +743,11 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
         seqs = &s_seq;
         total = s_total;
     }
+    const int P = tc_split_ctas(p, total);
     const int cb = blockIdx.x + 1;  // CTA range starting at tile t_c
-    const long long tc = tc_seg_begin(total, p.P, cb);
+    if (cb >= P)
+        return;
+    const long long tc = tc_seg_begin(total, P, cb);
     int b = 0;
     if constexpr (kBatched) {
         while (b + 1 < p.n_seq && tc >= seqs[b + 1].tile_base)
@@ -743,7 +758,7 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
     const long long u_first = sq.tile_base + (long long)u * sq.T, u_last = u_first + sq.T;
     if (tc == u_first)
         return;  // the boundary is a unit boundary
-    const int c_lo = tc_cta_of(total, p.P, u_first), c_hi = tc_cta_of(total, p.P, u_last - 1);
+    const int c_lo = tc_cta_of(total, P, u_first), c_hi = tc_cta_of(total, P, u_last - 1);
     if (cb != c_lo + 1)
         return;  // an earlier boundary inside this unit handles it
     const int nseg = c_hi - c_lo + 1;
@@ -756,7 +771,7 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
         return;
     {
         const int grow = rb * 128 + r;
-        if (!in_bounds(c_lo >= 0 && c_hi < p.P && layer_rel < p.n_layers && grow / p.group < sq.nstride &&
+        if (!in_bounds(c_lo >= 0 && c_hi < P && layer_rel < p.n_layers && grow / p.group < sq.nstride &&
                            head * p.group + grow % p.group < p.Hq,
                        p.status))
             return;
@@ -766,7 +781,7 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
     for (int j0 = 0; j0 < nseg; j0 += 32) {
         const int cc = c_lo + j0 + lane;
         if (j0 + lane < nseg) {
-            const float *sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, p.P, cc) >= u_first ? 0 : 1)) * kSlot;
+            const float *sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, P, cc) >= u_first ? 0 : 1)) * kSlot;
             M = fmaxf(M, __ldcg(sl + 128 * kD + r));
         }
     }
@@ -780,7 +795,7 @@ __global__ void __launch_bounds__(256, 4) k1_merge_split(const __grid_constant__
         const float *sl = p.part;
         float w = 0.f;
         if (j0 + lane < nseg) {
-            sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, p.P, cc) >= u_first ? 0 : 1)) * kSlot;
+            sl = p.part + ((size_t)cc * 2 + (tc_seg_begin(total, P, cc) >= u_first ? 0 : 1)) * kSlot;
             const float ms = __ldcg(sl + 128 * kD + r);
             w = (ms == -INFINITY) ? 0.f : ex2_approx(ms - M);
             lsum += w * __ldcg(sl + 128 * kD + 128 + r);

@@ -98,3 +98,16 @@ def test_every_wrapper_marshals_its_declared_arguments(fake):
     # the kv struct carries the rotary base
     c = fake.tree_attention.calls[0][2]._obj
     assert c.rope_theta == pytest.approx(10000.0) and c.L == 4 and c.L_cap == 16
+
+
+def test_policy_keeps_its_trace_alive():
+    """The library holds only the trace's address: the policy object keeps the
+    tensor alive, so a trace passed inline is not freed under it."""
+    import gc
+
+    t = torch.arange(4, dtype=torch.float32)
+    ptr = t.data_ptr()
+    pol = tv.make_policy(tv.TB_POLICY_BINARY, tv.TB_FEATURE_TRACE, [0, 1], a=1.0, b=0.5, trace=t)
+    del t
+    gc.collect()
+    assert pol.trace == ptr and pol._trace_ref.data_ptr() == ptr and pol.n_trace == 4

@@ -87,11 +87,9 @@ def _trace(steps, seed=3):
     return np.round(g.uniform(0.5, 3.5, steps) * 64).astype(np.float32) / np.float32(64)
 
 
-@pytest.mark.parametrize("d_head", [128, 64])
-def test_scheduled_loop_matches_oracle(dev, d_head):
-    steps = 24
-    lp = Loop(dev, steps, L0=100, d_head=d_head)
-    trace = _trace(steps)
+def _run_loop(dev, steps, L0, d_head, trace, seed=0):
+    """The loop against the oracle, step by step; returns the rungs visited."""
+    lp = Loop(dev, steps, L0=L0, seed=seed, d_head=d_head)
     tr_d = to_dev(trace, dev)
     pol = tv.make_policy(tv.TB_POLICY_HYSTERETIC_LADDER, tv.TB_FEATURE_TRACE, lp.ids, a=1.5, b=2.5, trace=tr_d,
                          node_stride=N_MAX)
@@ -123,8 +121,26 @@ def test_scheduled_loop_matches_oracle(dev, d_head):
         st = tv.parse_state(state)
         assert st == {"rung": nxt, "L": L + ka, "step": t + 1, "feature": float(trace[t]), "accept_len": ka}, t
         rung, L = nxt, L + ka
-    assert len(seen) >= 3  # the ladder moved across several trees
     lp.bank.close()
+    return seen
+
+
+@pytest.mark.parametrize("d_head", [128, 64])
+def test_scheduled_loop_matches_oracle(dev, d_head):
+    seen = _run_loop(dev, 24, 100, d_head, _trace(24))
+    assert len(seen) >= 3  # the ladder moved across several trees
+
+
+def test_scheduled_loop_few_tiles_per_step(dev):
+    """Steps with far fewer key tiles than CTAs (2 layers x 2 kv heads x 12
+    tiles against one CTA per SM) whose tree, and so the split of the tiles,
+    changes from step to step: the split merge must combine only partials the
+    step itself wrote (stale partials of earlier steps sit in the same
+    workspace slots)."""
+    g = np.random.default_rng(5)
+    trace = (np.round(g.uniform(0.5, 3.5, 12) * 64) / 64).astype(np.float32)
+    seen = _run_loop(dev, 12, 1500, 128, trace, seed=2048)
+    assert len(seen) >= 4
 
 
 def test_scheduled_graph_replay_matches_eager(dev):
