@@ -4,7 +4,8 @@ at L + depth(i)) against the fp64 oracle, through the C ABI.
 Attention: max-abs <= 1e-2 and mean-abs <= 1e-3 as everywhere.  The rotated
 tree keys are stored back into the bf16 cache: they may differ from the
 oracle's (fp64 rotation, rounded once) by one bf16 ulp where the float
-rotation lands next to a rounding boundary; everything else in the cache
+rotation lands next to a rounding boundary, or by a tiny absolute amount
+where the rotation cancels (see ROT_ABS_TOL); everything else in the cache
 (prefix keys, all values) must be byte-identical, and acceptance, path and
 bonus token exact.
 """
@@ -45,11 +46,25 @@ def _ordered(b):
     return np.where(x & 0x8000, 0x8000 - x, x)
 
 
+def _bf16_value(b):
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+# Where the rotation cancels (x1 c - x2 s far below the inputs' magnitude) the
+# absolute error of the fp32 rotation, a few roundings of 2^-24 of inputs that
+# are N(0, 1) bf16 (|x1| + |x2| below 10), spans several bf16 ulps of the small
+# result: such elements may differ by up to 2^-18 in value.
+ROT_ABS_TOL = 2.0 ** -18
+
+
 def check_rotated_keys(got, ref, what="rotated keys"):
     diff = np.abs(_ordered(got) - _ordered(ref))
-    assert diff.max() <= 1, f"{what}: {diff.max()} bf16 ulps apart"
+    far = diff > 1
+    if far.any():
+        gap = np.abs(_bf16_value(got[far]) - _bf16_value(ref[far]))
+        assert gap.max() <= ROT_ABS_TOL, f"{what}: {diff.max()} bf16 ulps and {gap.max():.2e} apart"
     frac = float((diff > 0).mean())
-    assert frac < 0.01, f"{what}: {frac:.4f} of the elements one ulp apart"
+    assert frac < 0.01, f"{what}: {frac:.4f} of the elements differ"
     return frac
 
 
