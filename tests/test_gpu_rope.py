@@ -13,7 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
-from helpers import STAT_TOL, bits, check_attention, gap_filtered_hidden, to_dev
+from helpers import STAT_TOL, abs_bits, bits, check_attention, check_attention_fuzz, gap_filtered_hidden, to_dev
 from paper_2606_27550_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -253,3 +253,42 @@ def test_rope_argument_errors(dev, bank):
         with pytest.raises(tv.TreeVerifyError) as e:
             tv.tree_attention(bank, bid, tv.KvCache(k, k.clone(), 4, rope_theta=theta), q, torch.empty_like(q), ws)
         assert e.value.status == tv.TB_EINVAL
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_rope_attention(dev, seed):
+    """Random shapes with the rotary embedding: random trees, prefix lengths
+    0-16000, head_dim 64 and 128, GQA groups, one or two layers; attention
+    within the derived bound of the fuzz tests (short prefixes give outputs
+    of order 1), rotated keys as above, prefix keys and values untouched."""
+    g = synth.rng(3300 + seed)
+    n = int(g.integers(1, 65))
+    parent = np.sort(synth.random_tree(g, n))
+    parent[0] = -1
+    d = int(g.choice([64, 128]))
+    Hkv = int(g.choice([1, 2, 4]))
+    group = int(g.choice([1, 2, 4]))
+    while n * group > 256:
+        group //= 2
+    Hq = Hkv * group
+    L = int(g.choice([0, 5, 130, 700, 3000, 16000]))
+    layers = int(g.integers(1, 3))
+    b = tv.Bank(4, 0)
+    bid, _ = b.add(parent)
+    k, v = synth.gen_kv(seed, layers, Hkv, L + n + 4, d, L + n)
+    q = synth.gen_q(seed, layers, n, Hq, d)
+    kd, vd = to_dev(k, dev), to_dev(v, dev)
+    out = torch.empty((layers, n, Hq, d), dtype=torch.bfloat16, device=dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(n, layers, Hkv, Hq, d, 1, 0), dev)
+    tv.tree_attention(b, bid, tv.KvCache(kd, vd, L, rope_theta=THETA), to_dev(q, dev), out, ws)
+    torch.cuda.synchronize()
+    got_k = bits(kd)
+    o = out.float().cpu().numpy()
+    for layer in range(layers):
+        ref, k_rot = oracle.tree_attention_rope(q[layer], k[layer], v[layer], L, parent, THETA)
+        ref_a, _ = oracle.tree_attention_rope(q[layer], k[layer], abs_bits(v[layer]), L, parent, THETA)
+        check_attention_fuzz(o[layer], ref, ref_a, f"seed {seed} layer {layer} (n={n} L={L} d={d} Hq={Hq} Hkv={Hkv})")
+        check_rotated_keys(got_k[layer][:, L:L + n], k_rot, f"seed {seed} layer {layer}")
+        assert np.array_equal(got_k[layer][:, :L], k[layer][:, :L])
+    assert np.array_equal(bits(vd), v)
+    b.close()

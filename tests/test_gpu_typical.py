@@ -371,3 +371,56 @@ def test_random_typical_step(dev, seed):
     assert np.array_equal(bits(kd), oracle.kv_compact(c["k"], L, path))
     assert np.array_equal(bits(vd), oracle.kv_compact(c["v"], L, path))
     b.close()
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_random_batched_typical_step(dev, seed):
+    """Random ragged batches in typical mode: 1-8 sequences with random trees
+    and prefix lengths, head_dim 64 and 128, GQA groups, ragged vocabularies."""
+    g = synth.rng(4400 + seed)
+    d = int(g.choice([64, 128]))
+    Hkv, group = int(g.choice([1, 2])), int(g.choice([1, 2, 4]))
+    Hq = Hkv * group
+    D, V = int(g.choice([64, 256])), int(g.choice([129, 1000, 3001]))
+    batch = int(g.integers(1, 9))
+    b = tv.Bank(16, 0)
+    W = synth.gen_lm_head(seed, V, D)
+    parents = []
+    for i in range(batch):
+        n = int(g.integers(1, 65))
+        while n * group > 256:
+            n //= 2
+        p = np.sort(synth.random_tree(g, max(n, 1)))
+        p[0] = -1
+        parents.append(p)
+    rows = sum(len(p) for p in parents)
+    hidden, am, t1, en, logits = gap_filtered_hidden(seed + 50, rows, W, want_logits=True)
+    seqs, host, r0 = [], [], 0
+    for i, parent in enumerate(parents):
+        N = len(parent)
+        L = int(g.choice([0, 7, 130, 900]))
+        drafts = typical_drafts(600 + 10 * seed + i, parent, logits[r0:r0 + N], *TYPICAL)
+        k, v = synth.gen_kv(900 + 10 * seed + i, 1, Hkv, L + N + 2, d, L + N)
+        q = synth.gen_q(900 + 10 * seed + i, 1, N, Hq, d)
+        bid, _ = b.add(parent)
+        s = tv.Seq(bid, tv.KvCache(to_dev(k, dev), to_dev(v, dev), L), to_dev(q, dev), to_dev(drafts, dev),
+                   torch.empty((1, N, Hq, d), dtype=torch.bfloat16, device=dev), tv.make_result(dev))
+        seqs.append(s)
+        host.append((parent, L, k, v, q, drafts, r0))
+        r0 += N
+    g_am = torch.empty(rows, dtype=torch.int32, device=dev)
+    g_t1, g_en = _f32(rows, dev), _f32(rows, dev)
+    ws = tv.make_workspace(tv.tb_workspace_size(rows, 1, Hkv, Hq, d, V, 0), dev)
+    tv.verify_step_batched_typical(b, seqs, to_dev(hidden, dev), to_dev(W, dev), g_am, g_t1, g_en, ws, *TYPICAL)
+    torch.cuda.synchronize()
+    assert np.array_equal(g_am.cpu().numpy(), am)
+    assert np.abs(g_en.cpu().numpy() - en).max() <= STAT_TOL
+    for s, (parent, L, k, v, q, drafts, r0) in zip(seqs, host):
+        N = len(parent)
+        r = tv.parse_result(s.result)
+        ka, path, bonus = oracle.typical_accept(parent, drafts, logits[r0:r0 + N], *TYPICAL)
+        assert (r["accept_len"], r["path"], r["bonus_token"], r["new_L"], r["status"]) == (ka, path, bonus, L + ka, 0)
+        check_attention_fuzz(s.attn_out[0].float().cpu().numpy(), oracle.tree_attention(q[0], k[0], v[0], L, parent),
+                             oracle.tree_attention(q[0], k[0], abs_bits(v[0]), L, parent), f"seed {seed}")
+        assert np.array_equal(bits(s.kv.k), oracle.kv_compact(k, L, path))
+    b.close()
