@@ -111,3 +111,19 @@ def test_policy_keeps_its_trace_alive():
     del t
     gc.collect()
     assert pol.trace == ptr and pol._trace_ref.data_ptr() == ptr and pol.n_trace == 4
+
+
+def test_kv_compact_passes_the_result_fields(fake):
+    """kv_compact(kv, result) hands the C call the result block's path and
+    accept_len fields: path 16 bytes in (after accept_len, bonus_token, new_L,
+    status), accept_len at the start."""
+    t = lambda *shape: torch.zeros(shape, dtype=torch.bfloat16)  # noqa: E731
+    kv = tv.KvCache(t(1, 2, 16, 64), t(1, 2, 16, 64), 4)
+    res = torch.zeros(tv.RESULT_INTS, dtype=torch.int32)
+    tv.kv_compact(kv, res, stream=0)
+    _, path, accept_len, _ = fake.kv_compact.calls[-1]
+    assert path == res.data_ptr() + 16 and accept_len == res.data_ptr()
+    p, n = torch.zeros(3, dtype=torch.int32), torch.zeros(1, dtype=torch.int32)
+    tv.kv_compact_path(kv, p, n, stream=0)
+    _, path, accept_len, _ = fake.kv_compact.calls[-1]
+    assert path == p.data_ptr() and accept_len == n.data_ptr()
